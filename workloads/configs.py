@@ -1,0 +1,115 @@
+"""The five seeded synthetic workloads (grammar, vocabulary, batch of prefixes, logits).
+
+1. tiny arithmetic grammar, V=512, B=8, prefixes of 1-64 bytes, fp32 logits ~N(0,1)
+2. JSON (RFC 8259), V=32,000, B=64, prefixes up to 512 bytes, bf16 logits ~N(0,2)
+3. schema-conformant JSON, V=128,256, B=256, prefixes up to 1024 bytes, bf16 logits ~N(0,2)
+4. C-like language, V=151,936, B=256, prefixes up to 2048 bytes, bf16 logits ~N(0,2)
+5. C-like language, V=262,144, B=1024, prefixes of 64-4096 bytes biased to deep nesting,
+   bf16 logits ~N(0,2), 32 decode steps
+
+N(0,2) is read as variance 2 (sigma = sqrt 2).  The paper's datasets, JSON
+schemas and tokenizers are not available; these stand in for them.
+"""
+from __future__ import annotations
+
+import functools
+import math
+from dataclasses import dataclass
+
+import numpy as np
+
+from . import grammars
+from .sample import TrieTokenizer, VocabSpec, build_prefixes, build_vocab
+
+
+@dataclass(frozen=True)
+class WorkloadSpec:
+    id: int
+    name: str
+    B: int
+    V: int
+    dtype: str               # "f32" or "bf16"
+    sigma: float
+    prefix_min: int
+    prefix_max: int
+    vocab_max_len: int
+    frac_grammar: float
+    nest_bias: float = 1.0
+    max_depth: int = 40
+    decode_steps: int = 1
+
+
+SPECS = {
+    1: WorkloadSpec(1, "arith_v512_b8", 8, 512, "f32", 1.0, 1, 64, 6, 400 / 413),
+    2: WorkloadSpec(2, "json_v32000_b64", 64, 32000, "bf16", math.sqrt(2), 1, 512, 16, 0.4),
+    3: WorkloadSpec(3, "schema_json_v128256_b256", 256, 128256, "bf16", math.sqrt(2), 1, 1024, 24,
+                    0.5),
+    4: WorkloadSpec(4, "c_like_v151936_b256", 256, 151936, "bf16", math.sqrt(2), 1, 2048, 32, 0.7),
+    5: WorkloadSpec(5, "c_like_v262144_b1024", 1024, 262144, "bf16", math.sqrt(2), 64, 4096, 32, 0.7,
+                    nest_bias=4.0, max_depth=500, decode_steps=32),
+}
+
+
+def grammar_spec(cfg: int) -> grammars.GrammarSpec:
+    if cfg == 1:
+        return grammars.arithmetic()
+    if cfg == 2:
+        return grammars.json_grammar()
+    if cfg == 3:
+        return grammars.schema_json(seed=int(np.random.default_rng([3, 1]).integers(0, 2**31)))
+    return grammars.c_like()
+
+
+@dataclass
+class Workload:
+    spec: WorkloadSpec
+    grammar_text: str
+    vocab: list[bytes]
+    eos_id: int
+    prefixes: list[bytes]
+    prefix_ids: list[list[int]]
+
+    @property
+    def B(self):
+        return self.spec.B
+
+    @property
+    def V(self):
+        return self.spec.V
+
+    def vocab_arrays(self):
+        """(blob uint8, offsets int64[V+1]) of the vocabulary."""
+        offs = np.zeros(len(self.vocab) + 1, dtype=np.int64)
+        offs[1:] = np.cumsum([len(t) for t in self.vocab])
+        blob = np.frombuffer(b"".join(self.vocab), dtype=np.uint8).copy()
+        return blob, offs
+
+    def token_matrix(self):
+        """Prefix token ids as a [B][T] int32 matrix padded with -1 (no-op)."""
+        T = max((len(p) for p in self.prefix_ids), default=0)
+        m = np.full((self.B, max(T, 1)), -1, dtype=np.int32)
+        for b, ids in enumerate(self.prefix_ids):
+            m[b, :len(ids)] = ids
+        return m
+
+    def logits(self, step: int = 0):
+        """Seeded CPU logits [B][V] (torch), fp32 or bf16."""
+        import torch
+        g = torch.Generator().manual_seed(1000 * self.spec.id + 4 + 7919 * step)
+        x = torch.randn(self.B, self.V, generator=g) * self.spec.sigma
+        return x if self.spec.dtype == "f32" else x.to(torch.bfloat16)
+
+
+@functools.lru_cache(maxsize=8)
+def load(cfg: int, batch: int | None = None) -> Workload:
+    """Build workload ``cfg`` (optionally with only the first ``batch`` rows)."""
+    s = SPECS[cfg]
+    g = grammar_spec(cfg)
+    vocab = build_vocab(g, VocabSpec(s.V, s.vocab_max_len, s.frac_grammar), [cfg, 2])
+    B = s.B if batch is None else batch
+    prefixes = build_prefixes(g, B, s.prefix_min, s.prefix_max, [cfg, 3],
+                              max_depth=s.max_depth, nest_bias=s.nest_bias)
+    tok = TrieTokenizer(vocab)
+    ids = [tok.encode(p) for p in prefixes]
+    spec = s if batch is None else WorkloadSpec(**{**s.__dict__, "B": B})
+    return Workload(spec, g.text(), vocab, len(vocab) - 1, prefixes, ids)
