@@ -1,0 +1,375 @@
+"""Benchmark: masked decode steps on the 1024 x 262,144 C-like workload.
+
+One step = one pass of the whole per-step path over the batch:
+  psc_fill_apply     classify every row's parser stack (classifier DFA walk) and
+                     apply its precomputed mask to the bf16 logits in place, also
+                     writing the packed bitmask [B][V/32]
+  psc_argmax_masked  greedy choice among the allowed tokens
+  psc_advance        lex + parse the chosen tokens on the device-resident stacks
+
+Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+For N > 1 launch with torch.distributed.run: every rank runs an independent
+replica (the rows of different sequences are independent; no collective on the
+data path) and the step rate is summed over ranks (weak scaling).
+The reference arm (--impl reference) times the CPU oracle on the host cores.
+"""
+from __future__ import annotations
+
+import argparse
+import ctypes
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+WORKLOAD = 5
+METRIC = "masked decode steps/s and µs/step at batch×vocab; HBM GB/s vs GB300 peak"
+UNIT = "steps/s"
+PROFILE_FILE = os.path.join(ROOT, "profiles", "fused_fill_apply_c5_traffic.txt")
+
+
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    return 6800.0, "fallback"
+
+
+# ------------------------------------------------------------ clock sampling
+class ClockSampler:
+    """Samples SM clock and clock-event reasons through NVML (read-only) while
+    the timed region runs; falls back to nvidia-smi."""
+
+    REASONS = {0x4: "sw_power_cap", 0x8: "hw_slowdown", 0x20: "sw_thermal_slowdown",
+               0x40: "hw_thermal_slowdown", 0x80: "hw_power_brake_slowdown"}
+
+    def __init__(self, index: int = 0, period_s: float = 0.002):
+        self.samples = []
+        self.reasons = set()
+        self.max_mhz = None
+        self.period = period_s
+        self._stop = threading.Event()
+        self._nvml = None
+        self._proc = None
+        try:
+            nv = ctypes.CDLL("libnvidia-ml.so.1")
+            if nv.nvmlInit_v2() == 0:
+                h = ctypes.c_void_p()
+                if nv.nvmlDeviceGetHandleByIndex_v2(index, ctypes.byref(h)) == 0:
+                    self._nvml, self._h = nv, h
+                    mx = ctypes.c_uint()
+                    if nv.nvmlDeviceGetMaxClockInfo(h, 1, ctypes.byref(mx)) == 0:
+                        self.max_mhz = mx.value
+        except OSError:
+            self._nvml = None
+
+    def _loop(self):
+        nv, h = self._nvml, self._h
+        clk, rs = ctypes.c_uint(), ctypes.c_ulonglong()
+        get_r = getattr(nv, "nvmlDeviceGetCurrentClocksEventReasons", None) or \
+            nv.nvmlDeviceGetCurrentClocksThrottleReasons
+        while not self._stop.is_set():
+            if nv.nvmlDeviceGetClockInfo(h, 1, ctypes.byref(clk)) == 0:
+                self.samples.append(clk.value)
+            if get_r(h, ctypes.byref(rs)) == 0:
+                for bit, name in self.REASONS.items():
+                    if rs.value & bit:
+                        self.reasons.add(name)
+            time.sleep(self.period)
+
+    def __enter__(self):
+        if self._nvml is not None:
+            self._t = threading.Thread(target=self._loop, daemon=True)
+            self._t.start()
+        else:
+            try:
+                self._proc = subprocess.Popen(
+                    ["nvidia-smi", "--query-gpu=clocks.sm,clocks.max.sm,clocks_event_reasons.active",
+                     "--format=csv,noheader,nounits", "-lms", "50"],
+                    stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            except OSError:
+                self._proc = None
+        return self
+
+    def __exit__(self, *a):
+        self._stop.set()
+        if self._nvml is not None:
+            self._t.join()
+        elif self._proc is not None:
+            self._proc.terminate()
+            out = self._proc.communicate(timeout=5)[0]
+            for line in out.splitlines():
+                parts = [p.strip() for p in line.split(",")]
+                try:
+                    self.samples.append(int(parts[0]))
+                    self.max_mhz = int(parts[1])
+                    mask = int(parts[2], 16)
+                    for bit, name in self.REASONS.items():
+                        if mask & bit:
+                            self.reasons.add(name)
+                except (ValueError, IndexError):
+                    pass
+
+    def summary(self):
+        return {"sm_mhz": statistics.median(self.samples) if self.samples else None,
+                "sm_max_mhz": self.max_mhz, "reasons": sorted(self.reasons),
+                "samples": len(self.samples)}
+
+
+# ---------------------------------------------------------------- oracle arm
+def oracle_rate(w, budget_s: float, threads: int):
+    """Time the CPU oracle (as it stands) on whole rows of the workload until
+    about budget_s seconds of wall time; returns (steps/s, rows, seconds)."""
+    from oracle import Oracle, Vocab
+    o = Oracle(w.grammar_text)
+    voc = Vocab.from_list(w.vocab, w.eos_id)
+    cfgs = []
+    rows = 0
+    spent = 0.0
+    n = 1
+    while spent < budget_s and rows < w.B:
+        batch = []
+        for b in range(rows, min(rows + n, w.B)):
+            oc = o.initial()
+            o.advance_tokens(oc, voc, w.prefix_ids[b])
+            batch.append(oc)
+        t0 = time.perf_counter()
+        o.masks(batch, voc, threads=threads)
+        spent += time.perf_counter() - t0
+        rows += len(batch)
+        cfgs.extend(batch)
+        n *= 2
+    return rows / (spent * w.B), rows, spent
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    from workloads import configs
+    w = configs.load(WORKLOAD)
+    threads = os.cpu_count() or 1
+    from oracle import Oracle, Vocab
+    o = Oracle(w.grammar_text)
+    voc = Vocab.from_list(w.vocab, w.eos_id)
+    # each step: the oracle's masks for one row (all V tokens), scaled to B rows
+    cfgs = []
+    for b in range(args.warmup + args.steps):
+        oc = o.initial()
+        o.advance_tokens(oc, voc, w.prefix_ids[b % w.B])
+        cfgs.append(oc)
+    for i in range(args.warmup):
+        o.masks([cfgs[i]], voc, threads=threads)
+    t0 = time.perf_counter()
+    for i in range(args.steps):
+        o.masks([cfgs[args.warmup + i]], voc, threads=threads)
+    dt = time.perf_counter() - t0
+    rows_per_s = args.steps / dt
+    value = rows_per_s / w.B
+    sample = f"{args.steps} steps, each the oracle's masks for 1 of {w.B} rows x {w.V} tokens, scaled to {w.B} rows"
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000.0 / value,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u32",
+        "data": "synthetic", "config": config_block(w, args.gpus),
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle", "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }))
+
+
+def config_block(w, n):
+    return {"workload": f"config 5: C-like grammar, vocab {w.V}, batch {w.B}, bf16 logits ~N(0,2), "
+                        "decode steps fill_apply+argmax+advance",
+            "batch": w.B, "vocab": w.V, "logit_dtype": "bf16", "grammar": "synthetic C-like (150 rules)",
+            "parallelism": f"replicas x{n}", "l2": "inputs larger than L2 (512 MiB logits per step)"}
+
+
+def traffic_from_profile(kernel_src_hash: str):
+    """Per-launch DRAM bytes of the fused kernel from the committed ncu summary,
+    if it was taken on the current kernel source."""
+    if not os.path.exists(PROFILE_FILE):
+        return None
+    vals = {}
+    with open(PROFILE_FILE) as f:
+        for line in f:
+            if ":" in line:
+                k, v = line.split(":", 1)
+                vals[k.strip()] = v.strip()
+    if vals.get("kernel_source_sha256") != kernel_src_hash:
+        return None
+    try:
+        return int(vals["dram_bytes_per_launch"])
+    except (KeyError, ValueError):
+        return None
+
+
+# ------------------------------------------------------------------ main arm
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=32)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="gb300")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+
+    import torch
+    import torch.distributed as dist
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+
+    from paper_2608_03065_gb300 import build, psc
+    from workloads import configs
+    build.build()
+    w = configs.load(WORKLOAD)
+    B, V = w.B, w.V
+    t0 = time.time()
+    h = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id)
+    compile_s = time.time() - t0
+    info = h.info()
+    st = psc.psc_state_init(h, B, 256)
+    tm = torch.from_numpy(w.token_matrix()).to(dev)
+    for j in range(tm.shape[1]):
+        psc.psc_advance(h, st, tm[:, j].contiguous())
+    torch.cuda.synchronize()
+
+    K, Wm = args.steps, args.warmup
+    n_buf = K + Wm
+    gen = torch.Generator(device=dev).manual_seed(1000 * WORKLOAD + 4 + rank)
+    sigma = w.spec.sigma
+    bufs = [(torch.randn(B, V, generator=gen, device=dev) * sigma).to(torch.bfloat16) for _ in range(n_buf)]
+    bitmask = torch.empty(B, h.W, dtype=torch.int32, device=dev)
+    tok = torch.empty(B, dtype=torch.int32, device=dev)
+    stat = torch.empty(B, dtype=torch.int32, device=dev)
+    stream = torch.cuda.current_stream()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+
+    def step(i, timed=None):
+        x = bufs[i]
+        if timed is not None:
+            ev[timed][0].record(stream)
+        psc.psc_fill_apply(h, st, x, bitmask, stream=stream)
+        if timed is not None:
+            ev[timed][1].record(stream)
+        psc.psc_argmax_masked(h, st, x, tok, stream=stream)
+        psc.psc_advance(h, st, tok, stat, stream=stream)
+
+    for i in range(Wm):
+        step(i)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(index=local) as clocks:
+        torch.cuda.nvtx.range_push("psc_steps")
+        t_start.record(stream)
+        for i in range(K):
+            step(Wm + i, timed=i)
+        t_end.record(stream)
+        torch.cuda.synchronize()
+        torch.cuda.nvtx.range_pop()
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    elapsed_ms = t_start.elapsed_time(t_end)
+    fused_ms = [a.elapsed_time(b) for a, b in ev]
+    if world > 1:
+        tt = torch.tensor([elapsed_ms], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        elapsed_ms = float(tt.item())
+    ms_per_step = elapsed_ms / K
+    value = world * K / (elapsed_ms / 1000.0)
+
+    # end to end through the public API with host buffers: H2D of each step's
+    # logits from pinned memory, the step, D2H of the chosen tokens
+    n_host = 2
+    host = [torch.empty(B, V, dtype=torch.bfloat16, pin_memory=True) for _ in range(n_host)]
+    for k in range(n_host):
+        host[k].copy_(bufs[k])
+    tok_host = torch.empty(B, dtype=torch.int32, pin_memory=True)
+    dbuf = bufs[0]
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for i in range(K):
+        dbuf.copy_(host[i % n_host], non_blocking=True)
+        psc.psc_fill_apply(h, st, dbuf, bitmask, stream=stream)
+        psc.psc_argmax_masked(h, st, dbuf, tok, stream=stream)
+        psc.psc_advance(h, st, tok, stat, stream=stream)
+        tok_host.copy_(tok, non_blocking=True)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = e0.elapsed_time(e1)
+    if world > 1:
+        tt = torch.tensor([e2e_ms], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        e2e_ms = float(tt.item())
+    e2e_value = world * K / (e2e_ms / 1000.0)
+
+    if rank != 0:
+        if world > 1:
+            dist.destroy_process_group()
+        return
+
+    peak, peak_kind = measured_peaks()
+    alg_bytes = B * V // 8 + 2 * B * V * 2
+    fused_avg_ms = sum(fused_ms) / len(fused_ms)
+    achieved = alg_bytes / (fused_avg_ms / 1000.0) / 1e9
+    src = open(os.path.join(ROOT, "paper_2608_03065_gb300", "csrc", "psc_capi.cu"), "rb").read()
+    traffic = traffic_from_profile(hashlib.sha256(src).hexdigest())
+
+    cpu = None
+    if world == 1 and not args.no_cpu_baseline:
+        threads = os.cpu_count() or 1
+        rate, rows, secs = oracle_rate(w, 10.0, threads)
+        cpu = {"value": rate, "unit": UNIT, "cores": threads, "kind": "oracle",
+               "sample": f"oracle masks of the first {rows} of {w.B} rows x all {V} tokens "
+                         f"({secs:.1f} s wall on {threads} threads), scaled to one {w.B}-row step"}
+
+    out = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K, "warmup": Wm,
+        "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "u32", "data": "synthetic", "config": config_block(w, world),
+        "us_per_step": ms_per_step * 1000.0,
+        "fused_fill_apply_us": fused_avg_ms * 1000.0,
+        "fused_fill_apply_hbm_gbs": achieved,
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                     "frac": achieved / peak, "traffic": traffic,
+                     "kernel": "psc_fill_apply (classify walk + fused mask apply + bitmask copy)",
+                     "algorithmic_bytes": alg_bytes, "peak_kind": peak_kind},
+        "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": B * V * 2,
+                "d2h_bytes_per_step": B * 4},
+        "gpu_launches": 4 * K,
+        "clocks": clocks.summary(),
+        "cpu_baseline": cpu,
+        "tables": {"classifier_states": info.n_classifier_states, "masks": info.n_masks,
+                   "classifier_bytes": info.classifier_bytes, "mask_bytes": info.mask_bytes,
+                   "compile_seconds": compile_s},
+    }
+    print(json.dumps(out))
+    if world > 1:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

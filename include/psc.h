@@ -1,0 +1,201 @@
+/*
+ * psc.h - C ABI of the GB300 PSC library: grammar-constrained decoding masks by
+ * Parser Stack Classification (Li, Dong, Li, Li, "Efficient Grammar-Constrained
+ * Decoding via Parser Stack Classification").
+ *
+ * The library computes, once per decoding step and for a whole batch of
+ * sequences, the vocabulary mask of Eq. (1): the tokens v such that the prefix
+ * followed by v can still be completed to a string of the grammar's language.
+ * Following the paper, the offline step (psc_compile, Algorithm 1) folds every
+ * token's acceptance condition on the parser stack into one classifier DFA over
+ * (lexer state, parser stack read from the top) and precomputes the mask of
+ * every classifier state; the online step (Algorithm 2) walks each sequence's
+ * stack once through that DFA and returns the precomputed mask.  Here the
+ * online step runs in CUDA kernels on the GPU that also applies the mask to
+ * the logits.
+ *
+ * Conventions for every call:
+ *  - Pointers named d_* are device memory owned by the caller (for example the
+ *    data_ptr() of a torch tensor); h_* are host memory owned by the caller.
+ *  - A psc_handle owns its device tables and a psc_states owns its device
+ *    arrays; both are freed only by their *_destroy call.
+ *  - Calls that take a cudaStream_t (passed as void*, NULL = the legacy default
+ *    stream) only enqueue work on that stream and return; they never
+ *    synchronise.  Their return value reports argument and launch errors only.
+ *  - Errors in the data (a token the mask does not allow, a stack that
+ *    overflows its capacity) are per-row statuses written by the kernels;
+ *    kernels never trap and never spin.
+ *  - psc_last_error() returns a thread-local message for the last failing call.
+ *  - Bit v of a packed mask row is bit (v & 31) of 32-bit word (v >> 5)
+ *    (least significant bit first); bits v >= V are zero.
+ */
+#ifndef PSC_H
+#define PSC_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    PSC_OK = 0,
+    PSC_ERR_ARG = 1,              /* bad argument (NULL, size, dtype, stride, host-only handle) */
+    PSC_ERR_GRAMMAR = 2,          /* grammar text cannot be read */
+    PSC_ERR_CONFLICT = 3,         /* grammar is not LALR(1) */
+    PSC_ERR_LEXER_AMBIGUOUS = 4,  /* a lexeme matches an ignored and a kept terminal */
+    PSC_ERR_LIMIT = 5,            /* a size limit of psc_options was exceeded */
+    PSC_ERR_OOM = 6,              /* host or device allocation failed */
+    PSC_ERR_CUDA = 7,             /* a CUDA runtime call failed */
+    PSC_ERR_IO = 8
+} psc_status;
+
+typedef enum { PSC_F32 = 0, PSC_BF16 = 1 } psc_dtype;
+
+/* per-row status words of a psc_states batch */
+enum {
+    PSC_ROW_OK = 0,        /* the row is inside the language's prefixes */
+    PSC_ROW_DONE = 1,      /* the end-of-sequence token was accepted; only it stays allowed */
+    PSC_ROW_REJECTED = 2,  /* a token outside the mask was advanced; nothing is allowed */
+    PSC_ROW_OVERFLOW = 3,  /* the parser stack exceeded the batch capacity; nothing is allowed */
+    PSC_ROW_LIMIT = 4      /* a bounded loop in the advance kernel ran out; nothing is allowed */
+};
+
+typedef struct psc_handle psc_handle;
+typedef struct psc_states psc_states;
+
+typedef struct {
+    int64_t max_states;      /* classifier states before PSC_ERR_LIMIT (0 = 4,000,000) */
+    int64_t max_mask_bytes;  /* host bytes of distinct mask rows before PSC_ERR_LIMIT (0 = 24 GiB) */
+    int32_t threads;         /* host threads for compilation (0 = all cores) */
+    int32_t host_only;       /* 1: build host tables only (no GPU needed; device calls fail) */
+} psc_options;
+
+typedef struct {
+    int32_t V, W;            /* vocabulary size, 32-bit words per mask row */
+    int32_t n_lexer_states;  /* Q: lexer DFA states (the lexing transducer of Section 2.2) */
+    int32_t n_parser_states; /* |Pi|: LALR(1) states = stack symbols (Section 2.4) */
+    int32_t n_terminals;     /* grammar terminals + the end marker */
+    int32_t n_classifier_states;  /* S: non-absorbing states of the classifier DFA (Eq. 9) */
+    int32_t n_masks;         /* distinct precomputed masks A_s (Section 3.5) */
+    int32_t eos_id;
+    int64_t classifier_bytes;  /* device bytes of the classifier tables (cf. Table 7, DFA) */
+    int64_t mask_bytes;        /* device bytes of the mask rows (cf. Table 7, masks) */
+    int64_t states_built;      /* classifier states before minimisation */
+    double compile_seconds;
+} psc_info_t;
+
+/* Offline construction (Algorithm 1, Section 3).  Reads the grammar text (a
+ * Lark-like notation, see the library's documentation), builds the lexer DFA,
+ * the LALR(1) tables, the realizable terminal sequences R_q(v) of every token
+ * from every lexer state (Section 3.1), the stack classifier of Eq. (9) and the
+ * mask of every classifier state, and uploads the tables to the current CUDA
+ * device unless opts->host_only.
+ *   grammar/grammar_len : grammar text (not NUL-terminated necessarily)
+ *   vocab_bytes         : all token byte strings concatenated (host)
+ *   vocab_offsets       : V+1 int64 offsets; token v = vocab_bytes[off[v], off[v+1])
+ *   V, eos_id           : vocabulary size and the end-of-sequence id (its bytes are ignored;
+ *                         -1 = no end-of-sequence token)
+ *   opts                : NULL = defaults
+ *   out                 : receives the handle (NULL on error)
+ * Errors: PSC_ERR_GRAMMAR / _CONFLICT / _LEXER_AMBIGUOUS for the grammar,
+ * PSC_ERR_LIMIT, PSC_ERR_OOM, PSC_ERR_CUDA, PSC_ERR_ARG. */
+psc_status psc_compile(const char* grammar, size_t grammar_len, const uint8_t* vocab_bytes,
+                       const int64_t* vocab_offsets, int32_t V, int32_t eos_id,
+                       const psc_options* opts, psc_handle** out);
+
+/* Frees the handle's host and device tables (NULL is a no-op).  No call that
+ * uses the handle may still be running on any stream. */
+void psc_destroy(psc_handle* h);
+
+/* Thread-local message of the last failed call on this thread ("" if none). */
+const char* psc_last_error(void);
+
+/* Table sizes of a compiled handle (Table 7 of the paper reports the same
+ * quantities for its CPU implementation). */
+psc_status psc_info(const psc_handle* h, psc_info_t* out);
+
+/* A batch of B parser configurations on the device (Algorithm 2, steps 1-2:
+ * the lexer state q and the parser stack alpha of each sequence, Section 3.2),
+ * all at the empty prefix: q = the empty lexeme, alpha = [0], status OK.
+ *   cap : stack capacity per row (>= 2); layout [B][cap] uint16, bottom first.
+ * The states object owns its device arrays; initialisation is enqueued on stream. */
+psc_status psc_state_init(const psc_handle* h, int32_t B, int32_t cap, void* stream, psc_states** out);
+
+/* Resets rows to the empty prefix: the n row indices in d_rows (device int32),
+ * or every row when d_rows is NULL. */
+psc_status psc_state_reset(psc_states* st, const int32_t* d_rows, int32_t n, void* stream);
+
+void psc_state_destroy(psc_states* st);
+
+/* Algorithm 2, steps 1-2, done incrementally on the device: for each row b with
+ * d_tokens[b] >= 0, first checks the token against the row's current mask; a
+ * token outside it sets PSC_ROW_REJECTED; the end-of-sequence token sets
+ * PSC_ROW_DONE; any other allowed token is lexed from the row's lexer state and
+ * the emitted terminals are fed to the LALR(1) parser on the row's stack.
+ * d_tokens[b] < 0 leaves row b unchanged.  B must equal the batch size.
+ *   d_row_status : optional device int32[B] copy of the statuses after the step. */
+psc_status psc_advance(const psc_handle* h, psc_states* st, const int32_t* d_tokens, int32_t B,
+                       int32_t* d_row_status, void* stream);
+
+/* Algorithm 2, steps 3-4: classifies every row's (q, alpha) with the classifier
+ * DFA (one pass over the stack from the top, stopping at absorbing states) and
+ * writes the precomputed mask of the resulting state as a packed bitmask.
+ *   d_bitmask : device uint32 [B][W], W = ceil(V/32), row-contiguous.
+ * Rows with status DONE get the end-of-sequence-only mask, failed rows the
+ * empty mask. */
+psc_status psc_fill_mask(const psc_handle* h, const psc_states* st, int32_t B, uint32_t* d_bitmask,
+                         void* stream);
+
+/* Applies packed bitmasks to logits in place: logits[b][v] = -inf where bit v
+ * of row b is 0 (bf16 0xFF80, f32 0xFF800000); allowed logits keep their exact
+ * bits.  Columns v >= V are not touched.  (The paper leaves this step to the
+ * serving engine and excludes it from its timing, Section 4.3 "Metrics".)
+ *   d_logits   : device [B] rows of row_stride elements of dtype
+ *   row_stride : elements between rows, >= V
+ *   d_bitmask  : device uint32 [B][ceil(V/32)] */
+psc_status psc_apply_mask(void* d_logits, psc_dtype dtype, int64_t row_stride, const uint32_t* d_bitmask,
+                          int32_t B, int32_t V, void* stream);
+
+/* psc_fill_mask and psc_apply_mask fused: the classifier walk picks each row's
+ * mask row, which is applied to the logits straight from the device mask table
+ * (the bitmask does not round-trip through memory).  V must equal the
+ * handle's vocabulary size.
+ *   d_bitmask_out : optional device uint32 [B][W] copy of the masks (NULL = none). */
+psc_status psc_fill_apply(const psc_handle* h, const psc_states* st, int32_t B, void* d_logits,
+                          psc_dtype dtype, int64_t row_stride, int32_t V, uint32_t* d_bitmask_out,
+                          void* stream);
+
+/* Greedy sampling over the allowed tokens: d_tokens[b] = the lowest index v
+ * with the largest logits[b][v] among the tokens of row b's mask, or -1 when
+ * the mask is empty.  Only allowed positions are read.  Rows are classified as
+ * in psc_fill_mask (call it after psc_fill_apply and before psc_advance). */
+psc_status psc_argmax_masked(const psc_handle* h, const psc_states* st, int32_t B, const void* d_logits,
+                             psc_dtype dtype, int64_t row_stride, int32_t V, int32_t* d_tokens,
+                             void* stream);
+
+/* Copies the batch to host memory and synchronises the stream (tests and
+ * debugging).  Any output pointer may be NULL.
+ *   h_q, h_depth, h_status : int32 [B];  h_stack : uint16 [B][cap] */
+psc_status psc_states_download(const psc_states* st, int32_t* h_q, int32_t* h_depth, uint16_t* h_stack,
+                               int32_t* h_status, void* stream);
+
+/* Host-side inspection of the compiled tables (no GPU needed):
+ * psc_host_classify walks the classifier DFA for one configuration and
+ * returns its mask id (or -1 on bad arguments); psc_host_mask_row copies mask
+ * row `mask_id` (W words) to h_row. */
+int32_t psc_host_classify(const psc_handle* h, int32_t q, const uint16_t* h_stack, int32_t depth,
+                          int32_t status);
+psc_status psc_host_mask_row(const psc_handle* h, int32_t mask_id, uint32_t* h_row);
+
+/* Host-side lexer+parser step of one configuration (tests and prefix set-up
+ * without a GPU): the same semantics as psc_advance for a single row held in
+ * host memory.  *q, *depth, *status and h_stack[cap] are updated in place. */
+psc_status psc_host_advance(const psc_handle* h, int32_t* q, uint16_t* h_stack, int32_t* depth, int32_t cap,
+                            int32_t* status, int32_t token);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* PSC_H */

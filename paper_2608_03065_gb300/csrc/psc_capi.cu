@@ -1,0 +1,856 @@
+// C ABI of the PSC library (include/psc.h) and its CUDA kernels for sm_103a.
+//
+// Online step of the paper (Algorithm 2), per decoding step and batch row:
+//   steps 1-2  incremental lexing and LR parsing of the sampled token on the
+//              row's device-resident stack                      -> k_advance
+//   step 3     one pass of the classifier DFA over (q, stack from the top),
+//              O(|stack|), stopping at absorbing states          -> k_classify
+//   step 4     the precomputed mask of the reached state         -> k_fill / k_apply_rows
+// plus applying the mask to the logits and greedy sampling over the allowed
+// tokens (left to the serving engine in the paper).
+//
+// Memory layout on the device (all tables uploaded once by psc_compile):
+//   dfa      int32 [S][n_lr]      next classifier state, or -(mask+1) when absorbing
+//   masks    uint32 [n_masks][Wp] mask rows, Wp = W rounded up to 4 words (16-byte rows)
+//   stacks   uint16 [B][cap]      parser stacks, bottom first; depth[b] entries used
+//   logits   [B][row_stride]      bf16 or f32, caller-owned, masked in place
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cstring>
+#include <memory>
+#include <new>
+#include <string>
+
+#include "../../include/psc.h"
+#include "psc_internal.h"
+
+namespace {
+
+thread_local std::string g_last_error;
+
+psc_status fail_with(psc_status code, const std::string& msg) {
+    g_last_error = msg;
+    return code;
+}
+
+constexpr unsigned FULL = 0xffffffffu;
+constexpr int ROW_OK = 0, ROW_DONE = 1, ROW_REJECTED = 2, ROW_OVERFLOW = 3, ROW_LIMIT = 4;
+
+struct DevTables {
+    const int16_t* lex_trans;
+    const int32_t* lex_accept;
+    const uint8_t* cls_ignored;
+    const int32_t* action;
+    const int32_t* go;
+    const int32_t* rule_len;
+    const int32_t* rule_lhs;
+    const int16_t* resolve;
+    const int32_t* dfa;
+    const int32_t* dfa_start;
+    const int32_t* dfa_mask;
+    const uint32_t* masks;
+    const uint8_t* vocab;
+    const int64_t* vocab_off;
+    int q0, nq, n_lr, n_terms, n_nts, end_term;
+    int V, W, Wp, eos_id, n_masks;
+};
+
+struct DevStates {
+    int32_t* q;
+    int32_t* depth;
+    int32_t* status;
+    uint16_t* stack;
+    int32_t* mid;
+    int B, cap;
+};
+
+}  // namespace
+
+struct psc_handle {
+    psc::Tables t;
+    bool host_only = true;
+    int device = -1;
+    DevTables d{};
+    void* blocks[16] = {};
+    int n_blocks = 0;
+};
+
+struct psc_states {
+    const psc_handle* h = nullptr;
+    DevStates d{};
+    int device = -1;
+    uint64_t gen = 1;        // bumped by every call that changes the rows
+    uint64_t mid_gen = 0;    // generation the mask ids in d.mid were computed for
+};
+
+namespace {
+
+// ------------------------------------------------------------------ helpers
+__device__ __forceinline__ void st_cs_v4(void* p, uint4 v) {
+    asm volatile("st.global.cs.v4.b32 [%0], {%1, %2, %3, %4};" ::"l"(p), "r"(v.x), "r"(v.y), "r"(v.z),
+                 "r"(v.w)
+                 : "memory");
+}
+
+__device__ __forceinline__ uint4 ld_nc_v4(const void* p) {
+    uint4 v;
+    asm volatile("ld.global.nc.v4.b32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "l"(p));
+    return v;
+}
+
+// Classifier walk for one row (Algorithm 2 step 3), executed by a full warp:
+// lanes load 32 stack symbols at a time (coalesced), the walk broadcasts them
+// with shuffles and follows the DFA; every lane ends with the same mask id.
+__device__ int warp_classify(const DevTables& T, const DevStates& S, int b, int lane) {
+    int status = S.status[b];
+    if (status == ROW_DONE) return 1;
+    if (status != ROW_OK) return 0;
+    int q = S.q[b];
+    int depth = S.depth[b];
+    if (q < 0 || q >= T.nq || depth < 1 || depth > S.cap) return 0;
+    int s = __ldg(T.dfa_start + q);
+    if (s < 0) return -s - 1;
+    const uint16_t* st = S.stack + (size_t)b * S.cap;
+    for (int top = depth - 1; top >= 0; top -= 32) {
+        int i = top - lane;
+        int x = i >= 0 ? st[i] : 0;
+        int n = top + 1 < 32 ? top + 1 : 32;
+        for (int j = 0; j < n; j++) {
+            int X = __shfl_sync(FULL, x, j);
+            int nx = __ldg(T.dfa + (size_t)s * T.n_lr + X);
+            if (nx < 0) return -nx - 1;
+            s = nx;
+        }
+    }
+    return __ldg(T.dfa_mask + s);
+}
+
+// the same walk by one thread
+__device__ int thread_classify(const DevTables& T, const DevStates& S, int b) {
+    int status = S.status[b];
+    if (status == ROW_DONE) return 1;
+    if (status != ROW_OK) return 0;
+    int q = S.q[b];
+    int depth = S.depth[b];
+    if (q < 0 || q >= T.nq || depth < 1 || depth > S.cap) return 0;
+    int s = __ldg(T.dfa_start + q);
+    if (s < 0) return -s - 1;
+    const uint16_t* st = S.stack + (size_t)b * S.cap;
+    for (int i = depth - 1; i >= 0; i--) {
+        int nx = __ldg(T.dfa + (size_t)s * T.n_lr + st[i]);
+        if (nx < 0) return -nx - 1;
+        s = nx;
+    }
+    return __ldg(T.dfa_mask + s);
+}
+
+// ------------------------------------------------------------------ kernels
+__global__ void k_state_init(DevStates S, int q0, const int32_t* rows, int n) {
+    int i = blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= n) return;
+    int b = rows ? rows[i] : i;
+    if (b < 0 || b >= S.B) return;
+    S.q[b] = q0;
+    S.depth[b] = 1;
+    S.status[b] = ROW_OK;
+    S.stack[(size_t)b * S.cap] = 0;
+    S.mid[b] = 0;
+}
+
+__global__ void k_classify(DevTables T, DevStates S, int B) {
+    int warp = (int)((blockIdx.x * (size_t)blockDim.x + threadIdx.x) >> 5);
+    int lane = threadIdx.x & 31;
+    if (warp >= B) return;
+    int mid = warp_classify(T, S, warp, lane);
+    if (lane == 0) S.mid[warp] = mid;
+}
+
+// out[b][:] = masks[mid[b]][:]   (16-byte vector copies when W % 4 == 0)
+__global__ void k_fill(const uint32_t* __restrict__ masks, int Wp, const int32_t* __restrict__ mid, int B, int W,
+                       uint32_t* __restrict__ out, int vec) {
+    size_t tid = blockIdx.x * (size_t)blockDim.x + threadIdx.x;
+    size_t stride = (size_t)gridDim.x * blockDim.x;
+    if (vec) {
+        int W4 = W >> 2;
+        size_t total = (size_t)B * W4;
+        for (size_t i = tid; i < total; i += stride) {
+            int b = (int)(i / W4), w = (int)(i % W4);
+            uint4 v = ld_nc_v4(masks + (size_t)mid[b] * Wp + 4 * w);
+            st_cs_v4(out + (size_t)b * W + 4 * w, v);
+        }
+    } else {
+        size_t total = (size_t)B * W;
+        for (size_t i = tid; i < total; i += stride) {
+            int b = (int)(i / W), w = (int)(i % W);
+            out[i] = __ldg(masks + (size_t)mid[b] * Wp + w);
+        }
+    }
+}
+
+template <typename T>
+struct NegInf;
+template <>
+struct NegInf<uint16_t> {
+    static constexpr uint32_t pair = 0xFF80FF80u;
+    static constexpr uint16_t one = 0xFF80u;
+};
+template <>
+struct NegInf<uint32_t> {
+    static constexpr uint32_t pair = 0xFF800000u;
+    static constexpr uint32_t one = 0xFF800000u;
+};
+
+// Apply one 1024-column chunk of row b: `word` is this lane's mask word for
+// columns [col0 + 32*lane, col0 + 32*lane + 32).  E = elements per 16 bytes.
+template <typename T>
+__device__ __forceinline__ void apply_chunk(T* row, int col0, uint32_t word, int lane) {
+    constexpr int E = 16 / sizeof(T);
+    constexpr int PASSES = 1024 / E / 32;
+    constexpr uint32_t FULLBITS = (1u << E) - 1u;
+    uint4 ninf = make_uint4(NegInf<T>::pair, NegInf<T>::pair, NegInf<T>::pair, NegInf<T>::pair);
+#pragma unroll
+    for (int k = 0; k < PASSES; k++) {
+        int c = k * 32 + lane;                      // 16-byte chunk index within the 1024 columns
+        int wsrc = (c * E) >> 5;
+        int sh = (c * E) & 31;
+        uint32_t bits = (__shfl_sync(FULL, word, wsrc) >> sh) & FULLBITS;
+        T* p = row + col0 + c * E;
+        if (bits == 0) {
+            st_cs_v4(p, ninf);
+        } else if (bits != FULLBITS) {
+            uint4 v = *reinterpret_cast<const uint4*>(p);
+            uint32_t w[4] = {v.x, v.y, v.z, v.w};
+            if (sizeof(T) == 2) {
+#pragma unroll
+                for (int e = 0; e < 8; e++)
+                    if (!((bits >> e) & 1)) {
+                        uint32_t& x = w[e >> 1];
+                        x = (e & 1) ? ((x & 0x0000FFFFu) | 0xFF800000u) : ((x & 0xFFFF0000u) | 0x0000FF80u);
+                    }
+            } else {
+#pragma unroll
+                for (int e = 0; e < 4; e++)
+                    if (!((bits >> e) & 1)) w[e] = 0xFF800000u;
+            }
+            *reinterpret_cast<uint4*>(p) = make_uint4(w[0], w[1], w[2], w[3]);
+        }
+    }
+}
+
+// element-by-element path for ragged chunks or unaligned rows: each lane
+// handles the 32 columns of its own mask word
+template <typename T>
+__device__ __forceinline__ void apply_chunk_scalar(T* row, int col0, int ncols, uint32_t word, int lane) {
+    int c0 = 32 * lane;
+    for (int e = 0; e < 32; e++) {
+        if (c0 + e >= ncols) break;
+        if (!((word >> e) & 1)) row[col0 + c0 + e] = (T)NegInf<T>::one;
+    }
+}
+
+// Mask source for the apply kernels: a caller bitmask [B][W], or the device
+// mask table row picked by the classifier (mid[b]).
+struct MaskSrc {
+    const uint32_t* bitmask;   // nullable
+    const uint32_t* table;
+    const int32_t* mid;
+    int W, Wp;
+    uint32_t* copy_out;        // nullable: also write the words here ([B][W])
+    __device__ __forceinline__ const uint32_t* row(int b) const {
+        return bitmask ? bitmask + (size_t)b * W : table + (size_t)__ldg(mid + b) * Wp;
+    }
+};
+
+template <typename T>
+__global__ void __launch_bounds__(256) k_apply_rows(T* logits, int64_t stride, MaskSrc M, int B, int V, int vec) {
+    int lane = threadIdx.x & 31;
+    int gw = (int)((blockIdx.x * (size_t)blockDim.x + threadIdx.x) >> 5);
+    int nw = (int)((gridDim.x * (size_t)blockDim.x) >> 5);
+    int cpr = (V + 1023) >> 10;
+    long total = (long)B * cpr;
+    for (long c = gw; c < total; c += nw) {
+        int b = (int)(c / cpr);
+        int j = (int)(c - (long)b * cpr);
+        int col0 = j << 10;
+        int wi = (col0 >> 5) + lane;
+        const uint32_t* mrow = M.row(b);
+        uint32_t word = wi < M.W ? __ldg(mrow + wi) : 0u;
+        if (M.copy_out && wi < M.W) M.copy_out[(size_t)b * M.W + wi] = word;
+        T* row = logits + (size_t)b * stride;
+        int ncols = V - col0;
+        if (vec && ncols >= 1024) apply_chunk<T>(row, col0, word, lane);
+        else apply_chunk_scalar<T>(row, col0, ncols < 1024 ? ncols : 1024, word, lane);
+    }
+}
+
+__device__ __forceinline__ float bf16_to_float(uint16_t h) { return __uint_as_float((uint32_t)h << 16); }
+
+// Greedy choice among allowed tokens: one block per row, reads only the
+// 16-byte chunks that hold an allowed position.
+template <typename T>
+__global__ void __launch_bounds__(256) k_argmax_masked(const T* logits, int64_t stride, DevTables D,
+                                                       const int32_t* mid, int B, int V, int vec,
+                                                       int32_t* tokens) {
+    int b = blockIdx.x;
+    if (b >= B) return;
+    int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarp = blockDim.x >> 5;
+    const uint32_t* mrow = D.masks + (size_t)mid[b] * D.Wp;
+    const T* row = logits + (size_t)b * stride;
+    float best = 0.f;
+    int bi = -1;
+    auto consider = [&](float v, int i) {
+        if (v != v) return;   // NaN never wins
+        if (bi < 0 || v > best || (v == best && i < bi)) {
+            best = v;
+            bi = i;
+        }
+    };
+    constexpr int E = 16 / sizeof(T);
+    int cpr = (V + 1023) >> 10;
+    for (int j = warp; j < cpr; j += nwarp) {
+        int col0 = j << 10;
+        int wi = (col0 >> 5) + lane;
+        uint32_t word = wi < D.W ? __ldg(mrow + wi) : 0u;
+        if (__ballot_sync(FULL, word != 0) == 0) continue;
+        int ncols = V - col0;
+        if (vec && ncols >= 1024) {
+#pragma unroll
+            for (int k = 0; k < 1024 / E / 32; k++) {
+                int c = k * 32 + lane;
+                uint32_t bits = (__shfl_sync(FULL, word, (c * E) >> 5) >> ((c * E) & 31)) & ((1u << E) - 1u);
+                if (!bits) continue;
+                uint4 v = ld_nc_v4(row + col0 + c * E);
+                uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+                for (int e = 0; e < E; e++) {
+                    if (!((bits >> e) & 1)) continue;
+                    float f;
+                    if (sizeof(T) == 2) f = bf16_to_float((uint16_t)((w[e >> 1] >> ((e & 1) * 16)) & 0xFFFF));
+                    else f = __uint_as_float(w[e]);
+                    consider(f, col0 + c * E + e);
+                }
+            }
+        } else {
+            for (int e = 0; e < 32; e++) {
+                int col = col0 + 32 * lane + e;
+                if (col >= V) break;
+                if ((word >> e) & 1) {
+                    float f = sizeof(T) == 2 ? bf16_to_float((uint16_t)row[col]) : __uint_as_float((uint32_t)row[col]);
+                    consider(f, col);
+                }
+            }
+        }
+    }
+    // warp then block reduction of (best, bi)
+    for (int off = 16; off; off >>= 1) {
+        float ov = __shfl_down_sync(FULL, best, off);
+        int oi = __shfl_down_sync(FULL, bi, off);
+        if (oi >= 0 && (bi < 0 || ov > best || (ov == best && oi < bi))) {
+            best = ov;
+            bi = oi;
+        }
+    }
+    __shared__ float sv[32];
+    __shared__ int si[32];
+    if (lane == 0) {
+        sv[warp] = best;
+        si[warp] = bi;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        for (int w = 1; w < nwarp; w++) {
+            if (si[w] >= 0 && (bi < 0 || sv[w] > best || (sv[w] == best && si[w] < bi))) {
+                best = sv[w];
+                bi = si[w];
+            }
+        }
+        tokens[b] = bi;
+    }
+}
+
+// Feed one lexeme class to the parser on a row's stack: resolve the class to a
+// terminal with the current top, reduce until it is shifted.  Returns a row status.
+__device__ int feed_class(const DevTables& T, uint16_t* st, int& depth, int cap, int cls) {
+    int top = st[depth - 1];
+    int t = T.resolve[(size_t)cls * T.n_lr + top];
+    if (t < 0) return ROW_REJECTED;
+    for (int guard = 0; guard < 4 * cap + 64; guard++) {
+        int32_t a = T.action[(size_t)st[depth - 1] * T.n_terms + t];
+        int kind = a & 3, val = a >> 2;
+        if (kind == psc::ACT_SHIFT) {
+            if (depth >= cap) return ROW_OVERFLOW;
+            st[depth++] = (uint16_t)val;
+            return ROW_OK;
+        }
+        if (kind != psc::ACT_REDUCE) return ROW_REJECTED;
+        int k = T.rule_len[val];
+        if (depth - k < 1) return ROW_REJECTED;
+        depth -= k;
+        int go = T.go[(size_t)st[depth - 1] * T.n_nts + T.rule_lhs[val]];
+        if (go < 0) return ROW_REJECTED;
+        if (depth >= cap) return ROW_OVERFLOW;
+        st[depth++] = (uint16_t)go;
+    }
+    return ROW_LIMIT;
+}
+
+// Algorithm 2 steps 1-2 for one row per thread.
+__global__ void k_advance(DevTables T, DevStates S, const int32_t* tokens, int B, int use_mid,
+                          int32_t* status_out) {
+    int b = blockIdx.x * blockDim.x + threadIdx.x;
+    if (b >= B) return;
+    int tok = tokens[b];
+    int status = S.status[b];
+    if (tok >= 0) {
+        if (status == ROW_DONE) {
+            status = tok == T.eos_id ? ROW_DONE : ROW_REJECTED;
+        } else if (status == ROW_OK) {
+            if (tok >= T.V) {
+                status = ROW_REJECTED;
+            } else {
+                int mid = use_mid ? S.mid[b] : thread_classify(T, S, b);
+                bool allowed = (__ldg(T.masks + (size_t)mid * T.Wp + (tok >> 5)) >> (tok & 31)) & 1;
+                if (!allowed) {
+                    status = ROW_REJECTED;
+                } else if (tok == T.eos_id) {
+                    status = ROW_DONE;
+                } else {
+                    int q = S.q[b], depth = S.depth[b];
+                    uint16_t* st = S.stack + (size_t)b * S.cap;
+                    int64_t lo = T.vocab_off[tok], hi = T.vocab_off[tok + 1];
+                    for (int64_t i = lo; i < hi && status == ROW_OK; i++) {
+                        int c = T.vocab[i];
+                        int nx = T.lex_trans[(size_t)q * 256 + c];
+                        if (nx >= 0) {
+                            q = nx;
+                            continue;
+                        }
+                        int cls = q == T.q0 ? -1 : T.lex_accept[q];
+                        if (cls < 0) {
+                            status = ROW_REJECTED;
+                            break;
+                        }
+                        if (!T.cls_ignored[cls]) status = feed_class(T, st, depth, S.cap, cls);
+                        q = T.lex_trans[(size_t)T.q0 * 256 + c];
+                        if (q < 0) status = ROW_REJECTED;
+                    }
+                    if (status == ROW_OK) {
+                        S.q[b] = q;
+                        S.depth[b] = depth;
+                    }
+                }
+            }
+        }
+        S.status[b] = status;
+    }
+    if (status_out) status_out[b] = status;
+}
+
+// ----------------------------------------------------------------- host glue
+psc_status cuda_check(cudaError_t e, const char* what) {
+    if (e == cudaSuccess) return PSC_OK;
+    return fail_with(e == cudaErrorMemoryAllocation ? PSC_ERR_OOM : PSC_ERR_CUDA,
+                     std::string(what) + ": " + cudaGetErrorString(e));
+}
+
+psc_status launch_check(const char* what) { return cuda_check(cudaGetLastError(), what); }
+
+int sm_count(int device) {
+    int n = 0;
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, device);
+    return n > 0 ? n : 1;
+}
+
+template <typename V>
+psc_status upload(psc_handle* h, const std::vector<V>& v, const V** dst, size_t pad_bytes = 0) {
+    size_t bytes = v.size() * sizeof(V) + pad_bytes;
+    if (bytes == 0) bytes = 16;
+    void* p = nullptr;
+    psc_status s = cuda_check(cudaMalloc(&p, bytes), "cudaMalloc(tables)");
+    if (s != PSC_OK) return s;
+    h->blocks[h->n_blocks++] = p;
+    if (!v.empty()) {
+        s = cuda_check(cudaMemcpy(p, v.data(), v.size() * sizeof(V), cudaMemcpyHostToDevice), "cudaMemcpy(tables)");
+        if (s != PSC_OK) return s;
+    }
+    *dst = static_cast<const V*>(p);
+    return PSC_OK;
+}
+
+psc_status check_device(const psc_handle* h, const char* what) {
+    if (!h) return fail_with(PSC_ERR_ARG, std::string(what) + ": NULL handle");
+    if (h->host_only) return fail_with(PSC_ERR_ARG, std::string(what) + ": handle was compiled host_only");
+    int dev = -1;
+    cudaGetDevice(&dev);
+    if (dev != h->device)
+        return fail_with(PSC_ERR_ARG, std::string(what) + ": current device differs from the handle's");
+    return PSC_OK;
+}
+
+psc_status ensure_mid(const psc_handle* h, const psc_states* st, cudaStream_t s) {
+    if (st->mid_gen == st->gen) return PSC_OK;
+    int B = st->d.B;
+    int threads = 256;
+    int blocks = (int)(((size_t)B * 32 + threads - 1) / threads);
+    k_classify<<<blocks, threads, 0, s>>>(h->d, st->d, B);
+    psc_status r = launch_check("k_classify");
+    if (r == PSC_OK) const_cast<psc_states*>(st)->mid_gen = st->gen;
+    return r;
+}
+
+bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+
+psc_status launch_apply(void* logits, psc_dtype dtype, int64_t row_stride, const MaskSrc& M, int B, int V,
+                        cudaStream_t s, int device) {
+    size_t esz = dtype == PSC_BF16 ? 2 : 4;
+    int vec = aligned16(logits) && ((row_stride * (int64_t)esz) % 16 == 0);
+    long chunks = (long)B * ((V + 1023) / 1024);
+    int threads = 256;
+    long want = (chunks + 7) / 8;
+    int blocks = (int)std::min<long>(want, (long)sm_count(device) * 8);
+    if (blocks < 1) blocks = 1;
+    if (dtype == PSC_BF16)
+        k_apply_rows<uint16_t><<<blocks, threads, 0, s>>>((uint16_t*)logits, row_stride, M, B, V, vec);
+    else
+        k_apply_rows<uint32_t><<<blocks, threads, 0, s>>>((uint32_t*)logits, row_stride, M, B, V, vec);
+    return launch_check("k_apply_rows");
+}
+
+// host-side parser step for psc_host_advance (same semantics as k_advance)
+int host_feed(const psc::Tables& T, uint16_t* st, int& depth, int cap, int cls) {
+    int t = T.resolve[(size_t)cls * T.n_lr + st[depth - 1]];
+    if (t < 0) return ROW_REJECTED;
+    for (int guard = 0; guard < 4 * cap + 64; guard++) {
+        int32_t a = T.action[(size_t)st[depth - 1] * T.n_terms + t];
+        int kind = a & 3, val = a >> 2;
+        if (kind == psc::ACT_SHIFT) {
+            if (depth >= cap) return ROW_OVERFLOW;
+            st[depth++] = (uint16_t)val;
+            return ROW_OK;
+        }
+        if (kind != psc::ACT_REDUCE) return ROW_REJECTED;
+        int k = T.rule_len[val];
+        if (depth - k < 1) return ROW_REJECTED;
+        depth -= k;
+        int go = T.go[(size_t)st[depth - 1] * T.n_nts + T.rule_lhs[val]];
+        if (go < 0) return ROW_REJECTED;
+        if (depth >= cap) return ROW_OVERFLOW;
+        st[depth++] = (uint16_t)go;
+    }
+    return ROW_LIMIT;
+}
+
+}  // namespace
+
+// ====================================================================== ABI
+extern "C" {
+
+const char* psc_last_error(void) { return g_last_error.c_str(); }
+
+psc_status psc_compile(const char* grammar, size_t grammar_len, const uint8_t* vocab_bytes,
+                       const int64_t* vocab_offsets, int32_t V, int32_t eos_id, const psc_options* opts,
+                       psc_handle** out) {
+    if (!out) return fail_with(PSC_ERR_ARG, "psc_compile: out is NULL");
+    *out = nullptr;
+    if (!grammar || !vocab_offsets || V <= 0 || (!vocab_bytes && vocab_offsets[V] > 0))
+        return fail_with(PSC_ERR_ARG, "psc_compile: bad grammar or vocabulary arguments");
+    if (eos_id >= V || eos_id < -1) return fail_with(PSC_ERR_ARG, "psc_compile: eos_id out of range");
+    for (int v = 0; v < V; v++)
+        if (vocab_offsets[v + 1] < vocab_offsets[v]) return fail_with(PSC_ERR_ARG, "psc_compile: offsets decrease");
+    psc::Options o;
+    bool host_only = false;
+    if (opts) {
+        if (opts->max_states > 0) o.max_states = opts->max_states;
+        if (opts->max_mask_bytes > 0) o.max_mask_bytes = opts->max_mask_bytes;
+        o.threads = opts->threads;
+        host_only = opts->host_only != 0;
+    }
+    std::unique_ptr<psc_handle> h(new (std::nothrow) psc_handle());
+    if (!h) return fail_with(PSC_ERR_OOM, "psc_compile: out of host memory");
+    try {
+        h->t = psc::compile_tables(std::string(grammar, grammar_len), vocab_bytes, vocab_offsets, V, eos_id, o);
+    } catch (const psc::Error& e) {
+        return fail_with((psc_status)e.code, e.what());
+    } catch (const std::bad_alloc&) {
+        return fail_with(PSC_ERR_OOM, "psc_compile: out of host memory");
+    }
+    h->host_only = host_only;
+    if (!host_only) {
+        const psc::Tables& t = h->t;
+        psc_status s = cuda_check(cudaGetDevice(&h->device), "cudaGetDevice");
+        if (s != PSC_OK) return s;
+        DevTables& d = h->d;
+        int Wp = (t.W + 3) & ~3;
+        std::vector<uint32_t> masks((size_t)t.n_masks * Wp, 0);
+        for (int m = 0; m < t.n_masks; m++)
+            std::memcpy(masks.data() + (size_t)m * Wp, t.masks.data() + (size_t)m * t.W, sizeof(uint32_t) * t.W);
+        std::vector<int32_t> dfa = t.dfa;
+        if (dfa.empty()) dfa.push_back(0);
+        std::vector<int32_t> dfa_mask = t.dfa_mask;
+        if (dfa_mask.empty()) dfa_mask.push_back(0);
+        if ((s = upload(h.get(), t.lex_trans, &d.lex_trans)) || (s = upload(h.get(), t.lex_accept, &d.lex_accept)) ||
+            (s = upload(h.get(), t.cls_ignored, &d.cls_ignored)) || (s = upload(h.get(), t.action, &d.action)) ||
+            (s = upload(h.get(), t.go, &d.go)) || (s = upload(h.get(), t.rule_len, &d.rule_len)) ||
+            (s = upload(h.get(), t.rule_lhs, &d.rule_lhs)) || (s = upload(h.get(), t.resolve, &d.resolve)) ||
+            (s = upload(h.get(), dfa, &d.dfa)) || (s = upload(h.get(), t.dfa_start, &d.dfa_start)) ||
+            (s = upload(h.get(), dfa_mask, &d.dfa_mask)) || (s = upload(h.get(), masks, &d.masks)) ||
+            (s = upload(h.get(), t.vocab_bytes, &d.vocab, 16)) || (s = upload(h.get(), t.vocab_off, &d.vocab_off))) {
+            for (int i = 0; i < h->n_blocks; i++) cudaFree(h->blocks[i]);
+            return s;
+        }
+        d.q0 = t.q0;
+        d.nq = t.nq;
+        d.n_lr = t.n_lr;
+        d.n_terms = t.n_terms;
+        d.n_nts = t.n_nts;
+        d.end_term = t.end_term;
+        d.V = t.V;
+        d.W = t.W;
+        d.Wp = Wp;
+        d.eos_id = t.eos_id;
+        d.n_masks = t.n_masks;
+    }
+    *out = h.release();
+    return PSC_OK;
+}
+
+void psc_destroy(psc_handle* h) {
+    if (!h) return;
+    for (int i = 0; i < h->n_blocks; i++) cudaFree(h->blocks[i]);
+    delete h;
+}
+
+psc_status psc_info(const psc_handle* h, psc_info_t* out) {
+    if (!h || !out) return fail_with(PSC_ERR_ARG, "psc_info: NULL argument");
+    const psc::Tables& t = h->t;
+    out->V = t.V;
+    out->W = t.W;
+    out->n_lexer_states = t.nq;
+    out->n_parser_states = t.n_lr;
+    out->n_terminals = t.n_terms;
+    out->n_classifier_states = t.S;
+    out->n_masks = t.n_masks;
+    out->eos_id = t.eos_id;
+    out->classifier_bytes = (int64_t)(t.dfa.size() + t.dfa_start.size() + t.dfa_mask.size()) * 4;
+    out->mask_bytes = (int64_t)t.n_masks * ((t.W + 3) & ~3) * 4;
+    out->states_built = t.n_dfa_states_built;
+    out->compile_seconds = t.seconds_total;
+    return PSC_OK;
+}
+
+psc_status psc_state_init(const psc_handle* h, int32_t B, int32_t cap, void* stream, psc_states** out) {
+    if (!out) return fail_with(PSC_ERR_ARG, "psc_state_init: out is NULL");
+    *out = nullptr;
+    psc_status s = check_device(h, "psc_state_init");
+    if (s != PSC_OK) return s;
+    if (B <= 0 || cap < 2 || cap > (1 << 20)) return fail_with(PSC_ERR_ARG, "psc_state_init: bad B or cap");
+    std::unique_ptr<psc_states> st(new (std::nothrow) psc_states());
+    if (!st) return fail_with(PSC_ERR_OOM, "psc_state_init: out of host memory");
+    st->h = h;
+    st->device = h->device;
+    DevStates& d = st->d;
+    d.B = B;
+    d.cap = cap;
+    void* p[5] = {};
+    size_t sz[5] = {sizeof(int32_t) * B, sizeof(int32_t) * B, sizeof(int32_t) * B, sizeof(uint16_t) * (size_t)B * cap,
+                    sizeof(int32_t) * B};
+    for (int i = 0; i < 5; i++) {
+        s = cuda_check(cudaMalloc(&p[i], sz[i]), "cudaMalloc(states)");
+        if (s != PSC_OK) {
+            for (int j = 0; j < i; j++) cudaFree(p[j]);
+            return s;
+        }
+    }
+    d.q = (int32_t*)p[0];
+    d.depth = (int32_t*)p[1];
+    d.status = (int32_t*)p[2];
+    d.stack = (uint16_t*)p[3];
+    d.mid = (int32_t*)p[4];
+    cudaStream_t cs = (cudaStream_t)stream;
+    k_state_init<<<(B + 255) / 256, 256, 0, cs>>>(d, h->d.q0, nullptr, B);
+    s = launch_check("k_state_init");
+    if (s != PSC_OK) {
+        for (int j = 0; j < 5; j++) cudaFree(p[j]);
+        return s;
+    }
+    *out = st.release();
+    return PSC_OK;
+}
+
+psc_status psc_state_reset(psc_states* st, const int32_t* d_rows, int32_t n, void* stream) {
+    if (!st) return fail_with(PSC_ERR_ARG, "psc_state_reset: NULL states");
+    int cnt = d_rows ? n : st->d.B;
+    if (cnt < 0) return fail_with(PSC_ERR_ARG, "psc_state_reset: negative count");
+    st->gen++;
+    if (cnt == 0) return PSC_OK;
+    k_state_init<<<(cnt + 255) / 256, 256, 0, (cudaStream_t)stream>>>(st->d, st->h->d.q0, d_rows, cnt);
+    return launch_check("k_state_init");
+}
+
+void psc_state_destroy(psc_states* st) {
+    if (!st) return;
+    cudaFree(st->d.q);
+    cudaFree(st->d.depth);
+    cudaFree(st->d.status);
+    cudaFree(st->d.stack);
+    cudaFree(st->d.mid);
+    delete st;
+}
+
+psc_status psc_advance(const psc_handle* h, psc_states* st, const int32_t* d_tokens, int32_t B,
+                       int32_t* d_row_status, void* stream) {
+    psc_status s = check_device(h, "psc_advance");
+    if (s != PSC_OK) return s;
+    if (!st || st->h != h || B != st->d.B || !d_tokens) return fail_with(PSC_ERR_ARG, "psc_advance: bad arguments");
+    int use_mid = st->mid_gen == st->gen ? 1 : 0;
+    k_advance<<<(B + 127) / 128, 128, 0, (cudaStream_t)stream>>>(h->d, st->d, d_tokens, B, use_mid, d_row_status);
+    st->gen++;
+    return launch_check("k_advance");
+}
+
+psc_status psc_fill_mask(const psc_handle* h, const psc_states* st, int32_t B, uint32_t* d_bitmask, void* stream) {
+    psc_status s = check_device(h, "psc_fill_mask");
+    if (s != PSC_OK) return s;
+    if (!st || st->h != h || B != st->d.B || !d_bitmask) return fail_with(PSC_ERR_ARG, "psc_fill_mask: bad arguments");
+    cudaStream_t cs = (cudaStream_t)stream;
+    if ((s = ensure_mid(h, st, cs)) != PSC_OK) return s;
+    int vec = (h->d.W % 4 == 0) && aligned16(d_bitmask);
+    size_t units = vec ? (size_t)B * (h->d.W / 4) : (size_t)B * h->d.W;
+    int blocks = (int)std::min<size_t>((units + 255) / 256, (size_t)sm_count(h->device) * 8);
+    if (blocks < 1) blocks = 1;
+    k_fill<<<blocks, 256, 0, cs>>>(h->d.masks, h->d.Wp, st->d.mid, B, h->d.W, d_bitmask, vec);
+    return launch_check("k_fill");
+}
+
+psc_status psc_apply_mask(void* d_logits, psc_dtype dtype, int64_t row_stride, const uint32_t* d_bitmask, int32_t B,
+                          int32_t V, void* stream) {
+    if (!d_logits || !d_bitmask || B < 0 || V <= 0 || row_stride < V || (dtype != PSC_F32 && dtype != PSC_BF16))
+        return fail_with(PSC_ERR_ARG, "psc_apply_mask: bad arguments");
+    if (B == 0) return PSC_OK;
+    int dev = 0;
+    cudaGetDevice(&dev);
+    MaskSrc M{d_bitmask, nullptr, nullptr, (V + 31) / 32, 0, nullptr};
+    return launch_apply(d_logits, dtype, row_stride, M, B, V, (cudaStream_t)stream, dev);
+}
+
+psc_status psc_fill_apply(const psc_handle* h, const psc_states* st, int32_t B, void* d_logits, psc_dtype dtype,
+                          int64_t row_stride, int32_t V, uint32_t* d_bitmask_out, void* stream) {
+    psc_status s = check_device(h, "psc_fill_apply");
+    if (s != PSC_OK) return s;
+    if (!st || st->h != h || B != st->d.B || !d_logits || V != h->d.V || row_stride < V ||
+        (dtype != PSC_F32 && dtype != PSC_BF16))
+        return fail_with(PSC_ERR_ARG, "psc_fill_apply: bad arguments");
+    cudaStream_t cs = (cudaStream_t)stream;
+    if ((s = ensure_mid(h, st, cs)) != PSC_OK) return s;
+    MaskSrc M{nullptr, h->d.masks, st->d.mid, h->d.W, h->d.Wp, d_bitmask_out};
+    return launch_apply(d_logits, dtype, row_stride, M, B, V, cs, h->device);
+}
+
+psc_status psc_argmax_masked(const psc_handle* h, const psc_states* st, int32_t B, const void* d_logits,
+                             psc_dtype dtype, int64_t row_stride, int32_t V, int32_t* d_tokens, void* stream) {
+    psc_status s = check_device(h, "psc_argmax_masked");
+    if (s != PSC_OK) return s;
+    if (!st || st->h != h || B != st->d.B || !d_logits || !d_tokens || V != h->d.V || row_stride < V ||
+        (dtype != PSC_F32 && dtype != PSC_BF16))
+        return fail_with(PSC_ERR_ARG, "psc_argmax_masked: bad arguments");
+    cudaStream_t cs = (cudaStream_t)stream;
+    if ((s = ensure_mid(h, st, cs)) != PSC_OK) return s;
+    size_t esz = dtype == PSC_BF16 ? 2 : 4;
+    int vec = aligned16(d_logits) && ((row_stride * (int64_t)esz) % 16 == 0);
+    if (dtype == PSC_BF16)
+        k_argmax_masked<uint16_t><<<B, 256, 0, cs>>>((const uint16_t*)d_logits, row_stride, h->d, st->d.mid, B, V, vec,
+                                                     d_tokens);
+    else
+        k_argmax_masked<uint32_t><<<B, 256, 0, cs>>>((const uint32_t*)d_logits, row_stride, h->d, st->d.mid, B, V, vec,
+                                                     d_tokens);
+    return launch_check("k_argmax_masked");
+}
+
+psc_status psc_states_download(const psc_states* st, int32_t* h_q, int32_t* h_depth, uint16_t* h_stack,
+                               int32_t* h_status, void* stream) {
+    if (!st) return fail_with(PSC_ERR_ARG, "psc_states_download: NULL states");
+    cudaStream_t cs = (cudaStream_t)stream;
+    const DevStates& d = st->d;
+    psc_status s = PSC_OK;
+    if (h_q && (s = cuda_check(cudaMemcpyAsync(h_q, d.q, sizeof(int32_t) * d.B, cudaMemcpyDeviceToHost, cs), "download q")))
+        return s;
+    if (h_depth && (s = cuda_check(cudaMemcpyAsync(h_depth, d.depth, sizeof(int32_t) * d.B, cudaMemcpyDeviceToHost, cs),
+                                   "download depth")))
+        return s;
+    if (h_stack && (s = cuda_check(cudaMemcpyAsync(h_stack, d.stack, sizeof(uint16_t) * (size_t)d.B * d.cap,
+                                                   cudaMemcpyDeviceToHost, cs),
+                                   "download stack")))
+        return s;
+    if (h_status && (s = cuda_check(cudaMemcpyAsync(h_status, d.status, sizeof(int32_t) * d.B, cudaMemcpyDeviceToHost, cs),
+                                    "download status")))
+        return s;
+    return cuda_check(cudaStreamSynchronize(cs), "cudaStreamSynchronize");
+}
+
+int32_t psc_host_classify(const psc_handle* h, int32_t q, const uint16_t* h_stack, int32_t depth, int32_t status) {
+    if (!h || (depth > 0 && !h_stack) || depth < 0) return -1;
+    for (int i = 0; i < depth; i++)
+        if (h_stack[i] >= h->t.n_lr) return -1;
+    return psc::classify_host(h->t, q, h_stack, depth, status);
+}
+
+psc_status psc_host_mask_row(const psc_handle* h, int32_t mask_id, uint32_t* h_row) {
+    if (!h || !h_row || mask_id < 0 || mask_id >= h->t.n_masks) return fail_with(PSC_ERR_ARG, "psc_host_mask_row: bad arguments");
+    std::memcpy(h_row, h->t.masks.data() + (size_t)mask_id * h->t.W, sizeof(uint32_t) * h->t.W);
+    return PSC_OK;
+}
+
+psc_status psc_host_advance(const psc_handle* h, int32_t* q, uint16_t* h_stack, int32_t* depth, int32_t cap,
+                            int32_t* status, int32_t tok) {
+    if (!h || !q || !h_stack || !depth || !status || cap < 2 || *depth < 1 || *depth > cap)
+        return fail_with(PSC_ERR_ARG, "psc_host_advance: bad arguments");
+    const psc::Tables& T = h->t;
+    if (tok < 0) return PSC_OK;
+    int st = *status;
+    if (st == ROW_DONE) {
+        *status = tok == T.eos_id ? ROW_DONE : ROW_REJECTED;
+        return PSC_OK;
+    }
+    if (st != ROW_OK) return PSC_OK;
+    if (tok >= T.V) {
+        *status = ROW_REJECTED;
+        return PSC_OK;
+    }
+    int mid = psc::classify_host(T, *q, h_stack, *depth, st);
+    if (mid < 0 || !((T.masks[(size_t)mid * T.W + (tok >> 5)] >> (tok & 31)) & 1)) {
+        *status = ROW_REJECTED;
+        return PSC_OK;
+    }
+    if (tok == T.eos_id) {
+        *status = ROW_DONE;
+        return PSC_OK;
+    }
+    int cq = *q, d = *depth;
+    for (int64_t i = T.vocab_off[tok]; i < T.vocab_off[tok + 1] && st == ROW_OK; i++) {
+        int c = T.vocab_bytes[i];
+        int nx = T.lex_trans[(size_t)cq * 256 + c];
+        if (nx >= 0) {
+            cq = nx;
+            continue;
+        }
+        int cls = cq == T.q0 ? -1 : T.lex_accept[cq];
+        if (cls < 0) {
+            st = ROW_REJECTED;
+            break;
+        }
+        if (!T.cls_ignored[cls]) st = host_feed(T, h_stack, d, cap, cls);
+        cq = T.lex_trans[(size_t)T.q0 * 256 + c];
+        if (cq < 0) st = ROW_REJECTED;
+    }
+    if (st == ROW_OK) {
+        *q = cq;
+        *depth = d;
+    }
+    *status = st;
+    return PSC_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,126 @@
+// Internal data structures of the PSC library (host side).
+//
+// The compile step (psc_compile) turns a grammar and a vocabulary into flat
+// tables: a byte-level lexer DFA (the lexing transducer of Section 2.2), LALR(1)
+// ACTION/GOTO tables (the deterministic push-down automaton of Section 2.4), the
+// stack classifier DFA built from every token's acceptance condition (Section
+// 3.5, Eq. 9, Algorithm 1), and the deduplicated vocabulary mask of every
+// classifier state (Section 3.5, the sets A_s).
+#pragma once
+
+#include <cstdint>
+#include <stdexcept>
+#include <string>
+#include <vector>
+
+namespace psc {
+
+// status codes shared with include/psc.h
+enum {
+    ST_OK = 0, ST_ERR_ARG = 1, ST_ERR_GRAMMAR = 2, ST_ERR_CONFLICT = 3, ST_ERR_LEXER_AMBIGUOUS = 4,
+    ST_ERR_LIMIT = 5, ST_ERR_OOM = 6, ST_ERR_CUDA = 7, ST_ERR_IO = 8
+};
+
+struct Error : std::runtime_error {
+    int code;
+    Error(int c, const std::string& m) : std::runtime_error(m), code(c) {}
+};
+
+// ---------------------------------------------------------------- grammar
+struct Terminal {
+    std::string name;      // display name; an anonymous literal is named by its quoted text
+    bool literal = false;
+    std::string pattern;   // literal bytes, or regex source
+    int priority = 0;
+    bool ignored = false;
+};
+
+struct Rule {
+    int lhs;                // nonterminal index
+    std::vector<int> rhs;   // symbol >= 0: terminal id; < 0: nonterminal ~index
+};
+
+struct Grammar {
+    std::vector<Terminal> terms;
+    std::vector<std::string> nts;
+    std::vector<Rule> rules;
+    int start_nt = -1;
+    bool contextual = false;
+};
+
+Grammar parse_grammar(const std::string& text);
+// rank[t]: order in which a lexeme matching several terminals prefers them
+// (higher priority first, then byte-wise ascending display name)
+std::vector<int> terminal_rank(const Grammar& g);
+
+// ------------------------------------------------------------------ lexer
+struct Lexer {
+    int nq = 0, q0 = 0;                       // q0: the empty pending lexeme
+    std::vector<int16_t> trans;               // [nq][256], -1: the byte ends the lexeme
+    std::vector<int32_t> accept_cls;          // [nq], class of a complete lexeme or -1
+    std::vector<std::vector<int>> classes;    // class id -> terminal ids in rank order
+    std::vector<uint8_t> class_ignored;
+    std::vector<std::vector<int>> tp;         // per state: T_p as class ids, -1 = empty sequence
+};
+
+Lexer build_lexer(const Grammar& g, const std::vector<int>& rank);
+
+// ----------------------------------------------------------------- parser
+enum { ACT_ERR = 0, ACT_SHIFT = 1, ACT_REDUCE = 2, ACT_ACCEPT = 3 };
+inline int32_t act_make(int kind, int v) { return (int32_t)((v << 2) | kind); }
+inline int act_kind(int32_t a) { return a & 3; }
+inline int act_val(int32_t a) { return a >> 2; }
+
+struct Parser {
+    int n_states = 0, n_terms = 0, n_nts = 0, end_term = 0;   // n_terms includes the end marker
+    std::vector<int32_t> action;      // [n_states][n_terms]
+    std::vector<int32_t> go;          // [n_states][n_nts], -1 = none
+    std::vector<int32_t> rule_len, rule_lhs;
+    std::vector<uint8_t> term_entered;  // state is entered by shifting a terminal (or is state 0)
+};
+
+Parser build_lalr(const Grammar& g);
+
+// ---------------------------------------------------------- compiled tables
+struct Options {
+    int64_t max_states = 4000000;     // classifier states before PSC_ERR_LIMIT
+    int64_t max_mask_bytes = int64_t(24) << 30;
+    int threads = 0;                  // 0 = hardware concurrency
+};
+
+struct Tables {
+    // lexer
+    int nq = 0, q0 = 0;
+    std::vector<int16_t> lex_trans;      // [nq][256]
+    std::vector<int32_t> lex_accept;     // [nq]
+    std::vector<uint8_t> cls_ignored;    // [n_classes]
+    int n_classes = 0;
+    // parser
+    int n_lr = 0, n_terms = 0, n_nts = 0, end_term = 0;
+    std::vector<int32_t> action, go, rule_len, rule_lhs;
+    std::vector<int16_t> resolve;        // [n_classes][n_lr]: terminal a class stands for, -1 none
+    bool contextual = false;
+    // classifier DFA over (lexer state, stack read from the top)
+    int S = 0;
+    std::vector<int32_t> dfa;            // [S][n_lr]: next state, or -(mask+1) when absorbing
+    std::vector<int32_t> dfa_start;      // [nq]: first state after reading q (same encoding)
+    std::vector<int32_t> dfa_mask;       // [S]: mask id when the stack ends in this state
+    // masks: row 0 = nothing allowed, row 1 = only the end-of-sequence token
+    int V = 0, W = 0, n_masks = 0;
+    std::vector<uint32_t> masks;         // [n_masks][W]
+    // vocabulary
+    std::vector<uint8_t> vocab_bytes;
+    std::vector<int64_t> vocab_off;      // [V+1]
+    int eos_id = -1;
+    // statistics
+    int64_t n_dfa_states_built = 0, n_threads = 0, n_trie_nodes = 0;
+    double seconds_lex = 0, seconds_dfa = 0, seconds_min = 0, seconds_total = 0;
+};
+
+Tables compile_tables(const std::string& grammar, const uint8_t* vocab_bytes, const int64_t* offsets,
+                      int V, int eos_id, const Options& opt);
+
+// host-side walk of the flattened classifier (inspection / tests): mask id of (q, stack)
+int classify_host(const Tables& t, int q, const uint16_t* stack, int depth, int status);
+
+}  // namespace psc

@@ -1,0 +1,333 @@
+"""GPU parity: the CUDA path (through the C ABI) against the CPU oracle.
+
+Masks, masked logits and advanced parser states must be bit-exact.  Configs 1-3
+are compared on every row and every token; configs 4 and 5 at full size in the
+launch configuration the benchmark uses, on sampled rows (all tokens) plus all
+rows on sampled tokens.
+"""
+from __future__ import annotations
+
+import os
+
+import numpy as np
+import pytest
+
+from oracle import ST_DONE, ST_ERROR, ST_OK, Oracle, Vocab
+from workloads import configs, grammars
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+THREADS = os.cpu_count() or 1
+
+
+@pytest.fixture(scope="module")
+def psc():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2608_03065_gb300 import build, psc as mod
+    build.build()
+    mod.load()
+    return mod
+
+
+class Case:
+    """A workload compiled on the device, with device states and oracle configs
+    advanced over the same prefix tokens."""
+
+    def __init__(self, psc, cfg_id, cap=256):
+        self.w = configs.load(cfg_id)
+        w = self.w
+        self.h = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id)
+        self.st = psc.psc_state_init(self.h, w.B, cap)
+        tm = torch.from_numpy(w.token_matrix()).cuda()
+        for j in range(tm.shape[1]):
+            psc.psc_advance(self.h, self.st, tm[:, j].contiguous())
+        torch.cuda.synchronize()
+        self.o = Oracle(w.grammar_text)
+        self.voc = Vocab.from_list(w.vocab, w.eos_id)
+        self.ocs = []
+        for ids in w.prefix_ids:
+            oc = self.o.initial()
+            self.o.advance_tokens(oc, self.voc, ids)
+            self.ocs.append(oc)
+
+
+_cases = {}
+
+
+def case(psc, cfg_id):
+    if cfg_id not in _cases:
+        _cases[cfg_id] = Case(psc, cfg_id)
+    return _cases[cfg_id]
+
+
+def bits_of(mask_np, V):
+    return np.unpackbits(mask_np.view(np.uint8), axis=-1, bitorder="little")[..., :V].astype(bool)
+
+
+def sampled_oracle(c: Case, rows, tokens):
+    """Oracle mask bits [len(rows)][len(tokens)] on a sub-vocabulary."""
+    toks = [c.w.vocab[t] for t in tokens]
+    eos_pos = [i for i, t in enumerate(tokens) if t == c.w.eos_id]
+    sub = Vocab.from_list(toks, eos_pos[0] if eos_pos else -1)
+    m = c.o.masks([c.ocs[r] for r in rows], sub, threads=THREADS)
+    return bits_of(m, len(tokens))
+
+
+def fill(psc, c):
+    out = torch.empty(c.w.B, c.h.W, dtype=torch.int32, device="cuda")
+    psc.psc_fill_mask(c.h, c.st, out)
+    torch.cuda.synchronize()
+    return out.cpu().numpy().view(np.uint32)
+
+
+def reference_masked(logits_cpu, allowed):
+    """where(allowed, logits, -inf) on raw bits."""
+    if logits_cpu.dtype == torch.bfloat16:
+        raw = logits_cpu.view(torch.int16).numpy().copy()
+        raw[~allowed] = np.int16(-128)        # 0xFF80
+    else:
+        raw = logits_cpu.view(torch.int32).numpy().copy()
+        raw[~allowed] = np.int32(-8388608)    # 0xFF800000
+    return raw
+
+
+def raw_bits(t):
+    t = t.cpu()
+    return t.view(torch.int16 if t.dtype == torch.bfloat16 else torch.int32).numpy()
+
+
+# --------------------------------------------------------------- full parity
+@pytest.mark.parametrize("cfg_id", [1, 2, 3])
+def test_fill_mask_bit_exact(psc, cfg_id):
+    c = case(psc, cfg_id)
+    dev = fill(psc, c)
+    ref = c.o.masks(c.ocs, c.voc, threads=THREADS)
+    assert dev.shape == ref.shape
+    bad = np.nonzero((dev != ref).any(axis=1))[0]
+    assert len(bad) == 0, f"rows {bad[:10]} differ"
+
+
+@pytest.mark.parametrize("cfg_id", [1, 2, 3])
+def test_apply_and_fused_bit_exact(psc, cfg_id):
+    c = case(psc, cfg_id)
+    ref_mask = c.o.masks(c.ocs, c.voc, threads=THREADS)
+    allowed = bits_of(ref_mask, c.w.V)
+    logits = c.w.logits()
+    want = reference_masked(logits, allowed)
+    # unfused: fill_mask then apply_mask
+    bm = torch.empty(c.w.B, c.h.W, dtype=torch.int32, device="cuda")
+    psc.psc_fill_mask(c.h, c.st, bm)
+    x = logits.cuda()
+    psc.psc_apply_mask(x, bm, c.w.B, c.w.V)
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(raw_bits(x), want)
+    # fused, with the bitmask copy
+    x2 = logits.cuda()
+    bm2 = torch.zeros_like(bm)
+    psc.psc_fill_apply(c.h, c.st, x2, bm2)
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(raw_bits(x2), want)
+    np.testing.assert_array_equal(bm2.cpu().numpy().view(np.uint32), ref_mask)
+
+
+@pytest.mark.parametrize("cfg_id", [1, 2, 3])
+def test_argmax_masked(psc, cfg_id):
+    c = case(psc, cfg_id)
+    allowed = bits_of(c.o.masks(c.ocs, c.voc, threads=THREADS), c.w.V)
+    logits = c.w.logits()
+    x = logits.cuda()
+    tok = torch.empty(c.w.B, dtype=torch.int32, device="cuda")
+    psc.psc_fill_apply(c.h, c.st, x)
+    psc.psc_argmax_masked(c.h, c.st, x, tok)
+    torch.cuda.synchronize()
+    lf = logits.float().numpy()
+    for b in range(c.w.B):
+        idx = np.nonzero(allowed[b])[0]
+        want = -1 if len(idx) == 0 else int(idx[np.argmax(lf[b, idx])])
+        assert int(tok[b]) == want, b
+
+
+# ------------------------------------------------------ large configs, sampled
+@pytest.mark.parametrize("cfg_id", [4, 5])
+def test_large_config_fused_sampled(psc, cfg_id):
+    c = case(psc, cfg_id)
+    B, V = c.w.B, c.w.V
+    rng = np.random.default_rng(cfg_id)
+    logits = c.w.logits()
+    x = logits.cuda()
+    bm = torch.zeros(B, c.h.W, dtype=torch.int32, device="cuda")
+    psc.psc_fill_apply(c.h, c.st, x, bm)
+    torch.cuda.synchronize()
+    dev_mask = bm.cpu().numpy().view(np.uint32)
+    dev_bits = bits_of(dev_mask, V)
+    # whole rows
+    rows = sorted(rng.choice(B, size=min(24, B), replace=False).tolist())
+    ref_rows = c.o.masks([c.ocs[r] for r in rows], c.voc, threads=THREADS)
+    np.testing.assert_array_equal(dev_mask[rows], ref_rows)
+    # all rows, sampled tokens
+    toks = sorted(set(rng.choice(V, size=1500, replace=False).tolist()) | {c.w.eos_id})
+    ref = sampled_oracle(c, list(range(B)), toks)
+    np.testing.assert_array_equal(dev_bits[:, toks], ref)
+    # masked logits on the sampled rows (fused path output)
+    got = raw_bits(x)
+    want = reference_masked(logits[rows], dev_bits[rows])
+    np.testing.assert_array_equal(got[rows], want)
+
+
+# ------------------------------------------------------------- decode loop
+@pytest.mark.parametrize("cfg_id,steps", [(2, 6), (5, 4)])
+def test_decode_loop_advance(psc, cfg_id, steps):
+    """fill_apply -> argmax -> advance for several steps; after every step the
+    device masks equal the oracle's after advancing it by the same tokens
+    (runs after the other tests of the same workload: it advances its states)."""
+    c = case(psc, cfg_id)
+    B, V = c.w.B, c.w.V
+    rng = np.random.default_rng(10 + cfg_id)
+    rows = list(range(B)) if B <= 64 else sorted(rng.choice(B, size=16, replace=False).tolist())
+    tok = torch.empty(B, dtype=torch.int32, device="cuda")
+    stat = torch.empty(B, dtype=torch.int32, device="cuda")
+    for step in range(steps):
+        x = c.w.logits(step + 1).cuda()
+        bm = torch.zeros(B, c.h.W, dtype=torch.int32, device="cuda")
+        psc.psc_fill_apply(c.h, c.st, x, bm)
+        psc.psc_argmax_masked(c.h, c.st, x, tok)
+        torch.cuda.synchronize()
+        dev_mask = bm.cpu().numpy().view(np.uint32)
+        ref = c.o.masks([c.ocs[r] for r in rows], c.voc, threads=THREADS)
+        np.testing.assert_array_equal(dev_mask[rows], ref)
+        psc.psc_advance(c.h, c.st, tok, stat)
+        torch.cuda.synchronize()
+        t = tok.cpu().numpy()
+        s = stat.cpu().numpy()
+        for r in rows:
+            if t[r] < 0:
+                continue
+            ost = c.o.advance(c.ocs[r], None if t[r] == c.w.eos_id else c.w.vocab[t[r]])
+            want = {ST_OK: psc.ROW_OK, ST_DONE: psc.ROW_DONE, ST_ERROR: psc.ROW_REJECTED}[ost]
+            assert s[r] == want, (step, r)
+
+
+# ---------------------------------------------------------------- edge cases
+def _small_vocab(n=1000, seed=0):
+    rng = np.random.default_rng(seed)
+    toks = {bytes([b]) for b in range(0x20, 0x7F)}
+    alphabet = b"0123456789abcxyz+-*/() "
+    while len(toks) < n - 1:
+        k = int(rng.integers(2, 6))
+        toks.add(bytes(alphabet[int(i)] for i in rng.integers(0, len(alphabet), k)))
+    return sorted(toks) + [b""]
+
+
+def test_ragged_vocab_unaligned_rows_and_statuses(psc):
+    """V = 1000 (not a multiple of 32 or 1024), odd row strides (element path),
+    rejected / finished / overflowed rows."""
+    g = grammars.arithmetic().text()
+    toks = _small_vocab()
+    V, eos = len(toks), len(toks) - 1
+    h = psc.psc_compile(g, toks, eos)
+    o = Oracle(g)
+    voc = Vocab.from_list(toks, eos)
+    idx = {t: i for i, t in enumerate(toks)}
+    prefixes = [b"", b"(1+", b"((((((((a", b"12*x", b"1", b"(", b")", b"((((((((((((((((((((((((1"]
+    B, cap = len(prefixes), 16
+    st = psc.psc_state_init(h, B, cap)
+    ocs = []
+    for b, p in enumerate(prefixes):
+        oc = o.initial()
+        for ch in p:
+            o.advance(oc, bytes([ch]))
+        ocs.append(oc)
+    T = max(len(p) for p in prefixes)
+    tm = np.full((B, T), -1, dtype=np.int32)
+    for b, p in enumerate(prefixes):
+        for j, ch in enumerate(p):
+            tm[b, j] = idx[bytes([ch])]
+    stat = torch.empty(B, dtype=torch.int32, device="cuda")
+    tmd = torch.from_numpy(tm).cuda()
+    for j in range(T):
+        psc.psc_advance(h, st, tmd[:, j].contiguous(), stat)
+    # row 4 finishes with EOS; row 7 overflows the 16-entry stack
+    psc.psc_advance(h, st, torch.tensor([-1, -1, -1, -1, eos, -1, -1, -1], dtype=torch.int32, device="cuda"), stat)
+    o.advance(ocs[4], None)
+    info = psc.psc_states_download(st)
+    assert info["status"][6] == psc.ROW_REJECTED           # ")" at the start
+    assert info["status"][4] == psc.ROW_DONE
+    assert info["status"][7] == psc.ROW_OVERFLOW
+    ref = o.masks(ocs, voc)
+    ref[7] = 0                                              # the oracle has no capacity limit
+    bm = torch.empty(B, h.W, dtype=torch.int32, device="cuda")
+    psc.psc_fill_mask(h, st, bm)
+    np.testing.assert_array_equal(bm.cpu().numpy().view(np.uint32), ref)
+    allowed = bits_of(ref, V)
+    for dt in (torch.float32, torch.bfloat16):
+        for stride in (V, V + 3, 1024):
+            base = torch.randn(B, stride, generator=torch.Generator().manual_seed(stride)).to(dt)
+            x = base.cuda()
+            psc.psc_fill_apply(h, st, x[:, :V] if stride == V else x, None, V=V)
+            torch.cuda.synchronize()
+            want = reference_masked(base[:, :V].contiguous(), allowed)
+            got = raw_bits(x)
+            np.testing.assert_array_equal(got[:, :V], want)
+            np.testing.assert_array_equal(got[:, V:], raw_bits(base)[:, V:])   # columns >= V untouched
+    tok = torch.empty(B, dtype=torch.int32, device="cuda")
+    x = torch.randn(B, V).cuda()
+    psc.psc_argmax_masked(h, st, x, tok)
+    t = tok.cpu().numpy()
+    assert t[6] == -1 and t[7] == -1 and t[4] == eos
+
+
+def test_nan_payloads_and_infinities_kept(psc):
+    """Allowed logits keep their exact bits (NaN payloads, infinities, denormals),
+    on the 16-byte vector path and on the element path."""
+    g = grammars.json_grammar().text()
+    singles = [bytes([b]) for b in range(0x20, 0x7F)]
+    toks = singles + [a + b for a in singles[:40] for b in singles[:40]][:2000] + [b"true", b"false", b""]
+    V = len(toks)
+    h = psc.psc_compile(g, toks, V - 1)
+    st = psc.psc_state_init(h, 2, 32)
+    psc.psc_advance(h, st, torch.tensor([toks.index(b"["), -1], dtype=torch.int32, device="cuda"))
+    bm = torch.empty(2, h.W, dtype=torch.int32, device="cuda")
+    psc.psc_fill_mask(h, st, bm)
+    allowed = bits_of(bm.cpu().numpy().view(np.uint32), V)
+    pattern = np.array([0x7FC00001, 0x7F800000, -8388608, 0x00000001, 0x7FBFFFFF], dtype=np.int64)
+    for stride in (2048 + 8, V + 1):
+        raw = np.resize(pattern, (2, stride)).astype(np.int32)
+        x = torch.from_numpy(raw.copy()).cuda().view(torch.float32)
+        psc.psc_fill_apply(h, st, x, None, V=V)
+        got = x.cpu().view(torch.int32).numpy()
+        want = raw.copy()
+        want[:, :V][~allowed] = np.int32(-8388608)
+        np.testing.assert_array_equal(got, want)
+
+
+def test_state_reset_rows(psc):
+    c = case(psc, 2)
+    rows = torch.tensor([0, 3, 5], dtype=torch.int32, device="cuda")
+    h, w = c.h, c.w
+    st = psc.psc_state_init(h, w.B, 256)
+    tm = torch.from_numpy(w.token_matrix()).cuda()
+    for j in range(tm.shape[1]):
+        psc.psc_advance(h, st, tm[:, j].contiguous())
+    psc.psc_state_reset(st, rows)
+    info = psc.psc_states_download(st)
+    for r in (0, 3, 5):
+        assert info["depth"][r] == 1 and info["q"][r] == 0 and info["status"][r] == psc.ROW_OK
+    dev = torch.empty(w.B, h.W, dtype=torch.int32, device="cuda")
+    psc.psc_fill_mask(h, st, dev)
+    m0 = c.o.masks([c.o.initial()], c.voc)[0]
+    for r in (0, 3, 5):
+        np.testing.assert_array_equal(dev[r].cpu().numpy().view(np.uint32), m0)
+
+
+def test_bad_arguments_are_reported(psc):
+    c = case(psc, 1)
+    lib = psc.load()
+    x = torch.zeros(c.w.B, c.w.V, device="cuda")
+    bm = torch.zeros(c.w.B, c.h.W, dtype=torch.int32, device="cuda")
+    assert lib.psc_fill_apply(c.h.ptr, c.st.ptr, c.w.B + 1, x.data_ptr(), 0, c.w.V, c.w.V, None, None) == 1
+    assert lib.psc_apply_mask(x.data_ptr(), 0, c.w.V - 1, bm.data_ptr(), c.w.B, c.w.V, None) == 1
+    assert lib.psc_apply_mask(x.data_ptr(), 7, c.w.V, bm.data_ptr(), c.w.B, c.w.V, None) == 1
+    assert lib.psc_fill_mask(c.h.ptr, c.st.ptr, c.w.B, None, None) == 1
+    assert b"bad arguments" in lib.psc_last_error()

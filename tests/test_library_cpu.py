@@ -1,0 +1,140 @@
+"""CPU-side tests of the library: it loads, exports every symbol the header
+declares, reports grammar errors, and its compiled host tables give the
+oracle's masks (a walk of the same flattened tables the GPU reads)."""
+from __future__ import annotations
+
+import os
+import re
+
+import numpy as np
+import pytest
+
+from oracle import Oracle, Vocab
+from workloads import configs, grammars
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="session")
+def psc():
+    from paper_2608_03065_gb300 import build, psc as mod
+    build.build()
+    mod.load()
+    return mod
+
+
+def _header_symbols():
+    text = open(os.path.join(ROOT, "include", "psc.h")).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(psc_[a-z_]+)\s*\(", text)))
+
+
+def test_library_exports_every_declared_symbol(psc):
+    lib = psc.load()
+    syms = _header_symbols()
+    assert len(syms) >= 16
+    for s in syms:
+        assert hasattr(lib, s), s
+    assert set(syms) == set(psc.EXPORTED)
+
+
+def _host_cfg(h, ids):
+    c = h.host_initial()
+    for v in ids:
+        c = h.host_advance(c, v)
+    return c
+
+
+def _host_mask(h, c):
+    return h.host_mask_row(h.host_classify(c["q"], c["stack"], c["status"]))
+
+
+@pytest.mark.parametrize("cfg_id,batch", [(1, 8), (2, 24), (3, 6)])
+def test_host_tables_match_oracle(psc, cfg_id, batch):
+    w = configs.load(cfg_id, batch=batch)
+    h = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id, host_only=True)
+    o = Oracle(w.grammar_text)
+    voc = Vocab.from_list(w.vocab, w.eos_id)
+    cfgs, ocs = [], []
+    for ids in w.prefix_ids:
+        cfgs.append(_host_cfg(h, ids))
+        oc = o.initial()
+        o.advance_tokens(oc, voc, ids)
+        ocs.append(oc)
+    om = o.masks(ocs, voc)
+    for b, c in enumerate(cfgs):
+        assert c["status"] == psc.ROW_OK
+        np.testing.assert_array_equal(_host_mask(h, c), om[b], err_msg=f"row {b}")
+
+
+def test_host_tables_deep_parentheses(psc):
+    """Balanced parentheses to depth 200: the classifier walk reads deep stacks."""
+    g = 'start: s\ns: | s "(" s ")"\n'
+    toks = [b"(", b")", b"((", b"))", b"()", b")(", b"())", b""]
+    h = psc.psc_compile(g, toks, 7, host_only=True)
+    o = Oracle(g)
+    voc = Vocab.from_list(toks, 7)
+    c, oc = h.host_initial(), o.initial()
+    for d in range(200):
+        c = h.host_advance(c, 0, cap=512)       # two stack entries per level
+        o.advance(oc, b"(")
+        if d % 37 == 0 or d == 199:
+            np.testing.assert_array_equal(_host_mask(h, c), o.masks([oc], voc)[0])
+    for d in range(200):
+        c = h.host_advance(c, 1, cap=512)
+        o.advance(oc, b")")
+    np.testing.assert_array_equal(_host_mask(h, c), o.masks([oc], voc)[0])
+    assert (_host_mask(h, c)[0] >> 7) & 1   # end of sequence allowed at depth 0
+
+
+def test_host_advance_statuses(psc):
+    g = grammars.json_grammar().text()
+    toks = [b"{", b"}", b"1", b" ", b'"a"', b":", b""]
+    h = psc.psc_compile(g, toks, 6, host_only=True)
+    c = h.host_initial()
+    c = h.host_advance(c, 0)
+    assert c["status"] == psc.ROW_OK
+    c2 = h.host_advance(c, 2)                  # "{1" is not JSON
+    assert c2["status"] == psc.ROW_REJECTED
+    assert h.host_classify(c2["q"], c2["stack"], c2["status"]) == 0
+    c = h.host_advance(c, 1)
+    c = h.host_advance(c, 6)                   # end of sequence after "{}"
+    assert c["status"] == psc.ROW_DONE
+    assert h.host_classify(c["q"], c["stack"], c["status"]) == 1
+    row = h.host_mask_row(1)
+    assert row[0] == 1 << 6
+    assert h.host_advance(c, 6)["status"] == psc.ROW_DONE
+    assert h.host_advance(c, 0)["status"] == psc.ROW_REJECTED
+    # stack overflow at a small capacity
+    arr = psc.psc_compile('start: s\ns: | s "(" s ")"\n', [b"(", b")", b""], 2, host_only=True)
+    c = arr.host_initial()
+    for _ in range(10):
+        c = arr.host_advance(c, 0, cap=8)
+    assert c["status"] == psc.ROW_OVERFLOW
+
+
+@pytest.mark.parametrize("text,code", [
+    ('start: a | b\na: "x"\nb: "x"\n', 3),                                  # reduce/reduce conflict
+    ('start: "x" | "x" "y"\nstart2: FOO\n', 2),                             # unknown terminal
+    ('start: NAME\nNAME: /[a-z]+/\nKW: "if"\nWS: /if/\n%ignore WS\n', 4),   # ignored and kept collide
+    ('start: A\nA: /x*/\n', 2),                                            # terminal matches empty
+    ('nostart: "x"\n', 2),
+])
+def test_grammar_errors(psc, text, code):
+    with pytest.raises(psc.PscError) as e:
+        psc.psc_compile(text, [b"x", b""], 1, host_only=True)
+    assert e.value.code == code, str(e.value)
+
+
+def test_state_limit(psc):
+    w = configs.load(2, batch=1)
+    with pytest.raises(psc.PscError) as e:
+        psc.psc_compile(w.grammar_text, w.vocab, w.eos_id, host_only=True, max_states=50)
+    assert e.value.code == 5
+
+
+def test_device_calls_refuse_host_only_handle(psc):
+    h = psc.psc_compile(grammars.arithmetic().text(), [b"1", b""], 1, host_only=True)
+    with pytest.raises(psc.PscError) as e:
+        psc.psc_state_init(h, 4, 16, stream=0)
+    assert e.value.code == 1
