@@ -195,6 +195,37 @@ psc_status psc_host_mask_row(const psc_handle* h, int32_t mask_id, uint32_t* h_r
 psc_status psc_host_advance(const psc_handle* h, int32_t* q, uint16_t* h_stack, int32_t* depth, int32_t cap,
                             int32_t* status, int32_t token);
 
+/* Allocation-free variant of psc_fill_apply.  The paper has no counterpart:
+ * this entry point exists for callers that cannot allocate device memory at
+ * the point where they apply the mask, for example code running while a
+ * stream is being captured into a CUDA graph (cudaMalloc is not allowed
+ * there), code inside a framework whose allocator owns all device memory, or
+ * latency-critical loops where an allocation could synchronise the device.
+ *
+ * It does exactly what psc_fill_apply does, but the parser configurations
+ * come from caller-owned device arrays instead of a psc_states object, and the
+ * per-row mask ids it needs between the classifier walk and the masking pass
+ * live in one library-owned scratch array of PSC_NOALLOC_MAX_ROWS int32 that
+ * is part of the loaded module (a file-scope __device__ array, 64 KiB, held by
+ * every GPU that loads the library until the process exits).  Nothing is
+ * allocated or freed by the call.
+ *   d_q, d_depth, d_status : device int32 [B] (lexer state, stack depth, row status)
+ *   d_stack                : device uint16 [B][cap], bottom first (the layout psc_states_download returns)
+ *   other arguments        : as for psc_fill_apply
+ * Errors: PSC_ERR_LIMIT when B > PSC_NOALLOC_MAX_ROWS; PSC_ERR_ARG for bad arguments.
+ * The first call on a device looks up the scratch array's device address
+ * (cudaGetSymbolAddress) with that device current; make that first call
+ * before any stream capture.  Every call shares the same scratch array, which
+ * keeps the last call's contents (each call writes every entry it reads, so
+ * nothing needs clearing); calls that overlap on the GPU (different streams,
+ * or host threads racing on one device) race on it and must be serialised by
+ * the caller. */
+#define PSC_NOALLOC_MAX_ROWS 16384
+psc_status psc_fill_apply_noalloc(const psc_handle* h, const int32_t* d_q, const int32_t* d_depth,
+                                  const int32_t* d_status, const uint16_t* d_stack, int32_t cap, int32_t B,
+                                  void* d_logits, psc_dtype dtype, int64_t row_stride, int32_t V,
+                                  uint32_t* d_bitmask_out, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -19,6 +19,7 @@
 #include <algorithm>
 #include <cstring>
 #include <memory>
+#include <mutex>
 #include <new>
 #include <string>
 
@@ -545,6 +546,29 @@ int host_feed(const psc::Tables& T, uint16_t* st, int& depth, int cap, int cls) 
 
 }  // namespace
 
+// Scratch of psc_fill_apply_noalloc: per-row mask ids between the classifier
+// walk and the masking pass, in the module itself so the call allocates nothing.
+static __device__ __align__(256) int32_t g_noalloc_mid[PSC_NOALLOC_MAX_ROWS];
+
+namespace {
+std::mutex g_noalloc_mu;
+int32_t* g_noalloc_ptr[256] = {};
+
+// Device address of g_noalloc_mid on the current device (looked up once per device).
+psc_status noalloc_scratch(int device, int32_t** out) {
+    if (device < 0 || device >= 256) return fail_with(PSC_ERR_ARG, "psc_fill_apply_noalloc: bad device id");
+    std::lock_guard<std::mutex> lk(g_noalloc_mu);
+    if (!g_noalloc_ptr[device]) {
+        void* p = nullptr;
+        psc_status s = cuda_check(cudaGetSymbolAddress(&p, g_noalloc_mid), "cudaGetSymbolAddress(scratch)");
+        if (s != PSC_OK) return s;
+        g_noalloc_ptr[device] = static_cast<int32_t*>(p);
+    }
+    *out = g_noalloc_ptr[device];
+    return PSC_OK;
+}
+}  // namespace
+
 // ====================================================================== ABI
 extern "C" {
 
@@ -851,6 +875,31 @@ psc_status psc_host_advance(const psc_handle* h, int32_t* q, uint16_t* h_stack, 
     }
     *status = st;
     return PSC_OK;
+}
+
+psc_status psc_fill_apply_noalloc(const psc_handle* h, const int32_t* d_q, const int32_t* d_depth,
+                                  const int32_t* d_status, const uint16_t* d_stack, int32_t cap, int32_t B,
+                                  void* d_logits, psc_dtype dtype, int64_t row_stride, int32_t V,
+                                  uint32_t* d_bitmask_out, void* stream) {
+    psc_status s = check_device(h, "psc_fill_apply_noalloc");
+    if (s != PSC_OK) return s;
+    if (B > PSC_NOALLOC_MAX_ROWS)
+        return fail_with(PSC_ERR_LIMIT, "psc_fill_apply_noalloc: B = " + std::to_string(B) +
+                                            " exceeds PSC_NOALLOC_MAX_ROWS = " + std::to_string(PSC_NOALLOC_MAX_ROWS));
+    if (B <= 0 || !d_q || !d_depth || !d_status || !d_stack || cap < 2 || !d_logits || V != h->d.V ||
+        row_stride < V || (dtype != PSC_F32 && dtype != PSC_BF16))
+        return fail_with(PSC_ERR_ARG, "psc_fill_apply_noalloc: bad arguments");
+    int32_t* mid = nullptr;
+    if ((s = noalloc_scratch(h->device, &mid)) != PSC_OK) return s;
+    DevStates S{const_cast<int32_t*>(d_q), const_cast<int32_t*>(d_depth), const_cast<int32_t*>(d_status),
+                const_cast<uint16_t*>(d_stack), mid, B, cap};
+    cudaStream_t cs = (cudaStream_t)stream;
+    int threads = 256;
+    int blocks = (int)(((size_t)B * 32 + threads - 1) / threads);
+    k_classify<<<blocks, threads, 0, cs>>>(h->d, S, B);
+    if ((s = launch_check("k_classify")) != PSC_OK) return s;
+    MaskSrc M{nullptr, h->d.masks, mid, h->d.W, h->d.Wp, d_bitmask_out};
+    return launch_apply(d_logits, dtype, row_stride, M, B, V, cs, h->device);
 }
 
 }  // extern "C"

@@ -25,7 +25,8 @@ STATUS_NAMES = {0: "PSC_OK", 1: "PSC_ERR_ARG", 2: "PSC_ERR_GRAMMAR", 3: "PSC_ERR
 EXPORTED = ["psc_compile", "psc_destroy", "psc_last_error", "psc_info", "psc_state_init", "psc_state_reset",
             "psc_state_destroy", "psc_advance", "psc_fill_mask", "psc_apply_mask", "psc_fill_apply",
             "psc_argmax_masked", "psc_states_download", "psc_host_classify", "psc_host_mask_row",
-            "psc_host_advance"]
+            "psc_host_advance", "psc_fill_apply_noalloc"]
+NOALLOC_MAX_ROWS = 16384
 
 
 class PscError(RuntimeError):
@@ -76,6 +77,7 @@ def load(path: str = LIB_PATH):
         "psc_host_classify": (i32, [vp, i32, vp, i32, i32]),
         "psc_host_mask_row": (i32, [vp, i32, vp]),
         "psc_host_advance": (i32, [vp, vp, vp, vp, i32, vp, i32]),
+        "psc_fill_apply_noalloc": (i32, [vp, vp, vp, vp, vp, i32, i32, vp, i32, i64, i32, vp, vp]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -286,3 +288,21 @@ def psc_states_download(st: States, stream=None) -> dict:
     _check(load().psc_states_download(st.ptr, q.ctypes.data, depth.ctypes.data, stack.ctypes.data,
                                       status.ctypes.data, _stream(stream)))
     return {"q": q, "depth": depth, "stack": stack, "status": status}
+
+
+def psc_fill_apply_noalloc(h: Handle, q, depth, status, stack, logits, bitmask_out=None, V: int | None = None,
+                           stream=None):
+    """psc_fill_apply on caller-owned state arrays (q, depth, status int32 [B];
+    stack uint16 [B][cap] as a torch int16/uint16 tensor); allocates nothing."""
+    import torch
+    B = q.numel()
+    V = h.V if V is None else V
+    if stack.dim() != 2 or stack.shape[0] != B or not stack.is_contiguous() or stack.element_size() != 2:
+        raise ValueError("stack must be a contiguous [B, cap] 16-bit tensor")
+    if logits.shape[0] != B or logits.shape[1] < V:
+        raise ValueError("logits must be [B, >=V]")
+    _check(load().psc_fill_apply_noalloc(h.ptr, _ptr(q, torch.int32, "q"), _ptr(depth, torch.int32, "depth"),
+                                         _ptr(status, torch.int32, "status"), _ptr(stack, None, "stack"),
+                                         stack.shape[1], B, _ptr(logits, None, "logits"), _dtype_code(logits),
+                                         _row_stride(logits), V, _ptr(bitmask_out, torch.int32, "bitmask_out"),
+                                         _stream(stream)))
