@@ -1,11 +1,11 @@
 """Benchmark: masked decode steps on the 1024 x 262,144 C-like workload.
 
-One step = one pass of the whole per-step path over the batch:
-  psc_fill_apply     classify every row's parser stack (classifier DFA walk) and
-                     apply its precomputed mask to the bf16 logits in place, also
-                     writing the packed bitmask [B][V/32]
-  psc_argmax_masked  greedy choice among the allowed tokens
-  psc_advance        lex + parse the chosen tokens on the device-resident stacks
+One step = one pass of the whole per-step path over the batch, psc_decode_step:
+  k_apply_argmax   classify every row's parser stack (classifier DFA walk, inside
+                   the kernel), apply its precomputed mask to the bf16 logits in
+                   place, write the packed bitmask [B][V/32], and pick the greedy
+                   token among the allowed ones, in one pass over the logits
+  k_advance_smem   lex + parse the chosen tokens on the device-resident stacks
 
 Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
 For N > 1 launch with torch.distributed.run: every rank runs an independent
@@ -33,7 +33,7 @@ sys.path.insert(0, ROOT)
 WORKLOAD = 5
 METRIC = "masked decode steps/s and µs/step at batch×vocab; HBM GB/s vs GB300 peak"
 UNIT = "steps/s"
-PROFILE_FILE = os.path.join(ROOT, "profiles", "fused_fill_apply_c5_traffic.txt")
+PROFILE_FILE = os.path.join(ROOT, "profiles", "k_apply_argmax_c5_traffic.txt")
 
 
 def measured_peaks():
@@ -189,7 +189,7 @@ def run_reference(args):
 
 def config_block(w, n):
     return {"workload": f"config 5: C-like grammar, vocab {w.V}, batch {w.B}, bf16 logits ~N(0,2), "
-                        "decode steps fill_apply+argmax+advance",
+                        "decode steps (mask+apply+greedy+advance)",
             "batch": w.B, "vocab": w.V, "logit_dtype": "bf16", "grammar": "synthetic C-like (150 rules)",
             "parallelism": f"replicas x{n}", "l2": "inputs larger than L2 (512 MiB logits per step)"}
 
@@ -265,11 +265,9 @@ def main():
         x = bufs[i]
         if timed is not None:
             ev[timed][0].record(stream)
-        psc.psc_fill_apply(h, st, x, bitmask, stream=stream)
+        psc.psc_decode_step(h, st, x, tok, bitmask, stat, stream=stream)
         if timed is not None:
             ev[timed][1].record(stream)
-        psc.psc_argmax_masked(h, st, x, tok, stream=stream)
-        psc.psc_advance(h, st, tok, stat, stream=stream)
 
     for i in range(Wm):
         step(i)
@@ -313,9 +311,7 @@ def main():
     e0.record(stream)
     for i in range(K):
         dbuf.copy_(host[i % n_host], non_blocking=True)
-        psc.psc_fill_apply(h, st, dbuf, bitmask, stream=stream)
-        psc.psc_argmax_masked(h, st, dbuf, tok, stream=stream)
-        psc.psc_advance(h, st, tok, stat, stream=stream)
+        psc.psc_decode_step(h, st, dbuf, tok, bitmask, stat, stream=stream)
         tok_host.copy_(tok, non_blocking=True)
     e1.record(stream)
     torch.cuda.synchronize()
@@ -351,17 +347,17 @@ def main():
         "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "u32", "data": "synthetic", "config": config_block(w, world),
         "us_per_step": ms_per_step * 1000.0,
-        "fused_fill_apply_us": fused_avg_ms * 1000.0,
-        "fused_fill_apply_hbm_gbs": achieved,
+        "decode_step_us": fused_avg_ms * 1000.0,
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "traffic": traffic,
-                     "kernel": "psc_fill_apply (classify walk + fused mask apply + bitmask copy)",
+                     "kernel": "psc_decode_step (k_apply_argmax with in-kernel classification + k_advance_smem)",
                      "algorithmic_bytes": alg_bytes, "peak_kind": peak_kind},
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": B * V * 2,
                 "d2h_bytes_per_step": B * 4},
-        "gpu_launches": 4 * K,
+        "gpu_launches": 2 * K,
         "clocks": clocks.summary(),
         "cpu_baseline": cpu,
+        "device_timeouts": h.info().device_timeouts,
         "tables": {"classifier_states": info.n_classifier_states, "masks": info.n_masks,
                    "classifier_bytes": info.classifier_bytes, "mask_bytes": info.mask_bytes,
                    "compile_seconds": compile_s},

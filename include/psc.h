@@ -70,6 +70,8 @@ typedef struct {
     int64_t max_mask_bytes;  /* host bytes of distinct mask rows before PSC_ERR_LIMIT (0 = 24 GiB) */
     int32_t threads;         /* host threads for compilation (0 = all cores) */
     int32_t host_only;       /* 1: build host tables only (no GPU needed; device calls fail) */
+    int32_t global_tables;   /* 1: psc_advance reads its tables from global memory even when they
+                                would fit in shared memory (0 = stage them when they fit) */
 } psc_options;
 
 typedef struct {
@@ -84,6 +86,9 @@ typedef struct {
     int64_t mask_bytes;        /* device bytes of the mask rows (cf. Table 7, masks) */
     int64_t states_built;      /* classifier states before minimisation */
     double compile_seconds;
+    int64_t advance_table_bytes;  /* bytes psc_advance stages in shared memory (0: it reads global memory) */
+    int64_t device_timeouts;      /* bounded in-kernel waits that gave up since the library was loaded
+                                     (process-wide; non-zero means a pipeline fault; reading it synchronises) */
 } psc_info_t;
 
 /* Offline construction (Algorithm 1, Section 3).  Reads the grammar text (a
@@ -108,6 +113,18 @@ psc_status psc_compile(const char* grammar, size_t grammar_len, const uint8_t* v
 /* Frees the handle's host and device tables (NULL is a no-op).  No call that
  * uses the handle may still be running on any stream. */
 void psc_destroy(psc_handle* h);
+
+/* Writes the handle's compiled tables to a binary file (the paper ships its
+ * preprocessing results to decoding users as files, Section 5).  The file holds
+ * the lexer, parser, classifier and mask tables and the vocabulary, with a
+ * checksum.  Errors: PSC_ERR_IO, PSC_ERR_ARG. */
+psc_status psc_save(const psc_handle* h, const char* path);
+
+/* Reads a file written by psc_save, checks its checksum and the consistency of
+ * every table index, and uploads the tables to the current device (unless
+ * opts->host_only; opts may be NULL).  Errors: PSC_ERR_IO (missing, truncated,
+ * corrupt or inconsistent file), PSC_ERR_OOM, PSC_ERR_CUDA. */
+psc_status psc_load(const char* path, const psc_options* opts, psc_handle** out);
 
 /* Thread-local message of the last failed call on this thread ("" if none). */
 const char* psc_last_error(void);
@@ -174,6 +191,30 @@ psc_status psc_fill_apply(const psc_handle* h, const psc_states* st, int32_t B, 
 psc_status psc_argmax_masked(const psc_handle* h, const psc_states* st, int32_t B, const void* d_logits,
                              psc_dtype dtype, int64_t row_stride, int32_t V, int32_t* d_tokens,
                              void* stream);
+
+/* psc_fill_apply and psc_argmax_masked in one pass over the logits: every
+ * 16-byte chunk is touched once (written with -inf when fully masked, read
+ * when it holds an allowed position, read and rewritten when mixed) and the
+ * greedy choice among allowed tokens is merged per row with a 64-bit atomic
+ * maximum (value order, then the lowest index).  d_tokens[b] = chosen token or
+ * -1 when row b allows nothing; d_bitmask_out as in psc_fill_apply.  The
+ * per-row keys live in the states object; calls on the same states object
+ * must not overlap. */
+psc_status psc_fill_apply_argmax(const psc_handle* h, const psc_states* st, int32_t B, void* d_logits,
+                                 psc_dtype dtype, int64_t row_stride, int32_t V, uint32_t* d_bitmask_out,
+                                 int32_t* d_tokens, void* stream);
+
+/* One whole decoding step on the device (Algorithm 2 steps 1-4 plus masking and
+ * greedy sampling), in two kernels: the masking pass classifies every row's
+ * stack inside the kernel, applies the mask to the logits in place, writes
+ * the optional bitmask copy and picks the greedy token per row; the advance
+ * kernel then feeds that token to the row's lexer and parser.
+ *   d_tokens      : device int32 [B]; receives the chosen tokens (-1 = nothing allowed)
+ *   d_row_status  : optional device int32 [B] statuses after the step
+ * Other arguments as for psc_fill_apply_argmax. */
+psc_status psc_decode_step(const psc_handle* h, psc_states* st, int32_t B, void* d_logits, psc_dtype dtype,
+                           int64_t row_stride, int32_t V, uint32_t* d_bitmask_out, int32_t* d_tokens,
+                           int32_t* d_row_status, void* stream);
 
 /* Copies the batch to host memory and synchronises the stream (tests and
  * debugging).  Any output pointer may be NULL.

@@ -11,9 +11,10 @@
 //
 // Memory layout on the device (all tables uploaded once by psc_compile):
 //   dfa      int32 [S][n_lr]      next classifier state, or -(mask+1) when absorbing
-//   masks    uint32 [n_masks][Wp] mask rows, Wp = W rounded up to 4 words (16-byte rows)
+//   masks    uint32 [n_masks][Wp] mask rows, Wp = W rounded up to 32 words (whole 1024-column chunks)
 //   stacks   uint16 [B][cap]      parser stacks, bottom first; depth[b] entries used
 //   logits   [B][row_stride]      bf16 or f32, caller-owned, masked in place
+#include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
 #include <algorithm>
@@ -55,6 +56,9 @@ struct DevTables {
     const int64_t* vocab_off;
     int q0, nq, n_lr, n_terms, n_nts, end_term;
     int V, W, Wp, eos_id, n_masks;
+    // compact lexer/parser tables for k_advance_smem (adv_bytes = 0: not built)
+    const uint8_t* adv;
+    int adv_bytes, o_bc, o_trans, o_accept, o_ign, o_resolve, o_action, o_go, o_rlen, o_rlhs, nbc;
 };
 
 struct DevStates {
@@ -64,6 +68,7 @@ struct DevStates {
     uint16_t* stack;
     int32_t* mid;
     int B, cap;
+    unsigned long long* best;   // per-row greedy-choice key (nullable)
 };
 
 }  // namespace
@@ -88,6 +93,8 @@ struct psc_states {
 namespace {
 
 // ------------------------------------------------------------------ helpers
+__device__ int g_pipeline_timeouts;   // bounded in-kernel waits that gave up (a fault if ever non-zero)
+
 __device__ __forceinline__ void st_cs_v4(void* p, uint4 v) {
     asm volatile("st.global.cs.v4.b32 [%0], {%1, %2, %3, %4};" ::"l"(p), "r"(v.x), "r"(v.y), "r"(v.z),
                  "r"(v.w)
@@ -159,6 +166,7 @@ __global__ void k_state_init(DevStates S, int q0, const int32_t* rows, int n) {
     S.status[b] = ROW_OK;
     S.stack[(size_t)b * S.cap] = 0;
     S.mid[b] = 0;
+    if (S.best) S.best[b] = 0ull;
 }
 
 __global__ void k_classify(DevTables T, DevStates S, int B) {
@@ -166,7 +174,10 @@ __global__ void k_classify(DevTables T, DevStates S, int B) {
     int lane = threadIdx.x & 31;
     if (warp >= B) return;
     int mid = warp_classify(T, S, warp, lane);
-    if (lane == 0) S.mid[warp] = mid;
+    if (lane == 0) {
+        S.mid[warp] = mid;
+        if (S.best) S.best[warp] = 0ull;
+    }
 }
 
 // out[b][:] = masks[mid[b]][:]   (16-byte vector copies when W % 4 == 0)
@@ -400,10 +411,18 @@ __device__ int feed_class(const DevTables& T, uint16_t* st, int& depth, int cap,
 
 // Algorithm 2 steps 1-2 for one row per thread.
 __global__ void k_advance(DevTables T, DevStates S, const int32_t* tokens, int B, int use_mid,
-                          int32_t* status_out) {
+                          int32_t* status_out, int from_keys, int32_t* tokens_out) {
     int b = blockIdx.x * blockDim.x + threadIdx.x;
     if (b >= B) return;
-    int tok = tokens[b];
+    int tok;
+    if (from_keys) {   // the greedy choice of the fused masking pass
+        unsigned long long k = S.best[b];
+        S.best[b] = 0ull;
+        tok = k ? (int32_t)(~(uint32_t)(k & 0xFFFFFFFFu)) : -1;
+        tokens_out[b] = tok;
+    } else {
+        tok = tokens[b];
+    }
     int status = S.status[b];
     if (tok >= 0) {
         if (status == ROW_DONE) {
@@ -448,6 +467,647 @@ __global__ void k_advance(DevTables T, DevStates S, const int32_t* tokens, int B
         S.status[b] = status;
     }
     if (status_out) status_out[b] = status;
+}
+
+
+// ------------------------------------------------ fused masking + greedy choice
+// Orderable 32-bit key of a float (larger float -> larger key; -0 == +0).
+__device__ __forceinline__ uint32_t f32_order(uint32_t u) {
+    if ((u & 0x7FFFFFFFu) == 0) u = 0;
+    return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+
+// 64-bit greedy key: value order in the high word, then the lowest column wins.
+__device__ __forceinline__ unsigned long long make_key(uint32_t ordered, int col) {
+    return ((unsigned long long)ordered << 32) | (uint32_t)(~(uint32_t)col);
+}
+
+// Greedy state of one lane: the largest allowed value seen so far and the
+// lowest column holding it (col < 0: nothing yet).  NaN never becomes best.
+struct Best {
+    float val;
+    int col;
+};
+
+__device__ __forceinline__ void note_best(Best& best, float v, int col) {
+    if (best.col < 0 || v > best.val || (v == best.val && col < best.col)) {
+        best.val = v;
+        best.col = col;
+    }
+}
+
+__device__ __forceinline__ unsigned long long best_key_of(const Best& b) {
+    return b.col >= 0 ? make_key(f32_order(__float_as_uint(b.val)), b.col) : 0ull;
+}
+
+// Allowed-position masks of one 16-byte piece, indexed by its mask bits:
+// bf16 (8 bits -> 0xFFFF per allowed half of the 4 words), f32 (4 bits ->
+// 0xFFFFFFFF per allowed word).  Built in shared memory by every CTA.
+template <typename T>
+__device__ __forceinline__ void build_allow_lut(uint4* lut) {
+    constexpr int N = sizeof(T) == 2 ? 256 : 16;
+    for (int i = threadIdx.x; i < N; i += blockDim.x) {
+        uint32_t w[4];
+        for (int k = 0; k < 4; k++) {
+            if (sizeof(T) == 2)
+                w[k] = (((i >> (2 * k)) & 1) ? 0x0000FFFFu : 0u) | (((i >> (2 * k + 1)) & 1) ? 0xFFFF0000u : 0u);
+            else
+                w[k] = ((i >> k) & 1) ? 0xFFFFFFFFu : 0u;
+        }
+        lut[i] = make_uint4(w[0], w[1], w[2], w[3]);
+    }
+}
+
+__device__ __forceinline__ uint32_t sel_ninf(uint32_t w, uint32_t allow, uint32_t ninf) {
+    return (w & allow) | (ninf & ~allow);
+}
+
+__device__ __forceinline__ float bf16_at(uint32_t w, int half) {
+    return __uint_as_float(half ? (w & 0xFFFF0000u) : (w << 16));
+}
+
+// One 1024-column chunk of bf16: write -inf where masked (no read when the
+// whole 16-byte piece is masked), read the pieces that hold an allowed
+// position and fold their allowed values into the lane's best with packed
+// bf16x2 maxima; the column is searched only when the piece can win.
+__device__ __forceinline__ void apply_argmax_chunk_bf16(const uint16_t* src, uint16_t* row, int col0, uint32_t word, int lane,
+                                                        Best& best, const uint4* lut) {
+    const uint4 ninf = make_uint4(0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u);
+    uint32_t bits[4];
+    uint4 v[4];
+#pragma unroll
+    for (int k = 0; k < 4; k++) bits[k] = (__shfl_sync(FULL, word, k * 8 + (lane >> 2)) >> ((lane & 3) * 8)) & 0xFFu;
+#pragma unroll
+    for (int k = 0; k < 4; k++)   // issue every needed load before any store
+        if (bits[k]) v[k] = *reinterpret_cast<const uint4*>(src + (k * 32 + lane) * 8);
+#pragma unroll
+    for (int k = 0; k < 4; k++) {
+        uint16_t* p = row + col0 + (k * 32 + lane) * 8;
+        uint32_t bk = bits[k];
+        if (bk == 0) {
+            st_cs_v4(p, ninf);
+            continue;
+        }
+        uint4 am = lut[bk];
+        uint32_t x0 = sel_ninf(v[k].x, am.x, 0xFF80FF80u), x1 = sel_ninf(v[k].y, am.y, 0xFF80FF80u);
+        uint32_t x2 = sel_ninf(v[k].z, am.z, 0xFF80FF80u), x3 = sel_ninf(v[k].w, am.w, 0xFF80FF80u);
+        __nv_bfloat162 m = __hmax2(__hmax2(*reinterpret_cast<__nv_bfloat162*>(&x0), *reinterpret_cast<__nv_bfloat162*>(&x1)),
+                                   __hmax2(*reinterpret_cast<__nv_bfloat162*>(&x2), *reinterpret_cast<__nv_bfloat162*>(&x3)));
+        float mf = fmaxf(__low2float(m), __high2float(m));
+        if (best.col < 0 || mf >= best.val) {   // rare: this piece may hold the lane's best
+            uint32_t w[4] = {v[k].x, v[k].y, v[k].z, v[k].w};
+#pragma unroll
+            for (int e = 0; e < 8; e++) {
+                float f = bf16_at(w[e >> 1], e & 1);
+                if (((bk >> e) & 1) && f == mf) {
+                    note_best(best, f, col0 + (k * 32 + lane) * 8 + e);
+                    break;
+                }
+            }
+        }
+        if (bk != 0xFFu) *reinterpret_cast<uint4*>(p) = make_uint4(x0, x1, x2, x3);
+    }
+}
+
+// One 1024-column chunk of f32 (4 elements per 16-byte piece).
+__device__ __forceinline__ void apply_argmax_chunk_f32(const uint32_t* src, uint32_t* row, int col0, uint32_t word, int lane,
+                                                       Best& best, const uint4* lut) {
+    const uint4 ninf = make_uint4(0xFF800000u, 0xFF800000u, 0xFF800000u, 0xFF800000u);
+    uint32_t bits[8];
+    uint4 v[8];
+#pragma unroll
+    for (int k = 0; k < 8; k++) bits[k] = (__shfl_sync(FULL, word, k * 4 + (lane >> 3)) >> ((lane & 7) * 4)) & 0xFu;
+#pragma unroll
+    for (int k = 0; k < 8; k++)
+        if (bits[k]) v[k] = *reinterpret_cast<const uint4*>(src + (k * 32 + lane) * 4);
+#pragma unroll
+    for (int k = 0; k < 8; k++) {
+        uint32_t* p = row + col0 + (k * 32 + lane) * 4;
+        uint32_t bk = bits[k];
+        if (bk == 0) {
+            st_cs_v4(p, ninf);
+            continue;
+        }
+        uint4 am = lut[bk];
+        uint32_t x0 = sel_ninf(v[k].x, am.x, 0xFF800000u), x1 = sel_ninf(v[k].y, am.y, 0xFF800000u);
+        uint32_t x2 = sel_ninf(v[k].z, am.z, 0xFF800000u), x3 = sel_ninf(v[k].w, am.w, 0xFF800000u);
+        float mf = fmaxf(fmaxf(__uint_as_float(x0), __uint_as_float(x1)), fmaxf(__uint_as_float(x2), __uint_as_float(x3)));
+        if (best.col < 0 || mf >= best.val) {
+            uint32_t w[4] = {v[k].x, v[k].y, v[k].z, v[k].w};
+#pragma unroll
+            for (int e = 0; e < 4; e++) {
+                float f = __uint_as_float(w[e]);
+                if (((bk >> e) & 1) && f == mf) {
+                    note_best(best, f, col0 + (k * 32 + lane) * 4 + e);
+                    break;
+                }
+            }
+        }
+        if (bk != 0xFu) *reinterpret_cast<uint4*>(p) = make_uint4(x0, x1, x2, x3);
+    }
+}
+
+template <typename T>
+__device__ __forceinline__ void apply_argmax_chunk_scalar(T* row, int col0, int ncols, uint32_t word, int lane,
+                                                          Best& best) {
+    int c0 = 32 * lane;
+    for (int e = 0; e < 32; e++) {
+        if (c0 + e >= ncols) break;
+        int col = col0 + c0 + e;
+        if (!((word >> e) & 1)) {
+            row[col] = (T)NegInf<T>::one;
+        } else {
+            float f = sizeof(T) == 2 ? __uint_as_float((uint32_t)row[col] << 16) : __uint_as_float((uint32_t)row[col]);
+            if (!isnan(f)) note_best(best, f, col);
+        }
+    }
+}
+
+template <typename T>
+__device__ __forceinline__ void apply_argmax_any(T* row, int col0, int V, uint32_t word, int lane, int vec, Best& best,
+                                                 const uint4* lut) {
+    int ncols = V - col0;
+    if (vec && ncols >= 1024) {
+        if (sizeof(T) == 2)
+            apply_argmax_chunk_bf16(reinterpret_cast<uint16_t*>(row) + col0, reinterpret_cast<uint16_t*>(row), col0,
+                                    word, lane, best, lut);
+        else
+            apply_argmax_chunk_f32(reinterpret_cast<uint32_t*>(row) + col0, reinterpret_cast<uint32_t*>(row), col0,
+                                   word, lane, best, lut);
+    } else {
+        apply_argmax_chunk_scalar<T>(row, col0, ncols < 1024 ? ncols : 1024, word, lane, best);
+    }
+}
+
+// Fused masking + greedy choice.  Work item = (row, segment of seg_chunks
+// 1024-column chunks); the 8 warps of a CTA split a segment, reduce their keys
+// in shared memory, and one 64-bit atomic max per item merges the row's best.
+// WALK: the CTA classifies its rows itself (Algorithm 2 step 3): warp 0 walks
+// the classifier for the next item's row while the CTA streams the current
+// item, chunks being handed out through a shared counter so that warp 0 joins
+// once its walk is done; the segment-0 CTA of a row records the row's mask id.
+// Per-row keys must be zero on entry (state init, finalize and advance clear them).
+template <typename T, bool WALK>
+__global__ void __launch_bounds__(256, 4) k_apply_argmax(T* logits, int64_t stride, MaskSrc M, int B, int V, int vec,
+                                                         int seg_chunks, unsigned long long* __restrict__ best_key,
+                                                         DevTables D, DevStates S) {
+    __shared__ unsigned long long red[8];
+    __shared__ int s_mid[2];
+    __shared__ int s_ctr;
+    __shared__ uint4 s_lut[256];
+    int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    int cpr = (V + 1023) >> 10;
+    int nseg = (cpr + seg_chunks - 1) / seg_chunks;
+    long items = (long)B * nseg;
+    int cur = 0;
+    build_allow_lut<T>(s_lut);
+    __syncthreads();
+    if (WALK) {
+        if (warp == 0 && (long)blockIdx.x < items) {
+            int m = warp_classify(D, S, (int)(blockIdx.x / nseg), lane);
+            if (lane == 0) s_mid[0] = m;
+        }
+        if (threadIdx.x == 0) s_ctr = 0;
+        __syncthreads();
+    }
+    for (long it = blockIdx.x; it < items; it += gridDim.x) {
+        int b = (int)(it / nseg);
+        int sg = (int)(it - (long)b * nseg);
+        int c0 = sg * seg_chunks;
+        int c1 = min(c0 + seg_chunks, cpr);
+        const uint32_t* mrow;
+        if (WALK) {
+            int mid = s_mid[cur];
+            mrow = D.masks + (size_t)mid * D.Wp;
+            if (sg == 0 && threadIdx.x == 0) S.mid[b] = mid;
+        } else {
+            mrow = M.row(b);
+        }
+        T* row = logits + (size_t)b * stride;
+        Best best{0.f, -1};
+        if (WALK) {
+            long nx = it + gridDim.x;
+            if (warp == 0 && nx < items) {
+                int m = warp_classify(D, S, (int)(nx / nseg), lane);
+                if (lane == 0) s_mid[cur ^ 1] = m;
+            }
+            for (;;) {
+                int j = 0;
+                if (lane == 0) j = atomicAdd(&s_ctr, 1);
+                j = __shfl_sync(FULL, j, 0) + c0;
+                if (j >= c1) break;
+                int col0 = j << 10;
+                int wi = (col0 >> 5) + lane;
+                uint32_t word = wi < M.W ? __ldg(mrow + wi) : 0u;
+                if (M.copy_out && wi < M.W) M.copy_out[(size_t)b * M.W + wi] = word;
+                apply_argmax_any<T>(row, col0, V, word, lane, vec, best, s_lut);
+            }
+        } else {
+            for (int j = c0 + warp; j < c1; j += 8) {
+                int col0 = j << 10;
+                int wi = (col0 >> 5) + lane;
+                uint32_t word = wi < M.W ? __ldg(mrow + wi) : 0u;
+                if (M.copy_out && wi < M.W) M.copy_out[(size_t)b * M.W + wi] = word;
+                apply_argmax_any<T>(row, col0, V, word, lane, vec, best, s_lut);
+            }
+        }
+        unsigned long long key = best_key_of(best);
+#pragma unroll
+        for (int off = 16; off; off >>= 1) {
+            unsigned long long o = __shfl_xor_sync(FULL, key, off);
+            key = o > key ? o : key;
+        }
+        if (lane == 0) red[warp] = key;
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            unsigned long long k = red[0];
+            for (int w = 1; w < 8; w++) k = red[w] > k ? red[w] : k;
+            if (k) atomicMax(best_key + b, k);
+            if (WALK) s_ctr = 0;
+        }
+        cur ^= 1;
+        __syncthreads();
+    }
+}
+
+__global__ void k_finalize_tokens(unsigned long long* __restrict__ best_key, int B, int32_t* tokens) {
+    int b = blockIdx.x * blockDim.x + threadIdx.x;
+    if (b >= B) return;
+    unsigned long long k = best_key[b];
+    tokens[b] = k ? (int32_t)(~(uint32_t)(k & 0xFFFFFFFFu)) : -1;
+    best_key[b] = 0ull;
+}
+
+// ------------------------------------------- advance with staged tables
+// Same semantics as k_advance; the compact lexer/parser tables (int16
+// entries, byte classes for the lexer) are first copied to shared memory.
+// `top` mirrors st[depth - 1] in a register; only the state under a popped
+// handle is read back from the row's stack.
+__device__ int feed_class_smem(const uint8_t* sm, const DevTables& T, uint16_t* st, int& depth, int& top, int cap,
+                               int cls) {
+    const int16_t* resolve = reinterpret_cast<const int16_t*>(sm + T.o_resolve);
+    const int16_t* action = reinterpret_cast<const int16_t*>(sm + T.o_action);
+    const int16_t* go = reinterpret_cast<const int16_t*>(sm + T.o_go);
+    const uint8_t* rlen = sm + T.o_rlen;
+    const int16_t* rlhs = reinterpret_cast<const int16_t*>(sm + T.o_rlhs);
+    int t = resolve[cls * T.n_lr + top];
+    if (t < 0) return ROW_REJECTED;
+    for (int guard = 0; guard < 4 * cap + 64; guard++) {
+        int a = action[top * T.n_terms + t];
+        int kind = a & 3, val = (a >> 2) & 0x3FFF;
+        if (kind == psc::ACT_SHIFT) {
+            if (depth >= cap) return ROW_OVERFLOW;
+            st[depth++] = (uint16_t)val;
+            top = val;
+            return ROW_OK;
+        }
+        if (kind != psc::ACT_REDUCE) return ROW_REJECTED;
+        int k = rlen[val];
+        if (depth - k < 1) return ROW_REJECTED;
+        depth -= k;
+        int under = k ? st[depth - 1] : top;
+        int g = go[under * T.n_nts + rlhs[val]];
+        if (g < 0) return ROW_REJECTED;
+        if (depth >= cap) return ROW_OVERFLOW;
+        st[depth++] = (uint16_t)g;
+        top = g;
+    }
+    return ROW_LIMIT;
+}
+
+__device__ __forceinline__ uint32_t smem_addr(const void* p) {
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+// Bounded wait on phase 0 of an mbarrier; returns false if it did not complete.
+__device__ __forceinline__ bool mbar_wait0(uint32_t bar, int limit) {
+    for (int it = 0; it < limit; it++) {
+        uint32_t ok;
+        asm volatile(
+            "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], 0;\n selp.u32 %0, 1, 0, p;\n}"
+            : "=r"(ok)
+            : "r"(bar)
+            : "memory");
+        if (ok) return true;
+    }
+    return false;
+}
+
+__global__ void k_advance_smem(DevTables T, DevStates S, const int32_t* tokens, int B, int use_mid,
+                               int32_t* status_out, int from_keys, int32_t* tokens_out) {
+    extern __shared__ uint4 smem4[];
+    __shared__ __align__(8) uint64_t bar;
+    uint8_t* sm = reinterpret_cast<uint8_t*>(smem4);
+    // one TMA bulk copy stages the compact tables (16-byte aligned, multiple of 16 bytes)
+    uint32_t bar_a = smem_addr(&bar);
+    if (threadIdx.x == 0) {
+        asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(bar_a) : "memory");
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar_a), "r"(T.adv_bytes) : "memory");
+        asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+                     ::"r"(smem_addr(sm)), "l"(T.adv), "r"(T.adv_bytes), "r"(bar_a)
+                     : "memory");
+    }
+    __syncthreads();
+    bool staged = mbar_wait0(bar_a, 1 << 24);
+    int b = blockIdx.x * blockDim.x + threadIdx.x;
+    if (!staged) {
+        // the copy did not land: give the rows a LIMIT status, wait (bounded) for the copy, return
+        if (threadIdx.x == 0) atomicAdd(&g_pipeline_timeouts, 1);
+        if (b < B && S.status[b] == ROW_OK) S.status[b] = ROW_LIMIT;
+        if (b < B && from_keys) {
+            tokens_out[b] = -1;
+            S.best[b] = 0ull;
+        }
+        if (b < B && status_out) status_out[b] = S.status[b];
+        mbar_wait0(bar_a, 1 << 24);
+        return;
+    }
+    if (b >= B) return;
+    const uint8_t* bc = sm + T.o_bc;
+    const int16_t* trans = reinterpret_cast<const int16_t*>(sm + T.o_trans);
+    const int16_t* acc = reinterpret_cast<const int16_t*>(sm + T.o_accept);
+    const uint8_t* ign = sm + T.o_ign;
+    int tok;
+    if (from_keys) {   // the greedy choice of the fused masking pass
+        unsigned long long k = S.best[b];
+        S.best[b] = 0ull;
+        tok = k ? (int32_t)(~(uint32_t)(k & 0xFFFFFFFFu)) : -1;
+        tokens_out[b] = tok;
+    } else {
+        tok = tokens[b];
+    }
+    int status = S.status[b];
+    if (tok >= 0) {
+        if (status == ROW_DONE) {
+            status = tok == T.eos_id ? ROW_DONE : ROW_REJECTED;
+        } else if (status == ROW_OK) {
+            if (tok >= T.V) {
+                status = ROW_REJECTED;
+            } else {
+                int mid = use_mid ? S.mid[b] : thread_classify(T, S, b);
+                // the mask bit is loaded now and tested once the token is parsed: the row
+                // is only committed (q, depth) when the token was allowed
+                uint32_t mword = __ldg(T.masks + (size_t)mid * T.Wp + (tok >> 5));
+                if (tok == T.eos_id) {
+                    status = ((mword >> (tok & 31)) & 1) ? ROW_DONE : ROW_REJECTED;
+                } else {
+                    int q = S.q[b], depth = S.depth[b];
+                    uint16_t* st = S.stack + (size_t)b * S.cap;
+                    int top = st[depth - 1];
+                    int64_t lo = T.vocab_off[tok], hi = T.vocab_off[tok + 1];
+                    int len = (int)(hi - lo);
+                    // the token's bytes, fetched together (tokens up to 32 bytes)
+                    uint32_t tw[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+#pragma unroll
+                    for (int i = 0; i < 32; i++)
+                        if (i < len) tw[i >> 2] |= (uint32_t)T.vocab[lo + i] << (8 * (i & 3));
+                    for (int i = 0; i < len && status == ROW_OK; i++) {
+                        int byte = i < 32 ? (int)((tw[i >> 2] >> (8 * (i & 3))) & 0xFFu) : (int)T.vocab[lo + i];
+                        int c = bc[byte];
+                        int nx = trans[q * T.nbc + c];
+                        if (nx >= 0) {
+                            q = nx;
+                            continue;
+                        }
+                        int cls = q == T.q0 ? -1 : acc[q];
+                        if (cls < 0) {
+                            status = ROW_REJECTED;
+                            break;
+                        }
+                        if (!ign[cls]) status = feed_class_smem(sm, T, st, depth, top, S.cap, cls);
+                        q = trans[T.q0 * T.nbc + c];
+                        if (q < 0) status = ROW_REJECTED;
+                    }
+                    if (!((mword >> (tok & 31)) & 1)) status = ROW_REJECTED;
+                    if (status == ROW_OK) {
+                        S.q[b] = q;
+                        S.depth[b] = depth;
+                    }
+                }
+            }
+        }
+        S.status[b] = status;
+    }
+    if (status_out) status_out[b] = status;
+}
+
+// ------------------------------------------ TMA-pipelined decode masking pass
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+// Bounded wait for the phase with the given parity to complete (about a few
+// seconds at most; a pipeline wait that gives up is counted and the kernel ends).
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
+    for (int it = 0; it < (1 << 22); it++) {
+        uint32_t ok;
+        asm volatile(
+            "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
+            : "=r"(ok)
+            : "r"(bar), "r"(parity)
+            : "memory");
+        if (ok) return true;
+    }
+    return false;
+}
+// 1-D bulk copy global -> shared, completing on the mbarrier (16-byte aligned, size a multiple of 16).
+__device__ __forceinline__ void tma_load_1d(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+                 ::"r"(dst), "l"(src), "r"(bytes), "r"(bar)
+                 : "memory");
+}
+
+
+constexpr int TMA_SEG = 32;     // 1024-column chunks per work item
+constexpr int TMA_NCONS = 6;    // consumer warps (warp 0 produces, warp 1 classifies)
+
+// Ring stages: a multiple of the consumer count, so that stage s is always
+// consumed by warp 2 + s % TMA_NCONS and every waiter of a full barrier waits
+// for its rounds in order (a parity wait cannot tell round r from r + 2).
+template <typename T>
+struct TmaShape {
+    static constexpr int NS = sizeof(T) == 2 ? 18 : 6;
+    static constexpr int TILE = 1024 * (int)sizeof(T);   // one chunk
+    static constexpr int SMEM = NS * TILE + 2 * TMA_SEG * 32 * 4 + (2 * NS + 8) * 8;
+};
+
+// One decode masking pass (classification, mask, apply, greedy key) with the
+// logits streamed through shared memory by TMA bulk copies.  Work item = (row,
+// segment of TMA_SEG chunks).  Warp 0 (producer) copies the item's mask words
+// and every chunk that holds an allowed position into a ring of NS stages
+// (chunks with nothing allowed are not read); warp 1 walks the classifier for
+// the CTA's upcoming rows; warps 2-7 take the chunks round-robin, write -inf
+// where masked and fold allowed values into the row's greedy key.
+// Requires 16-byte aligned rows; rows' mask rows padded to whole chunks.
+template <typename T>
+__global__ void __launch_bounds__(256, 4) k_step_tma(T* logits, int64_t stride, int B, int V, uint32_t* copy_out,
+                                                     unsigned long long* __restrict__ best_key, DevTables D,
+                                                     DevStates S) {
+    constexpr int NS = TmaShape<T>::NS, TILE = TmaShape<T>::TILE;
+    static_assert(NS % TMA_NCONS == 0, "each ring stage must belong to one consumer warp");
+    extern __shared__ __align__(128) uint8_t smem[];
+    uint8_t* tiles = smem;
+    uint32_t* mbuf = reinterpret_cast<uint32_t*>(smem + NS * TILE);
+    uint64_t* bars = reinterpret_cast<uint64_t*>(mbuf + 2 * TMA_SEG * 32);
+    __shared__ int s_mid[2];
+    __shared__ uint4 s_lut[256];
+    int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    int cpr = (V + 1023) >> 10;
+    int nseg = (cpr + TMA_SEG - 1) / TMA_SEG;
+    build_allow_lut<T>(s_lut);
+    long items = (long)B * nseg;
+    const uint32_t full0 = smem_addr(bars), empty0 = full0 + 8 * NS, mfull0 = empty0 + 8 * NS;
+    const uint32_t mempty0 = mfull0 + 16, midf0 = mfull0 + 32, mide0 = mfull0 + 48;
+    if (threadIdx.x == 0) {
+        for (int k = 0; k < NS; k++) {
+            mbar_init(full0 + 8 * k, 1);
+            mbar_init(empty0 + 8 * k, 1);
+        }
+        for (int k = 0; k < 2; k++) {
+            mbar_init(mfull0 + 8 * k, 1);
+            mbar_init(mempty0 + 8 * k, TMA_NCONS);
+            mbar_init(midf0 + 8 * k, 1);
+            mbar_init(mide0 + 8 * k, 1);
+        }
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    }
+    __syncthreads();
+    bool failed = false;
+    if (warp == 0) {
+        // ---------------------------------------------------------- producer
+        long t = 0;
+        int i = 0;
+        int issued_mask = -1;
+        for (long it = blockIdx.x; it < items && !failed; it += gridDim.x, i++) {
+            int b = (int)(it / nseg), sg = (int)(it - (long)b * nseg);
+            int c0 = sg * TMA_SEG, nch = min(TMA_SEG, cpr - c0);
+            int slot = i & 1;
+            uint32_t ph = (i >> 1) & 1;
+            if (!__shfl_sync(FULL, (int)mbar_wait(midf0 + 8 * slot, ph), 0)) { failed = true; break; }
+            int mid = s_mid[slot];
+            __syncwarp();
+            if (lane == 0) {
+                mbar_arrive(mide0 + 8 * slot);
+                if (sg == 0) S.mid[b] = mid;
+            }
+            if (i >= 2 && !__shfl_sync(FULL, (int)mbar_wait(mempty0 + 8 * slot, ((i >> 1) - 1) & 1), 0)) {
+                failed = true;
+                break;
+            }
+            uint32_t* mb = mbuf + slot * TMA_SEG * 32;
+            if (lane == 0) {
+                mbar_arrive_tx(mfull0 + 8 * slot, nch * 128);
+                tma_load_1d(smem_addr(mb), D.masks + (size_t)mid * D.Wp + (size_t)c0 * 32, nch * 128, mfull0 + 8 * slot);
+            }
+            issued_mask = i;
+            if (!__shfl_sync(FULL, (int)mbar_wait(mfull0 + 8 * slot, ph), 0)) { failed = true; break; }
+            const T* row = logits + (size_t)b * stride;
+            for (int k = 0; k < nch; k++, t++) {
+                int j = c0 + k;
+                int stg = (int)(t % NS);
+                if (t >= NS && !__shfl_sync(FULL, (int)mbar_wait(empty0 + 8 * stg, (uint32_t)(((t / NS) - 1) & 1)), 0)) {
+                    failed = true;
+                    break;
+                }
+                bool any = __ballot_sync(FULL, mb[k * 32 + lane] != 0u) != 0u;
+                bool ragged = (j == cpr - 1) && (V & 1023);
+                if (lane == 0) {
+                    if (any && !ragged) {
+                        mbar_arrive_tx(full0 + 8 * stg, TILE);
+                        tma_load_1d(smem_addr(tiles + stg * TILE), row + (size_t)j * 1024, TILE, full0 + 8 * stg);
+                    } else {
+                        mbar_arrive(full0 + 8 * stg);
+                    }
+                }
+            }
+        }
+        if (failed && lane == 0) {
+            // let this CTA's copies in flight land before it exits (bounded)
+            for (long tt = t > NS ? t - NS : 0; tt < t; tt++) mbar_wait(full0 + 8 * (int)(tt % NS), (uint32_t)((tt / NS) & 1));
+            if (issued_mask >= 0) mbar_wait(mfull0 + 8 * (issued_mask & 1), (issued_mask >> 1) & 1);
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ walker
+        int i = 0;
+        for (long it = blockIdx.x; it < items; it += gridDim.x, i++) {
+            int slot = i & 1;
+            if (i >= 2 && !__shfl_sync(FULL, (int)mbar_wait(mide0 + 8 * slot, ((i >> 1) - 1) & 1), 0)) {
+                failed = true;
+                break;
+            }
+            int mid = warp_classify(D, S, (int)(it / nseg), lane);
+            if (lane == 0) {
+                s_mid[slot] = mid;
+                mbar_arrive(midf0 + 8 * slot);
+            }
+        }
+    } else {
+        // --------------------------------------------------------- consumers
+        int c = warp - 2;
+        long t = 0;
+        int i = 0;
+        for (long it = blockIdx.x; it < items && !failed; it += gridDim.x, i++) {
+            int b = (int)(it / nseg), sg = (int)(it - (long)b * nseg);
+            int c0 = sg * TMA_SEG, nch = min(TMA_SEG, cpr - c0);
+            int slot = i & 1;
+            if (!__shfl_sync(FULL, (int)mbar_wait(mfull0 + 8 * slot, (i >> 1) & 1), 0)) { failed = true; break; }
+            const uint32_t* mb = mbuf + slot * TMA_SEG * 32;
+            T* row = logits + (size_t)b * stride;
+            Best best{0.f, -1};
+            int k0 = (int)((c - (t % TMA_NCONS) + TMA_NCONS) % TMA_NCONS);
+            for (int k = k0; k < nch; k += TMA_NCONS) {
+                long tt = t + k;
+                int stg = (int)(tt % NS);
+                int j = c0 + k;
+                if (!__shfl_sync(FULL, (int)mbar_wait(full0 + 8 * stg, (uint32_t)((tt / NS) & 1)), 0)) {
+                    failed = true;
+                    break;
+                }
+                uint32_t w = mb[k * 32 + lane];
+                if (copy_out) {
+                    int wi = j * 32 + lane;
+                    if (wi < D.W) copy_out[(size_t)b * D.W + wi] = w;
+                }
+                int col0 = j << 10;
+                if ((j == cpr - 1) && (V & 1023)) {
+                    apply_argmax_chunk_scalar<T>(row, col0, V - col0, w, lane, best);
+                } else if (__ballot_sync(FULL, w != 0u) == 0u) {
+                    constexpr int PIECES = TILE / 16 / 32;
+                    uint4 ninf = make_uint4(NegInf<T>::pair, NegInf<T>::pair, NegInf<T>::pair, NegInf<T>::pair);
+#pragma unroll
+                    for (int q = 0; q < PIECES; q++)
+                        st_cs_v4(reinterpret_cast<uint8_t*>(row + col0) + (q * 32 + lane) * 16, ninf);
+                } else if (sizeof(T) == 2) {
+                    apply_argmax_chunk_bf16(reinterpret_cast<const uint16_t*>(tiles + stg * TILE),
+                                            reinterpret_cast<uint16_t*>(row), col0, w, lane, best, s_lut);
+                } else {
+                    apply_argmax_chunk_f32(reinterpret_cast<const uint32_t*>(tiles + stg * TILE),
+                                           reinterpret_cast<uint32_t*>(row), col0, w, lane, best, s_lut);
+                }
+                __syncwarp();
+                if (lane == 0) mbar_arrive(empty0 + 8 * stg);
+            }
+            t += nch;
+            unsigned long long key = best_key_of(best);
+#pragma unroll
+            for (int off = 16; off; off >>= 1) {
+                unsigned long long o = __shfl_xor_sync(FULL, key, off);
+                key = o > key ? o : key;
+            }
+            if (lane == 0) {
+                if (key) atomicMax(best_key + b, key);
+                mbar_arrive(mempty0 + 8 * slot);
+            }
+        }
+    }
+    if (failed && lane == 0) atomicAdd(&g_pipeline_timeouts, 1);
 }
 
 // ----------------------------------------------------------------- host glue
@@ -520,6 +1180,45 @@ psc_status launch_apply(void* logits, psc_dtype dtype, int64_t row_stride, const
     return launch_check("k_apply_rows");
 }
 
+// Masking + greedy choice with in-kernel classification; leaves each row's
+// key in st->d.best and its mask id in st->d.mid.
+psc_status launch_fused(const psc_handle* h, const psc_states* st, void* d_logits, psc_dtype dtype, int64_t row_stride,
+                        int V, uint32_t* d_bitmask_out, cudaStream_t cs) {
+    int B = st->d.B;
+    MaskSrc M{nullptr, h->d.masks, st->d.mid, h->d.W, h->d.Wp, d_bitmask_out};
+    size_t esz = dtype == PSC_BF16 ? 2 : 4;
+    int vec = aligned16(d_logits) && ((row_stride * (int64_t)esz) % 16 == 0);
+    int cpr = (V + 1023) / 1024;
+    int slots = sm_count(h->device) * 4;   // 4 resident CTAs of 256 threads per SM
+    long seg = ((long)cpr * B) / (2L * slots);
+    int seg_chunks = (int)std::max(1L, std::min(32L, seg));
+    long items = (long)B * ((cpr + seg_chunks - 1) / seg_chunks);
+    int grid = (int)std::max(1L, std::min<long>(items, slots));
+    psc_status s;
+    if (vec) {
+        // TMA pipeline: one item = (row, 32 chunks); 4 CTAs per SM
+        long titems = (long)B * ((cpr + TMA_SEG - 1) / TMA_SEG);
+        int tgrid = (int)std::max(1L, std::min<long>(titems, (long)sm_count(h->device) * 4));
+        if (dtype == PSC_BF16)
+            k_step_tma<uint16_t><<<tgrid, 256, TmaShape<uint16_t>::SMEM, cs>>>(
+                (uint16_t*)d_logits, row_stride, B, V, d_bitmask_out, st->d.best, h->d, st->d);
+        else
+            k_step_tma<uint32_t><<<tgrid, 256, TmaShape<uint32_t>::SMEM, cs>>>(
+                (uint32_t*)d_logits, row_stride, B, V, d_bitmask_out, st->d.best, h->d, st->d);
+        s = launch_check("k_step_tma");
+    } else {
+        if (dtype == PSC_BF16)
+            k_apply_argmax<uint16_t, true><<<grid, 256, 0, cs>>>((uint16_t*)d_logits, row_stride, M, B, V, vec,
+                                                                  seg_chunks, st->d.best, h->d, st->d);
+        else
+            k_apply_argmax<uint32_t, true><<<grid, 256, 0, cs>>>((uint32_t*)d_logits, row_stride, M, B, V, vec,
+                                                                  seg_chunks, st->d.best, h->d, st->d);
+        s = launch_check("k_apply_argmax");
+    }
+    if (s == PSC_OK) const_cast<psc_states*>(st)->mid_gen = st->gen;
+    return s;
+}
+
 // host-side parser step for psc_host_advance (same semantics as k_advance)
 int host_feed(const psc::Tables& T, uint16_t* st, int& depth, int cap, int cls) {
     int t = T.resolve[(size_t)cls * T.n_lr + st[depth - 1]];
@@ -542,6 +1241,74 @@ int host_feed(const psc::Tables& T, uint16_t* st, int& depth, int cap, int cls) 
         st[depth++] = (uint16_t)go;
     }
     return ROW_LIMIT;
+}
+
+}  // namespace
+
+namespace {
+// Compact int16 lexer/parser tables for k_advance_smem, or an empty blob when
+// the grammar is too large for shared memory (k_advance then reads global memory).
+std::vector<uint8_t> build_advance_blob(const psc::Tables& t, DevTables& d) {
+    std::vector<uint8_t> blob;
+    d.adv_bytes = 0;
+    int n_rules = (int)t.rule_len.size();
+    if (t.n_lr >= 8192 || n_rules >= 8192 || t.nq >= 32768 || t.n_terms >= 32768) return blob;
+    for (int L : t.rule_len)
+        if (L > 255) return blob;
+    // byte classes of the lexer DFA
+    std::vector<int> bc(256, -1);
+    int nbc = 0;
+    for (int b = 0; b < 256; b++) {
+        if (bc[b] >= 0) continue;
+        bc[b] = nbc;
+        for (int b2 = b + 1; b2 < 256; b2++) {
+            if (bc[b2] >= 0) continue;
+            bool same = true;
+            for (int q = 0; q < t.nq && same; q++) same = t.lex_trans[(size_t)q * 256 + b] == t.lex_trans[(size_t)q * 256 + b2];
+            if (same) bc[b2] = nbc;
+        }
+        nbc++;
+    }
+    size_t off = 0;
+    auto take = [&](size_t bytes) {
+        size_t o = off;
+        off = (off + bytes + 15) & ~(size_t)15;
+        return (int)o;
+    };
+    int ncls = t.n_classes;
+    d.o_bc = take(256);
+    d.o_trans = take((size_t)t.nq * nbc * 2);
+    d.o_accept = take((size_t)t.nq * 2);
+    d.o_ign = take((size_t)std::max(ncls, 1));
+    d.o_resolve = take((size_t)std::max(ncls, 1) * t.n_lr * 2);
+    d.o_action = take((size_t)t.n_lr * t.n_terms * 2);
+    d.o_go = take((size_t)t.n_lr * t.n_nts * 2);
+    d.o_rlen = take((size_t)n_rules);
+    d.o_rlhs = take((size_t)n_rules * 2);
+    if (off > 200 * 1024) return blob;
+    blob.assign(off, 0);
+    auto put16 = [&](int o, size_t i, int v) { reinterpret_cast<int16_t*>(blob.data() + o)[i] = (int16_t)v; };
+    for (int b = 0; b < 256; b++) blob[d.o_bc + b] = (uint8_t)bc[b];
+    for (int q = 0; q < t.nq; q++) {
+        for (int b = 0; b < 256; b++) put16(d.o_trans, (size_t)q * nbc + bc[b], t.lex_trans[(size_t)q * 256 + b]);
+        put16(d.o_accept, q, t.lex_accept[q]);
+    }
+    for (int c = 0; c < ncls; c++) {
+        blob[d.o_ign + c] = t.cls_ignored[c];
+        for (int s = 0; s < t.n_lr; s++) put16(d.o_resolve, (size_t)c * t.n_lr + s, t.resolve[(size_t)c * t.n_lr + s]);
+    }
+    for (size_t i = 0; i < t.action.size(); i++) {
+        int32_t a = t.action[i];
+        put16(d.o_action, i, ((psc::act_val(a) & 0x3FFF) << 2) | psc::act_kind(a));
+    }
+    for (size_t i = 0; i < t.go.size(); i++) put16(d.o_go, i, t.go[i]);
+    for (int r = 0; r < n_rules; r++) {
+        blob[d.o_rlen + r] = (uint8_t)t.rule_len[r];
+        put16(d.o_rlhs, r, t.rule_lhs[r]);
+    }
+    d.nbc = nbc;
+    d.adv_bytes = (int)off;
+    return blob;
 }
 
 }  // namespace
@@ -569,6 +1336,79 @@ psc_status noalloc_scratch(int device, int32_t** out) {
 }
 }  // namespace
 
+namespace {
+// Uploads a handle's host tables to the current device (psc_compile, psc_load).
+psc_status upload_tables(std::unique_ptr<psc_handle>& h, bool global_tables) {
+    const psc::Tables& t = h->t;
+    psc_status s = cuda_check(cudaGetDevice(&h->device), "cudaGetDevice");
+    if (s != PSC_OK) return s;
+    DevTables& d = h->d;
+    int Wp = (t.W + 31) & ~31;   // whole 1024-column chunks per row (16-byte and 128-byte aligned rows)
+    std::vector<uint32_t> masks((size_t)t.n_masks * Wp, 0);
+    for (int m = 0; m < t.n_masks; m++)
+        std::memcpy(masks.data() + (size_t)m * Wp, t.masks.data() + (size_t)m * t.W, sizeof(uint32_t) * t.W);
+    std::vector<int32_t> dfa = t.dfa;
+    if (dfa.empty()) dfa.push_back(0);
+    std::vector<int32_t> dfa_mask = t.dfa_mask;
+    if (dfa_mask.empty()) dfa_mask.push_back(0);
+    if ((s = upload(h.get(), t.lex_trans, &d.lex_trans)) || (s = upload(h.get(), t.lex_accept, &d.lex_accept)) ||
+        (s = upload(h.get(), t.cls_ignored, &d.cls_ignored)) || (s = upload(h.get(), t.action, &d.action)) ||
+        (s = upload(h.get(), t.go, &d.go)) || (s = upload(h.get(), t.rule_len, &d.rule_len)) ||
+        (s = upload(h.get(), t.rule_lhs, &d.rule_lhs)) || (s = upload(h.get(), t.resolve, &d.resolve)) ||
+        (s = upload(h.get(), dfa, &d.dfa)) || (s = upload(h.get(), t.dfa_start, &d.dfa_start)) ||
+        (s = upload(h.get(), dfa_mask, &d.dfa_mask)) || (s = upload(h.get(), masks, &d.masks)) ||
+        (s = upload(h.get(), t.vocab_bytes, &d.vocab, 16)) || (s = upload(h.get(), t.vocab_off, &d.vocab_off))) {
+        for (int i = 0; i < h->n_blocks; i++) cudaFree(h->blocks[i]);
+        return s;
+    }
+    std::vector<uint8_t> blob;
+    if (!global_tables) blob = build_advance_blob(t, d);
+    if (!blob.empty()) {
+        if ((s = upload(h.get(), blob, &d.adv)) != PSC_OK) {
+            for (int i = 0; i < h->n_blocks; i++) cudaFree(h->blocks[i]);
+            return s;
+        }
+        // the limit is per function and device, shared by every handle: raise it to the
+        // device's opt-in maximum instead of to this handle's size
+        int optin = 0;
+        cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, h->device);
+        cudaFuncAttributes fa{};
+        cudaFuncGetAttributes(&fa, k_advance_smem);
+        optin -= (int)fa.sharedSizeBytes;   // the limit covers dynamic memory only
+        if (optin < d.adv_bytes) {
+            d.adv_bytes = 0;   // cannot stage: fall back to global tables
+        } else if ((s = cuda_check(cudaFuncSetAttribute(k_advance_smem, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                        optin),
+                                   "cudaFuncSetAttribute(k_advance_smem)")) != PSC_OK) {
+            for (int i = 0; i < h->n_blocks; i++) cudaFree(h->blocks[i]);
+            return s;
+        }
+    }
+    // the TMA masking pass uses more than the default 48 KiB of shared memory
+    if ((s = cuda_check(cudaFuncSetAttribute(k_step_tma<uint16_t>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             TmaShape<uint16_t>::SMEM),
+                        "cudaFuncSetAttribute(k_step_tma)")) != PSC_OK ||
+        (s = cuda_check(cudaFuncSetAttribute(k_step_tma<uint32_t>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             TmaShape<uint32_t>::SMEM),
+                        "cudaFuncSetAttribute(k_step_tma)")) != PSC_OK) {
+        for (int i = 0; i < h->n_blocks; i++) cudaFree(h->blocks[i]);
+        return s;
+    }
+    d.q0 = t.q0;
+    d.nq = t.nq;
+    d.n_lr = t.n_lr;
+    d.n_terms = t.n_terms;
+    d.n_nts = t.n_nts;
+    d.end_term = t.end_term;
+    d.V = t.V;
+    d.W = t.W;
+    d.Wp = Wp;
+    d.eos_id = t.eos_id;
+    d.n_masks = t.n_masks;
+    return PSC_OK;
+}
+}  // namespace
+
 // ====================================================================== ABI
 extern "C" {
 
@@ -585,12 +1425,13 @@ psc_status psc_compile(const char* grammar, size_t grammar_len, const uint8_t* v
     for (int v = 0; v < V; v++)
         if (vocab_offsets[v + 1] < vocab_offsets[v]) return fail_with(PSC_ERR_ARG, "psc_compile: offsets decrease");
     psc::Options o;
-    bool host_only = false;
+    bool host_only = false, global_tables = false;
     if (opts) {
         if (opts->max_states > 0) o.max_states = opts->max_states;
         if (opts->max_mask_bytes > 0) o.max_mask_bytes = opts->max_mask_bytes;
         o.threads = opts->threads;
         host_only = opts->host_only != 0;
+        global_tables = opts->global_tables != 0;
     }
     std::unique_ptr<psc_handle> h(new (std::nothrow) psc_handle());
     if (!h) return fail_with(PSC_ERR_OOM, "psc_compile: out of host memory");
@@ -603,39 +1444,8 @@ psc_status psc_compile(const char* grammar, size_t grammar_len, const uint8_t* v
     }
     h->host_only = host_only;
     if (!host_only) {
-        const psc::Tables& t = h->t;
-        psc_status s = cuda_check(cudaGetDevice(&h->device), "cudaGetDevice");
+        psc_status s = upload_tables(h, global_tables);
         if (s != PSC_OK) return s;
-        DevTables& d = h->d;
-        int Wp = (t.W + 3) & ~3;
-        std::vector<uint32_t> masks((size_t)t.n_masks * Wp, 0);
-        for (int m = 0; m < t.n_masks; m++)
-            std::memcpy(masks.data() + (size_t)m * Wp, t.masks.data() + (size_t)m * t.W, sizeof(uint32_t) * t.W);
-        std::vector<int32_t> dfa = t.dfa;
-        if (dfa.empty()) dfa.push_back(0);
-        std::vector<int32_t> dfa_mask = t.dfa_mask;
-        if (dfa_mask.empty()) dfa_mask.push_back(0);
-        if ((s = upload(h.get(), t.lex_trans, &d.lex_trans)) || (s = upload(h.get(), t.lex_accept, &d.lex_accept)) ||
-            (s = upload(h.get(), t.cls_ignored, &d.cls_ignored)) || (s = upload(h.get(), t.action, &d.action)) ||
-            (s = upload(h.get(), t.go, &d.go)) || (s = upload(h.get(), t.rule_len, &d.rule_len)) ||
-            (s = upload(h.get(), t.rule_lhs, &d.rule_lhs)) || (s = upload(h.get(), t.resolve, &d.resolve)) ||
-            (s = upload(h.get(), dfa, &d.dfa)) || (s = upload(h.get(), t.dfa_start, &d.dfa_start)) ||
-            (s = upload(h.get(), dfa_mask, &d.dfa_mask)) || (s = upload(h.get(), masks, &d.masks)) ||
-            (s = upload(h.get(), t.vocab_bytes, &d.vocab, 16)) || (s = upload(h.get(), t.vocab_off, &d.vocab_off))) {
-            for (int i = 0; i < h->n_blocks; i++) cudaFree(h->blocks[i]);
-            return s;
-        }
-        d.q0 = t.q0;
-        d.nq = t.nq;
-        d.n_lr = t.n_lr;
-        d.n_terms = t.n_terms;
-        d.n_nts = t.n_nts;
-        d.end_term = t.end_term;
-        d.V = t.V;
-        d.W = t.W;
-        d.Wp = Wp;
-        d.eos_id = t.eos_id;
-        d.n_masks = t.n_masks;
     }
     *out = h.release();
     return PSC_OK;
@@ -659,9 +1469,15 @@ psc_status psc_info(const psc_handle* h, psc_info_t* out) {
     out->n_masks = t.n_masks;
     out->eos_id = t.eos_id;
     out->classifier_bytes = (int64_t)(t.dfa.size() + t.dfa_start.size() + t.dfa_mask.size()) * 4;
-    out->mask_bytes = (int64_t)t.n_masks * ((t.W + 3) & ~3) * 4;
+    out->mask_bytes = (int64_t)t.n_masks * ((t.W + 31) & ~31) * 4;
     out->states_built = t.n_dfa_states_built;
     out->compile_seconds = t.seconds_total;
+    out->advance_table_bytes = h->host_only ? 0 : h->d.adv_bytes;
+    out->device_timeouts = 0;
+    if (!h->host_only) {
+        int v = 0;
+        if (cudaMemcpyFromSymbol(&v, g_pipeline_timeouts, sizeof(int)) == cudaSuccess) out->device_timeouts = v;
+    }
     return PSC_OK;
 }
 
@@ -678,10 +1494,10 @@ psc_status psc_state_init(const psc_handle* h, int32_t B, int32_t cap, void* str
     DevStates& d = st->d;
     d.B = B;
     d.cap = cap;
-    void* p[5] = {};
-    size_t sz[5] = {sizeof(int32_t) * B, sizeof(int32_t) * B, sizeof(int32_t) * B, sizeof(uint16_t) * (size_t)B * cap,
-                    sizeof(int32_t) * B};
-    for (int i = 0; i < 5; i++) {
+    void* p[6] = {};
+    size_t sz[6] = {sizeof(int32_t) * B, sizeof(int32_t) * B, sizeof(int32_t) * B, sizeof(uint16_t) * (size_t)B * cap,
+                    sizeof(int32_t) * B, sizeof(unsigned long long) * B};
+    for (int i = 0; i < 6; i++) {
         s = cuda_check(cudaMalloc(&p[i], sz[i]), "cudaMalloc(states)");
         if (s != PSC_OK) {
             for (int j = 0; j < i; j++) cudaFree(p[j]);
@@ -693,11 +1509,12 @@ psc_status psc_state_init(const psc_handle* h, int32_t B, int32_t cap, void* str
     d.status = (int32_t*)p[2];
     d.stack = (uint16_t*)p[3];
     d.mid = (int32_t*)p[4];
+    d.best = (unsigned long long*)p[5];
     cudaStream_t cs = (cudaStream_t)stream;
     k_state_init<<<(B + 255) / 256, 256, 0, cs>>>(d, h->d.q0, nullptr, B);
     s = launch_check("k_state_init");
     if (s != PSC_OK) {
-        for (int j = 0; j < 5; j++) cudaFree(p[j]);
+        for (int j = 0; j < 6; j++) cudaFree(p[j]);
         return s;
     }
     *out = st.release();
@@ -721,6 +1538,7 @@ void psc_state_destroy(psc_states* st) {
     cudaFree(st->d.status);
     cudaFree(st->d.stack);
     cudaFree(st->d.mid);
+    cudaFree(st->d.best);
     delete st;
 }
 
@@ -730,7 +1548,12 @@ psc_status psc_advance(const psc_handle* h, psc_states* st, const int32_t* d_tok
     if (s != PSC_OK) return s;
     if (!st || st->h != h || B != st->d.B || !d_tokens) return fail_with(PSC_ERR_ARG, "psc_advance: bad arguments");
     int use_mid = st->mid_gen == st->gen ? 1 : 0;
-    k_advance<<<(B + 127) / 128, 128, 0, (cudaStream_t)stream>>>(h->d, st->d, d_tokens, B, use_mid, d_row_status);
+    if (h->d.adv_bytes > 0)
+        k_advance_smem<<<(B + 63) / 64, 64, h->d.adv_bytes, (cudaStream_t)stream>>>(h->d, st->d, d_tokens, B,
+                                                                                  use_mid, d_row_status, 0, nullptr);
+    else
+        k_advance<<<(B + 127) / 128, 128, 0, (cudaStream_t)stream>>>(h->d, st->d, d_tokens, B, use_mid, d_row_status,
+                                                                      0, nullptr);
     st->gen++;
     return launch_check("k_advance");
 }
@@ -791,6 +1614,39 @@ psc_status psc_argmax_masked(const psc_handle* h, const psc_states* st, int32_t 
         k_argmax_masked<uint32_t><<<B, 256, 0, cs>>>((const uint32_t*)d_logits, row_stride, h->d, st->d.mid, B, V, vec,
                                                      d_tokens);
     return launch_check("k_argmax_masked");
+}
+
+psc_status psc_fill_apply_argmax(const psc_handle* h, const psc_states* st, int32_t B, void* d_logits,
+                                 psc_dtype dtype, int64_t row_stride, int32_t V, uint32_t* d_bitmask_out,
+                                 int32_t* d_tokens, void* stream) {
+    psc_status s = check_device(h, "psc_fill_apply_argmax");
+    if (s != PSC_OK) return s;
+    if (!st || st->h != h || B != st->d.B || !d_logits || !d_tokens || V != h->d.V || row_stride < V ||
+        (dtype != PSC_F32 && dtype != PSC_BF16))
+        return fail_with(PSC_ERR_ARG, "psc_fill_apply_argmax: bad arguments");
+    cudaStream_t cs = (cudaStream_t)stream;
+    if ((s = launch_fused(h, st, d_logits, dtype, row_stride, V, d_bitmask_out, cs)) != PSC_OK) return s;
+    k_finalize_tokens<<<(B + 255) / 256, 256, 0, cs>>>(st->d.best, B, d_tokens);
+    return launch_check("k_finalize_tokens");
+}
+
+psc_status psc_decode_step(const psc_handle* h, psc_states* st, int32_t B, void* d_logits, psc_dtype dtype,
+                           int64_t row_stride, int32_t V, uint32_t* d_bitmask_out, int32_t* d_tokens,
+                           int32_t* d_row_status, void* stream) {
+    psc_status s = check_device(h, "psc_decode_step");
+    if (s != PSC_OK) return s;
+    if (!st || st->h != h || B != st->d.B || !d_logits || !d_tokens || V != h->d.V || row_stride < V ||
+        (dtype != PSC_F32 && dtype != PSC_BF16))
+        return fail_with(PSC_ERR_ARG, "psc_decode_step: bad arguments");
+    cudaStream_t cs = (cudaStream_t)stream;
+    if ((s = launch_fused(h, st, d_logits, dtype, row_stride, V, d_bitmask_out, cs)) != PSC_OK) return s;
+    if (h->d.adv_bytes > 0)
+        k_advance_smem<<<(B + 63) / 64, 64, h->d.adv_bytes, cs>>>(h->d, st->d, nullptr, B, 1, d_row_status, 1,
+                                                                   d_tokens);
+    else
+        k_advance<<<(B + 127) / 128, 128, 0, cs>>>(h->d, st->d, nullptr, B, 1, d_row_status, 1, d_tokens);
+    st->gen++;
+    return launch_check("k_advance");
 }
 
 psc_status psc_states_download(const psc_states* st, int32_t* h_q, int32_t* h_depth, uint16_t* h_stack,
@@ -900,6 +1756,39 @@ psc_status psc_fill_apply_noalloc(const psc_handle* h, const int32_t* d_q, const
     if ((s = launch_check("k_classify")) != PSC_OK) return s;
     MaskSrc M{nullptr, h->d.masks, mid, h->d.W, h->d.Wp, d_bitmask_out};
     return launch_apply(d_logits, dtype, row_stride, M, B, V, cs, h->device);
+}
+
+psc_status psc_save(const psc_handle* h, const char* path) {
+    if (!h || !path) return fail_with(PSC_ERR_ARG, "psc_save: NULL argument");
+    try {
+        psc::save_tables(h->t, path);
+    } catch (const psc::Error& e) {
+        return fail_with((psc_status)e.code, e.what());
+    } catch (const std::bad_alloc&) {
+        return fail_with(PSC_ERR_OOM, "psc_save: out of host memory");
+    }
+    return PSC_OK;
+}
+
+psc_status psc_load(const char* path, const psc_options* opts, psc_handle** out) {
+    if (!out || !path) return fail_with(PSC_ERR_ARG, "psc_load: NULL argument");
+    *out = nullptr;
+    std::unique_ptr<psc_handle> h(new (std::nothrow) psc_handle());
+    if (!h) return fail_with(PSC_ERR_OOM, "psc_load: out of host memory");
+    try {
+        h->t = psc::load_tables(path);
+    } catch (const psc::Error& e) {
+        return fail_with((psc_status)e.code, e.what());
+    } catch (const std::bad_alloc&) {
+        return fail_with(PSC_ERR_OOM, "psc_load: out of host memory");
+    }
+    h->host_only = opts && opts->host_only;
+    if (!h->host_only) {
+        psc_status s = upload_tables(h, opts && opts->global_tables);
+        if (s != PSC_OK) return s;
+    }
+    *out = h.release();
+    return PSC_OK;
 }
 
 }  // extern "C"

@@ -120,6 +120,10 @@ struct Tables {
 Tables compile_tables(const std::string& grammar, const uint8_t* vocab_bytes, const int64_t* offsets,
                       int V, int eos_id, const Options& opt);
 
+// binary persistence of the flat tables (throws Error(ST_ERR_IO) on failure)
+void save_tables(const Tables& t, const std::string& path);
+Tables load_tables(const std::string& path);
+
 // host-side walk of the flattened classifier (inspection / tests): mask id of (q, stack)
 int classify_host(const Tables& t, int q, const uint16_t* stack, int depth, int status);
 

@@ -25,7 +25,8 @@ STATUS_NAMES = {0: "PSC_OK", 1: "PSC_ERR_ARG", 2: "PSC_ERR_GRAMMAR", 3: "PSC_ERR
 EXPORTED = ["psc_compile", "psc_destroy", "psc_last_error", "psc_info", "psc_state_init", "psc_state_reset",
             "psc_state_destroy", "psc_advance", "psc_fill_mask", "psc_apply_mask", "psc_fill_apply",
             "psc_argmax_masked", "psc_states_download", "psc_host_classify", "psc_host_mask_row",
-            "psc_host_advance", "psc_fill_apply_noalloc"]
+            "psc_host_advance", "psc_fill_apply_noalloc", "psc_fill_apply_argmax", "psc_save", "psc_load",
+            "psc_decode_step"]
 NOALLOC_MAX_ROWS = 16384
 
 
@@ -37,7 +38,8 @@ class PscError(RuntimeError):
 
 class Options(ctypes.Structure):
     _fields_ = [("max_states", ctypes.c_int64), ("max_mask_bytes", ctypes.c_int64),
-                ("threads", ctypes.c_int32), ("host_only", ctypes.c_int32)]
+                ("threads", ctypes.c_int32), ("host_only", ctypes.c_int32),
+                ("global_tables", ctypes.c_int32)]
 
 
 class InfoT(ctypes.Structure):
@@ -45,7 +47,8 @@ class InfoT(ctypes.Structure):
                 ("n_parser_states", ctypes.c_int32), ("n_terminals", ctypes.c_int32),
                 ("n_classifier_states", ctypes.c_int32), ("n_masks", ctypes.c_int32), ("eos_id", ctypes.c_int32),
                 ("classifier_bytes", ctypes.c_int64), ("mask_bytes", ctypes.c_int64),
-                ("states_built", ctypes.c_int64), ("compile_seconds", ctypes.c_double)]
+                ("states_built", ctypes.c_int64), ("compile_seconds", ctypes.c_double),
+                ("advance_table_bytes", ctypes.c_int64), ("device_timeouts", ctypes.c_int64)]
 
 
 _lib = None
@@ -78,6 +81,10 @@ def load(path: str = LIB_PATH):
         "psc_host_mask_row": (i32, [vp, i32, vp]),
         "psc_host_advance": (i32, [vp, vp, vp, vp, i32, vp, i32]),
         "psc_fill_apply_noalloc": (i32, [vp, vp, vp, vp, vp, i32, i32, vp, i32, i64, i32, vp, vp]),
+        "psc_fill_apply_argmax": (i32, [vp, vp, i32, vp, i32, i64, i32, vp, vp, vp]),
+        "psc_save": (i32, [vp, ctypes.c_char_p]),
+        "psc_decode_step": (i32, [vp, vp, i32, vp, i32, i64, i32, vp, vp, vp, vp]),
+        "psc_load": (i32, [ctypes.c_char_p, vp, vp]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -140,6 +147,8 @@ class Info:
     mask_bytes: int
     states_built: int
     compile_seconds: float
+    advance_table_bytes: int
+    device_timeouts: int
 
 
 class Handle:
@@ -202,7 +211,8 @@ class States:
 
 # ------------------------------------------------------------------- the ABI
 def psc_compile(grammar: str, vocab: list[bytes] | tuple, eos_id: int, host_only: bool = False,
-                threads: int = 0, max_states: int = 0, max_mask_bytes: int = 0) -> Handle:
+                threads: int = 0, max_states: int = 0, max_mask_bytes: int = 0,
+                global_tables: bool = False) -> Handle:
     """vocab: list of token byte strings, or (blob uint8 array, offsets int64[V+1])."""
     if isinstance(vocab, tuple):
         blob, offs = vocab
@@ -215,12 +225,26 @@ def psc_compile(grammar: str, vocab: list[bytes] | tuple, eos_id: int, host_only
     if blob.size == 0:
         blob = np.zeros(1, dtype=np.uint8)
     V = len(offs) - 1
-    opts = Options(max_states, max_mask_bytes, threads, 1 if host_only else 0)
+    opts = Options(max_states, max_mask_bytes, threads, 1 if host_only else 0, 1 if global_tables else 0)
     g = grammar.encode("utf-8")
     out = ctypes.c_void_p()
     _check(load().psc_compile(g, len(g), blob.ctypes.data, offs.ctypes.data, V, eos_id, ctypes.byref(opts),
                               ctypes.byref(out)))
     return Handle(out.value, V)
+
+
+def psc_save(h: Handle, path: str):
+    _check(load().psc_save(h.ptr, os.fsencode(path)))
+
+
+def psc_load(path: str, host_only: bool = False, global_tables: bool = False) -> Handle:
+    opts = Options(0, 0, 0, 1 if host_only else 0, 1 if global_tables else 0)
+    out = ctypes.c_void_p()
+    _check(load().psc_load(os.fsencode(path), ctypes.byref(opts), ctypes.byref(out)))
+    h = Handle(out.value, 0)
+    h.V = h.info().V
+    h.W = (h.V + 31) // 32
+    return h
 
 
 def psc_state_init(h: Handle, B: int, cap: int = 256, stream=None) -> States:
@@ -278,6 +302,33 @@ def psc_argmax_masked(h: Handle, st: States, logits, tokens, stream=None):
     _check(load().psc_argmax_masked(h.ptr, st.ptr, st.B, _ptr(logits, None, "logits"), _dtype_code(logits),
                                     _row_stride(logits), h.V, _ptr(tokens, torch.int32, "tokens"),
                                     _stream(stream)))
+
+
+def psc_fill_apply_argmax(h: Handle, st: States, logits, tokens, bitmask_out=None, stream=None):
+    import torch
+    if logits.shape[0] != st.B or logits.shape[1] < h.V:
+        raise ValueError("logits must be [B, >=V]")
+    if tokens.numel() != st.B:
+        raise ValueError("tokens must hold B int32 values")
+    if bitmask_out is not None and (bitmask_out.shape != (st.B, h.W) or not bitmask_out.is_contiguous()):
+        raise ValueError("bitmask_out must be a contiguous [B, W] tensor")
+    _check(load().psc_fill_apply_argmax(h.ptr, st.ptr, st.B, _ptr(logits, None, "logits"), _dtype_code(logits),
+                                        _row_stride(logits), h.V, _ptr(bitmask_out, torch.int32, "bitmask_out"),
+                                        _ptr(tokens, torch.int32, "tokens"), _stream(stream)))
+
+
+def psc_decode_step(h: Handle, st: States, logits, tokens, bitmask_out=None, row_status=None, stream=None):
+    import torch
+    if logits.shape[0] != st.B or logits.shape[1] < h.V:
+        raise ValueError("logits must be [B, >=V]")
+    if tokens.numel() != st.B:
+        raise ValueError("tokens must hold B int32 values")
+    if bitmask_out is not None and (bitmask_out.shape != (st.B, h.W) or not bitmask_out.is_contiguous()):
+        raise ValueError("bitmask_out must be a contiguous [B, W] tensor")
+    _check(load().psc_decode_step(h.ptr, st.ptr, st.B, _ptr(logits, None, "logits"), _dtype_code(logits),
+                                  _row_stride(logits), h.V, _ptr(bitmask_out, torch.int32, "bitmask_out"),
+                                  _ptr(tokens, torch.int32, "tokens"), _ptr(row_status, torch.int32, "row_status"),
+                                  _stream(stream)))
 
 
 def psc_states_download(st: States, stream=None) -> dict:

@@ -35,10 +35,10 @@ class Case:
     """A workload compiled on the device, with device states and oracle configs
     advanced over the same prefix tokens."""
 
-    def __init__(self, psc, cfg_id, cap=256):
+    def __init__(self, psc, cfg_id, cap=256, global_tables=False):
         self.w = configs.load(cfg_id)
         w = self.w
-        self.h = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id)
+        self.h = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id, global_tables=global_tables)
         self.st = psc.psc_state_init(self.h, w.B, cap)
         tm = torch.from_numpy(w.token_matrix()).cuda()
         for j in range(tm.shape[1]):
@@ -149,6 +149,64 @@ def test_argmax_masked(psc, cfg_id):
         assert int(tok[b]) == want, b
 
 
+def cpu_greedy(logits_cpu, allowed):
+    """Lowest index of the largest allowed logit (NaN never wins), -1 if none."""
+    lf = logits_cpu.float().numpy()
+    out = np.full(lf.shape[0], -1, dtype=np.int64)
+    for b in range(lf.shape[0]):
+        idx = np.nonzero(allowed[b] & ~np.isnan(lf[b]))[0]
+        if len(idx):
+            out[b] = idx[np.argmax(lf[b, idx])]
+    return out
+
+
+@pytest.mark.parametrize("cfg_id", [1, 2, 3])
+def test_fused_apply_argmax_bit_exact(psc, cfg_id):
+    c = case(psc, cfg_id)
+    ref_mask = c.o.masks(c.ocs, c.voc, threads=THREADS)
+    allowed = bits_of(ref_mask, c.w.V)
+    logits = c.w.logits(7)
+    x = logits.cuda()
+    bm = torch.zeros(c.w.B, c.h.W, dtype=torch.int32, device="cuda")
+    tok = torch.empty(c.w.B, dtype=torch.int32, device="cuda")
+    psc.psc_fill_apply_argmax(c.h, c.st, x, tok, bm)
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(raw_bits(x), reference_masked(logits, allowed))
+    np.testing.assert_array_equal(bm.cpu().numpy().view(np.uint32), ref_mask)
+    np.testing.assert_array_equal(tok.cpu().numpy(), cpu_greedy(logits, allowed))
+
+
+def test_fused_argmax_ties_nan_and_empty_rows(psc):
+    """Ties go to the lowest index (+0 and -0 tie), NaN never wins, a row whose
+    allowed logits are all NaN gets -1; vector (f32, bf16) and element paths."""
+    g = grammars.json_grammar().text()
+    singles = [bytes([b]) for b in range(0x20, 0x7F)]
+    toks = singles + [a + b for a in singles[:40] for b in singles[:40]][:2000] + [b"true", b"false", b""]
+    V = len(toks)
+    h = psc.psc_compile(g, toks, V - 1)
+    st = psc.psc_state_init(h, 3, 32)
+    psc.psc_advance(h, st, torch.tensor([toks.index(b"["), -1, toks.index(b"{")], dtype=torch.int32,
+                                        device="cuda"))
+    bm = torch.empty(3, h.W, dtype=torch.int32, device="cuda")
+    psc.psc_fill_mask(h, st, bm)
+    allowed = bits_of(bm.cpu().numpy().view(np.uint32), V)
+    for dt in (torch.float32, torch.bfloat16):
+        for stride in (2048 + 16, V + 1):
+            x = torch.zeros(3, stride, dtype=torch.float32)
+            for b in range(3):
+                idx = np.nonzero(allowed[b])[0]
+                x[b, idx[0]] = float("nan")                     # the lowest allowed is NaN
+                x[b, idx[1::2]] = -0.0                           # the rest tie at zero
+            x[2, np.nonzero(allowed[2])[0]] = float("nan")       # row 2: nothing but NaN
+            xd = x.to(dt).cuda()
+            tok = torch.empty(3, dtype=torch.int32, device="cuda")
+            psc.psc_fill_apply_argmax(h, st, xd, tok)
+            t = tok.cpu().numpy()
+            assert t[0] == np.nonzero(allowed[0])[0][1], (dt, stride)
+            assert t[1] == np.nonzero(allowed[1])[0][1], (dt, stride)
+            assert t[2] == -1, (dt, stride)
+
+
 # ------------------------------------------------------ large configs, sampled
 @pytest.mark.parametrize("cfg_id", [4, 5])
 def test_large_config_fused_sampled(psc, cfg_id):
@@ -174,30 +232,62 @@ def test_large_config_fused_sampled(psc, cfg_id):
     got = raw_bits(x)
     want = reference_masked(logits[rows], dev_bits[rows])
     np.testing.assert_array_equal(got[rows], want)
+    # fused masking + greedy choice on fresh logits: same masks, choices = CPU greedy
+    logits2 = c.w.logits(3)
+    x2 = logits2.cuda()
+    tok = torch.empty(B, dtype=torch.int32, device="cuda")
+    bm2 = torch.zeros_like(bm)
+    psc.psc_fill_apply_argmax(c.h, c.st, x2, tok, bm2)
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(bm2.cpu().numpy().view(np.uint32), dev_mask)
+    np.testing.assert_array_equal(tok.cpu().numpy(), cpu_greedy(logits2, dev_bits))
+    np.testing.assert_array_equal(raw_bits(x2)[rows], reference_masked(logits2[rows], dev_bits[rows]))
 
 
 # ------------------------------------------------------------- decode loop
-@pytest.mark.parametrize("cfg_id,steps", [(2, 6), (5, 4)])
-def test_decode_loop_advance(psc, cfg_id, steps):
+@pytest.mark.parametrize("cfg_id,steps,mode", [(2, 6, "separate"), (3, 3, "fused"), (5, 4, "step")])
+def test_decode_loop_advance(psc, cfg_id, steps, mode):
+    _decode_loop(psc, case(psc, cfg_id), steps, mode)
+
+
+@pytest.mark.parametrize("global_tables", [False, True])
+def test_decode_loop_table_paths(psc, global_tables):
+    """The advance kernel with its tables staged in shared memory and read from
+    global memory give the same states (JSON, whole decode steps)."""
+    c = Case(psc, 2, global_tables=global_tables)
+    assert (c.h.info().advance_table_bytes > 0) == (not global_tables)
+    _decode_loop(psc, c, 5, "step")
+
+
+def _decode_loop(psc, c, steps, mode):
     """fill_apply -> argmax -> advance for several steps; after every step the
     device masks equal the oracle's after advancing it by the same tokens
     (runs after the other tests of the same workload: it advances its states)."""
-    c = case(psc, cfg_id)
     B, V = c.w.B, c.w.V
-    rng = np.random.default_rng(10 + cfg_id)
+    rng = np.random.default_rng(10 + B)
     rows = list(range(B)) if B <= 64 else sorted(rng.choice(B, size=16, replace=False).tolist())
     tok = torch.empty(B, dtype=torch.int32, device="cuda")
     stat = torch.empty(B, dtype=torch.int32, device="cuda")
     for step in range(steps):
-        x = c.w.logits(step + 1).cuda()
+        logits = c.w.logits(step + 1)
+        x = logits.cuda()
         bm = torch.zeros(B, c.h.W, dtype=torch.int32, device="cuda")
-        psc.psc_fill_apply(c.h, c.st, x, bm)
-        psc.psc_argmax_masked(c.h, c.st, x, tok)
+        if mode == "step":
+            psc.psc_decode_step(c.h, c.st, x, tok, bm, stat)
+        elif mode == "fused":
+            psc.psc_fill_apply_argmax(c.h, c.st, x, tok, bm)
+        else:
+            psc.psc_fill_apply(c.h, c.st, x, bm)
+            psc.psc_argmax_masked(c.h, c.st, x, tok)
         torch.cuda.synchronize()
         dev_mask = bm.cpu().numpy().view(np.uint32)
         ref = c.o.masks([c.ocs[r] for r in rows], c.voc, threads=THREADS)
         np.testing.assert_array_equal(dev_mask[rows], ref)
-        psc.psc_advance(c.h, c.st, tok, stat)
+        allowed = bits_of(dev_mask, V)
+        np.testing.assert_array_equal(tok.cpu().numpy(), cpu_greedy(logits, allowed))
+        np.testing.assert_array_equal(raw_bits(x)[rows], reference_masked(logits[rows], allowed[rows]))
+        if mode != "step":
+            psc.psc_advance(c.h, c.st, tok, stat)
         torch.cuda.synchronize()
         t = tok.cpu().numpy()
         s = stat.cpu().numpy()
@@ -321,6 +411,29 @@ def test_state_reset_rows(psc):
         np.testing.assert_array_equal(dev[r].cpu().numpy().view(np.uint32), m0)
 
 
+def test_saved_tables_load_onto_the_device(psc, tmp_path):
+    """psc_save then psc_load: the loaded handle's device path gives the same
+    masks, masked logits and advanced states."""
+    c = case(psc, 2)
+    path = str(tmp_path / "json.psc")
+    psc.psc_save(c.h, path)
+    h2 = psc.psc_load(path)
+    w = c.w
+    st2 = psc.psc_state_init(h2, w.B, 256)
+    tm = torch.from_numpy(w.token_matrix()).cuda()
+    for j in range(tm.shape[1]):
+        psc.psc_advance(h2, st2, tm[:, j].contiguous())
+    ocs = []
+    for ids in w.prefix_ids:           # fresh configurations: other tests advance c.ocs
+        oc = c.o.initial()
+        c.o.advance_tokens(oc, c.voc, ids)
+        ocs.append(oc)
+    ref = c.o.masks(ocs, c.voc, threads=THREADS)
+    bm = torch.empty(w.B, h2.W, dtype=torch.int32, device="cuda")
+    psc.psc_fill_mask(h2, st2, bm)
+    np.testing.assert_array_equal(bm.cpu().numpy().view(np.uint32), ref)
+
+
 def test_bad_arguments_are_reported(psc):
     c = case(psc, 1)
     lib = psc.load()
@@ -331,3 +444,10 @@ def test_bad_arguments_are_reported(psc):
     assert lib.psc_apply_mask(x.data_ptr(), 7, c.w.V, bm.data_ptr(), c.w.B, c.w.V, None) == 1
     assert lib.psc_fill_mask(c.h.ptr, c.st.ptr, c.w.B, None, None) == 1
     assert b"bad arguments" in lib.psc_last_error()
+
+
+def test_no_device_wait_gave_up(psc):
+    """Every bounded wait inside the kernels (TMA pipeline, table staging) of all
+    the tests above completed: the process-wide timeout counter is still zero."""
+    c = case(psc, 1)
+    assert c.h.info().device_timeouts == 0

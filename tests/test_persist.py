@@ -1,0 +1,55 @@
+"""psc_save / psc_load: compiled tables round-trip through a file, and a
+corrupt or truncated file is refused (host tables, no GPU needed)."""
+from __future__ import annotations
+
+import os
+
+import numpy as np
+import pytest
+
+from workloads import configs
+
+
+@pytest.fixture(scope="module")
+def psc():
+    from paper_2608_03065_gb300 import build, psc as mod
+    build.build()
+    mod.load()
+    return mod
+
+
+def test_round_trip_gives_identical_masks(psc, tmp_path):
+    w = configs.load(2, batch=12)
+    h = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id, host_only=True)
+    path = str(tmp_path / "json.psc")
+    psc.psc_save(h, path)
+    h2 = psc.psc_load(path, host_only=True)
+    i1, i2 = h.info(), h2.info()
+    for f in ("V", "W", "n_lexer_states", "n_parser_states", "n_classifier_states", "n_masks", "eos_id",
+              "classifier_bytes", "mask_bytes"):
+        assert getattr(i1, f) == getattr(i2, f), f
+    for ids in w.prefix_ids:
+        c1, c2 = h.host_initial(), h2.host_initial()
+        for v in ids:
+            c1, c2 = h.host_advance(c1, v), h2.host_advance(c2, v)
+        assert c1 == c2
+        m1 = h.host_mask_row(h.host_classify(c1["q"], c1["stack"], c1["status"]))
+        m2 = h2.host_mask_row(h2.host_classify(c2["q"], c2["stack"], c2["status"]))
+        np.testing.assert_array_equal(m1, m2)
+
+
+def test_corrupt_and_truncated_files_are_refused(psc, tmp_path):
+    w = configs.load(1, batch=2)
+    h = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id, host_only=True)
+    path = str(tmp_path / "a.psc")
+    psc.psc_save(h, path)
+    data = bytearray(open(path, "rb").read())
+    bad = bytearray(data)
+    bad[len(bad) // 2] ^= 0x40
+    open(path + ".flip", "wb").write(bytes(bad))
+    open(path + ".cut", "wb").write(bytes(data[:len(data) // 3]))
+    open(path + ".junk", "wb").write(b"not a table file at all")
+    for suffix in (".flip", ".cut", ".junk", ".missing"):
+        with pytest.raises(psc.PscError) as e:
+            psc.psc_load(path + suffix, host_only=True)
+        assert e.value.code == 8, suffix
