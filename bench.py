@@ -1,10 +1,11 @@
 """Benchmark: masked decode steps on the 1024 x 262,144 C-like workload.
 
 One step = one pass of the whole per-step path over the batch, psc_decode_step:
-  k_apply_argmax   classify every row's parser stack (classifier DFA walk, inside
+  k_step_tma       classify every row's parser stack (classifier DFA walk, inside
                    the kernel), apply its precomputed mask to the bf16 logits in
                    place, write the packed bitmask [B][V/32], and pick the greedy
-                   token among the allowed ones, in one pass over the logits
+                   token among the allowed ones, in one TMA-pipelined pass over
+                   the logits
   k_advance_smem   lex + parse the chosen tokens on the device-resident stacks
 
 Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
@@ -33,7 +34,7 @@ sys.path.insert(0, ROOT)
 WORKLOAD = 5
 METRIC = "masked decode steps/s and µs/step at batch×vocab; HBM GB/s vs GB300 peak"
 UNIT = "steps/s"
-PROFILE_FILE = os.path.join(ROOT, "profiles", "k_apply_argmax_c5_traffic.txt")
+PROFILE_FILE = os.path.join(ROOT, "profiles", "k_step_tma_c5_traffic.txt")
 
 
 def measured_peaks():
@@ -350,7 +351,7 @@ def main():
         "decode_step_us": fused_avg_ms * 1000.0,
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "traffic": traffic,
-                     "kernel": "psc_decode_step (k_apply_argmax with in-kernel classification + k_advance_smem)",
+                     "kernel": "psc_decode_step (k_step_tma with in-kernel classification + k_advance_smem)",
                      "algorithmic_bytes": alg_bytes, "peak_kind": peak_kind},
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": B * V * 2,
                 "d2h_bytes_per_step": B * 4},

@@ -56,7 +56,7 @@ struct DevTables {
     const int64_t* vocab_off;
     int q0, nq, n_lr, n_terms, n_nts, end_term;
     int V, W, Wp, eos_id, n_masks;
-    // compact lexer/parser tables for k_advance_smem (adv_bytes = 0: not built)
+    // compact lexer/parser tables for k_advance_warp (adv_bytes = 0: not built)
     const uint8_t* adv;
     int adv_bytes, o_bc, o_trans, o_accept, o_ign, o_resolve, o_action, o_go, o_rlen, o_rlhs, nbc;
 };
@@ -80,6 +80,7 @@ struct psc_handle {
     DevTables d{};
     void* blocks[16] = {};
     int n_blocks = 0;
+    int tma_ctas[2] = {1, 1};   // resident k_step_tma CTAs per SM (bf16, f32)
 };
 
 struct psc_states {
@@ -565,7 +566,7 @@ __device__ __forceinline__ void apply_argmax_chunk_bf16(const uint16_t* src, uin
                 }
             }
         }
-        if (bk != 0xFFu) *reinterpret_cast<uint4*>(p) = make_uint4(x0, x1, x2, x3);
+        st_cs_v4(p, make_uint4(x0, x1, x2, x3));   // whole pieces: no partly written sectors
     }
 }
 
@@ -603,7 +604,97 @@ __device__ __forceinline__ void apply_argmax_chunk_f32(const uint32_t* src, uint
                 }
             }
         }
-        if (bk != 0xFu) *reinterpret_cast<uint4*>(p) = make_uint4(x0, x1, x2, x3);
+        st_cs_v4(p, make_uint4(x0, x1, x2, x3));
+    }
+}
+
+// Greedy state of a lane that streams bf16 chunks: the largest allowed value
+// seen so far and the 16-byte piece holding its first occurrence (the piece's
+// values and mask bits), resolved to a column once per work item.  The per-piece
+// update is a handful of selects, so no lane diverges while it streams.
+struct BestPiece {
+    float val;       // -inf until an allowed value is seen
+    int col;         // first column of the piece (-1: nothing yet)
+    uint32_t bits;   // the piece's mask bits
+    uint4 x;         // the piece's values
+};
+
+__device__ __forceinline__ BestPiece best_piece_none() {
+    return BestPiece{-INFINITY, -1, 0u, make_uint4(0u, 0u, 0u, 0u)};
+}
+
+// Column and key of the piece's first allowed value equal to the best.
+__device__ __forceinline__ unsigned long long best_piece_key_bf16(const BestPiece& bp) {
+    if (bp.col < 0) return 0ull;
+    uint32_t w[4] = {bp.x.x, bp.x.y, bp.x.z, bp.x.w};
+    int at = 0;
+#pragma unroll
+    for (int e = 7; e >= 0; e--)
+        if (((bp.bits >> e) & 1) && bf16_at(w[e >> 1], e & 1) == bp.val) at = e;
+    return make_key(f32_order(__float_as_uint(bp.val)), bp.col + at);
+}
+
+// A lane's four 16-byte pieces of a bf16 chunk in registers: the mask bits of
+// each piece and its values with -inf where masked.
+struct ChunkRegs {
+    uint32_t bits[4];
+    uint4 x[4];
+};
+
+// Reads the lane's pieces of one 1024-column bf16 chunk from shared memory
+// (pieces with nothing allowed are not read) and masks them.  The stage may be
+// handed back as soon as this returns.
+__device__ __forceinline__ void load_mask_chunk_bf16(const uint16_t* src, uint32_t word, int lane, const uint4* lut,
+                                                     ChunkRegs& r) {
+    uint4 v[4];
+#pragma unroll
+    for (int k = 0; k < 4; k++) r.bits[k] = (__shfl_sync(FULL, word, k * 8 + (lane >> 2)) >> ((lane & 3) * 8)) & 0xFFu;
+#pragma unroll
+    for (int k = 0; k < 4; k++)
+        v[k] = r.bits[k] ? *reinterpret_cast<const uint4*>(src + (k * 32 + lane) * 8) : make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+    for (int k = 0; k < 4; k++) {
+        uint4 am = lut[r.bits[k]];
+        r.x[k] = make_uint4(sel_ninf(v[k].x, am.x, 0xFF80FF80u), sel_ninf(v[k].y, am.y, 0xFF80FF80u),
+                            sel_ninf(v[k].z, am.z, 0xFF80FF80u), sel_ninf(v[k].w, am.w, 0xFF80FF80u));
+    }
+}
+
+// Folds a masked chunk into the lane's best piece with packed bf16x2 maxima (NaN
+// never wins: the maximum returns the other operand) and writes it to the row.
+// Every lane runs the same instructions for every piece; only a piece whose
+// allowed values are all -inf or NaN, met before any other allowed value, takes
+// a short scalar path.
+__device__ __forceinline__ void fold_store_chunk_bf16(uint16_t* row, int col0, int lane, const ChunkRegs& r,
+                                                      BestPiece& bp) {
+#pragma unroll
+    for (int k = 0; k < 4; k++) {
+        uint32_t bk = r.bits[k];
+        uint32_t x0 = r.x[k].x, x1 = r.x[k].y, x2 = r.x[k].z, x3 = r.x[k].w;
+        __nv_bfloat162 m = __hmax2(__hmax2(*reinterpret_cast<__nv_bfloat162*>(&x0), *reinterpret_cast<__nv_bfloat162*>(&x1)),
+                                   __hmax2(*reinterpret_cast<__nv_bfloat162*>(&x2), *reinterpret_cast<__nv_bfloat162*>(&x3)));
+        float mf = fmaxf(__low2float(m), __high2float(m));
+        int pc = col0 + (k * 32 + lane) * 8;
+        bool upd = mf > bp.val;
+        if (!upd && bk != 0u && bp.col < 0) {
+            // nothing allowed seen yet and this piece's allowed values are -inf or NaN:
+            // an allowed -inf is still a valid choice
+#pragma unroll
+            for (int e = 0; e < 8; e++) {
+                uint32_t wv = e < 2 ? x0 : e < 4 ? x1 : e < 6 ? x2 : x3;
+                if (((bk >> e) & 1) && bf16_at(wv, e & 1) == -INFINITY) upd = true;
+            }
+        }
+        bp.val = upd ? mf : bp.val;
+        bp.col = upd ? pc : bp.col;
+        bp.bits = upd ? bk : bp.bits;
+        bp.x.x = upd ? x0 : bp.x.x;
+        bp.x.y = upd ? x1 : bp.x.y;
+        bp.x.z = upd ? x2 : bp.x.z;
+        bp.x.w = upd ? x3 : bp.x.w;
+        // every piece is written, also one with every position allowed: a partly written
+        // 32-byte sector costs a read-modify-write when the L2 evicts it
+        st_cs_v4(row + pc, r.x[k]);
     }
 }
 
@@ -739,41 +830,18 @@ __global__ void k_finalize_tokens(unsigned long long* __restrict__ best_key, int
 }
 
 // ------------------------------------------- advance with staged tables
-// Same semantics as k_advance; the compact lexer/parser tables (int16
-// entries, byte classes for the lexer) are first copied to shared memory.
-// `top` mirrors st[depth - 1] in a register; only the state under a popped
-// handle is read back from the row's stack.
-__device__ int feed_class_smem(const uint8_t* sm, const DevTables& T, uint16_t* st, int& depth, int& top, int cap,
-                               int cls) {
-    const int16_t* resolve = reinterpret_cast<const int16_t*>(sm + T.o_resolve);
-    const int16_t* action = reinterpret_cast<const int16_t*>(sm + T.o_action);
-    const int16_t* go = reinterpret_cast<const int16_t*>(sm + T.o_go);
-    const uint8_t* rlen = sm + T.o_rlen;
-    const int16_t* rlhs = reinterpret_cast<const int16_t*>(sm + T.o_rlhs);
-    int t = resolve[cls * T.n_lr + top];
-    if (t < 0) return ROW_REJECTED;
-    for (int guard = 0; guard < 4 * cap + 64; guard++) {
-        int a = action[top * T.n_terms + t];
-        int kind = a & 3, val = (a >> 2) & 0x3FFF;
-        if (kind == psc::ACT_SHIFT) {
-            if (depth >= cap) return ROW_OVERFLOW;
-            st[depth++] = (uint16_t)val;
-            top = val;
-            return ROW_OK;
-        }
-        if (kind != psc::ACT_REDUCE) return ROW_REJECTED;
-        int k = rlen[val];
-        if (depth - k < 1) return ROW_REJECTED;
-        depth -= k;
-        int under = k ? st[depth - 1] : top;
-        int g = go[under * T.n_nts + rlhs[val]];
-        if (g < 0) return ROW_REJECTED;
-        if (depth >= cap) return ROW_OVERFLOW;
-        st[depth++] = (uint16_t)g;
-        top = g;
-    }
-    return ROW_LIMIT;
-}
+// One warp per row.  The compact lexer/parser tables (int16 entries, byte
+// classes for the lexer) are staged in shared memory by one bulk copy per CTA,
+// and the top ADV_KEEP entries of the row's stack are copied into a per-warp
+// window, so the parser's dependent reads are shared-memory reads.  After the
+// token is consumed the warp walks the classifier for the new configuration
+// (Algorithm 2 step 3) and stores the row's mask id for the next masking pass.
+constexpr int ADV_WARPS = 8;     // rows per CTA
+constexpr int ADV_WIN = 256;     // stack entries held per row
+constexpr int ADV_KEEP = 192;    // entries copied in (the rest is room for pushes)
+
+// Dynamic shared memory of k_advance_warp: the staged tables, then the stack windows.
+int adv_smem(const DevTables& d) { return d.adv_bytes + ADV_WARPS * ADV_WIN * 2; }
 
 __device__ __forceinline__ uint32_t smem_addr(const void* p) {
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -793,8 +861,87 @@ __device__ __forceinline__ bool mbar_wait0(uint32_t bar, int limit) {
     return false;
 }
 
-__global__ void k_advance_smem(DevTables T, DevStates S, const int32_t* tokens, int B, int use_mid,
-                               int32_t* status_out, int from_keys, int32_t* tokens_out) {
+// A row's stack seen through its window: indices in [base, base + ADV_WIN) live
+// in shared memory, the others in global memory.  `lo` tracks the lowest window
+// index written (for the write-back).
+struct StackView {
+    uint16_t* win;
+    uint16_t* st;
+    int base;
+    int lo;
+    __device__ __forceinline__ bool in_win(int i) const { return i >= base && i < base + ADV_WIN; }
+    __device__ __forceinline__ int get(int i) const { return in_win(i) ? win[i - base] : st[i]; }
+    __device__ __forceinline__ void set(int i, int v) {
+        if (in_win(i)) {
+            win[i - base] = (uint16_t)v;
+            lo = i < lo ? i : lo;
+        } else {
+            st[i] = (uint16_t)v;
+        }
+    }
+};
+
+// Feed one lexeme class to the parser: resolve it to a terminal with the
+// current top (contextual lexing), reduce until it is shifted.  Returns a row status.
+__device__ int feed_class_win(const uint8_t* sm, const DevTables& T, StackView& sv, int& depth, int& top, int cap,
+                              int cls) {
+    const int16_t* resolve = reinterpret_cast<const int16_t*>(sm + T.o_resolve);
+    const int16_t* action = reinterpret_cast<const int16_t*>(sm + T.o_action);
+    const int16_t* go = reinterpret_cast<const int16_t*>(sm + T.o_go);
+    const uint8_t* rlen = sm + T.o_rlen;
+    const int16_t* rlhs = reinterpret_cast<const int16_t*>(sm + T.o_rlhs);
+    int t = resolve[cls * T.n_lr + top];
+    if (t < 0) return ROW_REJECTED;
+    for (int guard = 0; guard < 4 * cap + 64; guard++) {
+        int a = action[top * T.n_terms + t];
+        int kind = a & 3, val = (a >> 2) & 0x3FFF;
+        if (kind == psc::ACT_SHIFT) {
+            if (depth >= cap) return ROW_OVERFLOW;
+            sv.set(depth++, val);
+            top = val;
+            return ROW_OK;
+        }
+        if (kind != psc::ACT_REDUCE) return ROW_REJECTED;
+        int k = rlen[val];
+        if (depth - k < 1) return ROW_REJECTED;
+        depth -= k;
+        int under = k ? sv.get(depth - 1) : top;
+        int g = go[under * T.n_nts + rlhs[val]];
+        if (g < 0) return ROW_REJECTED;
+        if (depth >= cap) return ROW_OVERFLOW;
+        sv.set(depth++, g);
+        top = g;
+    }
+    return ROW_LIMIT;
+}
+
+// Classifier walk of a configuration (lexer state q, stack of the given depth
+// read through the view) by a full warp: lanes fetch 32 stack symbols at a time,
+// the walk broadcasts them with shuffles.  Every lane returns the mask id.
+__device__ int warp_walk(const DevTables& T, const StackView& sv, int q, int depth, int lane) {
+    if (q < 0 || q >= T.nq || depth < 1) return 0;
+    int s = __ldg(T.dfa_start + q);
+    if (s < 0) return -s - 1;
+    for (int top = depth - 1; top >= 0; top -= 32) {
+        int i = top - lane;
+        int x = i >= 0 ? sv.get(i) : 0;
+        int n = top + 1 < 32 ? top + 1 : 32;
+        for (int j = 0; j < n; j++) {
+            int X = __shfl_sync(FULL, x, j);
+            int nx = __ldg(T.dfa + (size_t)s * T.n_lr + X);
+            if (nx < 0) return -nx - 1;
+            s = nx;
+        }
+    }
+    return __ldg(T.dfa_mask + s);
+}
+
+// Algorithm 2 steps 1-3 for one row per warp: consume the row's token (the
+// given one, or the greedy choice of the fused masking pass when from_keys),
+// then classify the new configuration into S.mid.
+__global__ void __launch_bounds__(ADV_WARPS * 32) k_advance_warp(DevTables T, DevStates S, const int32_t* tokens,
+                                                                 int B, int use_mid, int32_t* status_out,
+                                                                 int from_keys, int32_t* tokens_out) {
     extern __shared__ uint4 smem4[];
     __shared__ __align__(8) uint64_t bar;
     uint8_t* sm = reinterpret_cast<uint8_t*>(smem4);
@@ -809,17 +956,21 @@ __global__ void k_advance_smem(DevTables T, DevStates S, const int32_t* tokens, 
                      : "memory");
     }
     __syncthreads();
-    bool staged = mbar_wait0(bar_a, 1 << 24);
-    int b = blockIdx.x * blockDim.x + threadIdx.x;
+    bool staged = __all_sync(FULL, mbar_wait0(bar_a, 1 << 24));
+    int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    int b = blockIdx.x * ADV_WARPS + warp;
     if (!staged) {
         // the copy did not land: give the rows a LIMIT status, wait (bounded) for the copy, return
         if (threadIdx.x == 0) atomicAdd(&g_pipeline_timeouts, 1);
-        if (b < B && S.status[b] == ROW_OK) S.status[b] = ROW_LIMIT;
-        if (b < B && from_keys) {
-            tokens_out[b] = -1;
-            S.best[b] = 0ull;
+        if (b < B && lane == 0) {
+            if (S.status[b] == ROW_OK) S.status[b] = ROW_LIMIT;
+            if (from_keys) {
+                tokens_out[b] = -1;
+                S.best[b] = 0ull;
+            }
+            if (status_out) status_out[b] = S.status[b];
+            S.mid[b] = 0;
         }
-        if (b < B && status_out) status_out[b] = S.status[b];
         mbar_wait0(bar_a, 1 << 24);
         return;
     }
@@ -828,16 +979,25 @@ __global__ void k_advance_smem(DevTables T, DevStates S, const int32_t* tokens, 
     const int16_t* trans = reinterpret_cast<const int16_t*>(sm + T.o_trans);
     const int16_t* acc = reinterpret_cast<const int16_t*>(sm + T.o_accept);
     const uint8_t* ign = sm + T.o_ign;
-    int tok;
-    if (from_keys) {   // the greedy choice of the fused masking pass
-        unsigned long long k = S.best[b];
-        S.best[b] = 0ull;
-        tok = k ? (int32_t)(~(uint32_t)(k & 0xFFFFFFFFu)) : -1;
-        tokens_out[b] = tok;
-    } else {
-        tok = tokens[b];
+    StackView sv{reinterpret_cast<uint16_t*>(sm + T.adv_bytes) + warp * ADV_WIN, S.stack + (size_t)b * S.cap, 0,
+                 0x7FFFFFFF};
+    int tok = 0, status = ROW_OK;
+    if (lane == 0) {
+        if (from_keys) {   // the greedy choice of the fused masking pass
+            unsigned long long k = S.best[b];
+            S.best[b] = 0ull;
+            tok = k ? (int32_t)(~(uint32_t)(k & 0xFFFFFFFFu)) : -1;
+            tokens_out[b] = tok;
+        } else {
+            tok = tokens[b];
+        }
+        status = S.status[b];
     }
-    int status = S.status[b];
+    tok = __shfl_sync(FULL, tok, 0);
+    status = __shfl_sync(FULL, status, 0);
+    int q = S.q[b], depth = S.depth[b];
+    bool parse = false;
+    uint32_t mword = 0;
     if (tok >= 0) {
         if (status == ROW_DONE) {
             status = tok == T.eos_id ? ROW_DONE : ROW_REJECTED;
@@ -845,51 +1005,92 @@ __global__ void k_advance_smem(DevTables T, DevStates S, const int32_t* tokens, 
             if (tok >= T.V) {
                 status = ROW_REJECTED;
             } else {
-                int mid = use_mid ? S.mid[b] : thread_classify(T, S, b);
-                // the mask bit is loaded now and tested once the token is parsed: the row
-                // is only committed (q, depth) when the token was allowed
-                uint32_t mword = __ldg(T.masks + (size_t)mid * T.Wp + (tok >> 5));
-                if (tok == T.eos_id) {
-                    status = ((mword >> (tok & 31)) & 1) ? ROW_DONE : ROW_REJECTED;
+                int mid;
+                if (use_mid) {
+                    mid = S.mid[b];
                 } else {
-                    int q = S.q[b], depth = S.depth[b];
-                    uint16_t* st = S.stack + (size_t)b * S.cap;
-                    int top = st[depth - 1];
-                    int64_t lo = T.vocab_off[tok], hi = T.vocab_off[tok + 1];
-                    int len = (int)(hi - lo);
-                    // the token's bytes, fetched together (tokens up to 32 bytes)
-                    uint32_t tw[8] = {0, 0, 0, 0, 0, 0, 0, 0};
-#pragma unroll
-                    for (int i = 0; i < 32; i++)
-                        if (i < len) tw[i >> 2] |= (uint32_t)T.vocab[lo + i] << (8 * (i & 3));
-                    for (int i = 0; i < len && status == ROW_OK; i++) {
-                        int byte = i < 32 ? (int)((tw[i >> 2] >> (8 * (i & 3))) & 0xFFu) : (int)T.vocab[lo + i];
-                        int c = bc[byte];
-                        int nx = trans[q * T.nbc + c];
-                        if (nx >= 0) {
-                            q = nx;
-                            continue;
-                        }
-                        int cls = q == T.q0 ? -1 : acc[q];
-                        if (cls < 0) {
-                            status = ROW_REJECTED;
-                            break;
-                        }
-                        if (!ign[cls]) status = feed_class_smem(sm, T, st, depth, top, S.cap, cls);
-                        q = trans[T.q0 * T.nbc + c];
-                        if (q < 0) status = ROW_REJECTED;
-                    }
-                    if (!((mword >> (tok & 31)) & 1)) status = ROW_REJECTED;
-                    if (status == ROW_OK) {
-                        S.q[b] = q;
-                        S.depth[b] = depth;
-                    }
+                    StackView g{nullptr, sv.st, 0x40000000, 0x7FFFFFFF};   // all of the stack in global memory
+                    mid = depth >= 1 && depth <= S.cap ? warp_walk(T, g, q, depth, lane) : 0;
                 }
+                // the token's mask bit; the row is only committed (q, depth) when it is set
+                mword = __ldg(T.masks + (size_t)mid * T.Wp + (tok >> 5));
+                if (tok == T.eos_id) status = ((mword >> (tok & 31)) & 1) ? ROW_DONE : ROW_REJECTED;
+                else parse = true;
             }
         }
-        S.status[b] = status;
     }
-    if (status_out) status_out[b] = status;
+    if (parse) {
+        if (depth < 1 || depth > S.cap) {
+            parse = false;
+            status = ROW_REJECTED;
+        }
+    }
+    if (parse) {
+        sv.base = depth > ADV_KEEP ? depth - ADV_KEEP : 0;
+        for (int i = lane; i < depth - sv.base; i += 32) sv.win[i] = sv.st[sv.base + i];
+        __syncwarp();
+        int nq = q, nd = depth;
+        if (lane == 0) {
+            int top = sv.win[depth - 1 - sv.base];
+            int64_t lo = T.vocab_off[tok], hi = T.vocab_off[tok + 1];
+            int len = (int)(hi - lo);
+            // the token's bytes, fetched together (tokens up to 32 bytes)
+            uint32_t tw[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+#pragma unroll
+            for (int i = 0; i < 32; i++)
+                if (i < len) tw[i >> 2] |= (uint32_t)T.vocab[lo + i] << (8 * (i & 3));
+            for (int i = 0; i < len && status == ROW_OK; i++) {
+                int byte = i < 32 ? (int)((tw[i >> 2] >> (8 * (i & 3))) & 0xFFu) : (int)T.vocab[lo + i];
+                int c = bc[byte];
+                int nx = trans[nq * T.nbc + c];
+                if (nx >= 0) {
+                    nq = nx;
+                    continue;
+                }
+                int cls = nq == T.q0 ? -1 : acc[nq];
+                if (cls < 0) {
+                    status = ROW_REJECTED;
+                    break;
+                }
+                if (!ign[cls]) status = feed_class_win(sm, T, sv, nd, top, S.cap, cls);
+                nq = trans[T.q0 * T.nbc + c];
+                if (nq < 0) status = ROW_REJECTED;
+            }
+            if (!((mword >> (tok & 31)) & 1)) status = ROW_REJECTED;
+            if (status == ROW_OK) {
+                S.q[b] = nq;
+                S.depth[b] = nd;
+            }
+        }
+        status = __shfl_sync(FULL, status, 0);
+        q = __shfl_sync(FULL, nq, 0);
+        depth = __shfl_sync(FULL, nd, 0);
+        sv.lo = __shfl_sync(FULL, sv.lo, 0);
+        __syncwarp();
+        if (status == ROW_OK) {
+            // window entries from the lowest one written up to the new depth (lo stays
+            // INT_MAX when nothing was written: clamp before adding the lane)
+            int hi = depth < sv.base + ADV_WIN ? depth : sv.base + ADV_WIN;
+            int from = sv.lo > sv.base ? sv.lo : sv.base;
+            from = from < hi ? from : hi;
+            for (int i = from + lane; i < hi; i += 32) sv.st[i] = sv.win[i - sv.base];
+        }
+    }
+    if (lane == 0) {
+        if (tok >= 0) S.status[b] = status;
+        if (status_out) status_out[b] = status;
+    }
+    // the next masking pass's mask id
+    int mid;
+    if (status == ROW_DONE) {
+        mid = 1;
+    } else if (status != ROW_OK) {
+        mid = 0;
+    } else {
+        if (!parse) sv.base = 0x40000000;   // window not loaded: read the stack from global memory
+        mid = depth >= 1 && depth <= S.cap ? warp_walk(T, sv, q, depth, lane) : 0;
+    }
+    if (lane == 0) S.mid[b] = mid;
 }
 
 // ------------------------------------------ TMA-pipelined decode masking pass
@@ -922,40 +1123,62 @@ __device__ __forceinline__ void tma_load_1d(uint32_t dst, const void* src, uint3
                  ::"r"(dst), "l"(src), "r"(bytes), "r"(bar)
                  : "memory");
 }
+// The same with an L2 cache policy (the streamed logits go first when L2 evicts,
+// so the classifier table and mask rows the walks and the mask copies read stay).
+__device__ __forceinline__ void tma_load_1d_hint(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar,
+                                                 uint64_t policy) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], %4;"
+        ::"r"(dst), "l"(src), "r"(bytes), "r"(bar), "l"(policy)
+        : "memory");
+}
+__device__ __forceinline__ uint64_t l2_evict_first_policy() {
+    uint64_t p;
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+    return p;
+}
 
 
-constexpr int TMA_SEG = 32;     // 1024-column chunks per work item
-constexpr int TMA_NCONS = 6;    // consumer warps (warp 0 produces, warp 1 classifies)
+constexpr int TMA_SEG = 32;     // 1024-column chunks per work item (one per lane of a warp)
+constexpr int TMA_NCONS = 8;    // consumer warps; a ring stage holds one chunk for each of them
+constexpr int TMA_WARPS = TMA_NCONS + 2;   // + producer + walker
+constexpr int TMA_MIDS = 4;     // classified rows the walker may run ahead (it walks them together)
+constexpr int TMA_MSLOTS = 3;   // mask-word buffers: the next item's words load while this item streams
 
-// Ring stages: a multiple of the consumer count, so that stage s is always
-// consumed by warp 2 + s % TMA_NCONS and every waiter of a full barrier waits
-// for its rounds in order (a parity wait cannot tell round r from r + 2).
+// Shared-memory plan of the pipelined pass: NS ring stages of TMA_NCONS chunks,
+// TMA_MSLOTS mask-word buffers (TMA_SEG x 32 words each), then the mbarriers.
 template <typename T>
 struct TmaShape {
-    static constexpr int NS = sizeof(T) == 2 ? 18 : 6;
-    static constexpr int TILE = 1024 * (int)sizeof(T);   // one chunk
-    static constexpr int SMEM = NS * TILE + 2 * TMA_SEG * 32 * 4 + (2 * NS + 8) * 8;
+    static constexpr int CHUNK = 1024 * (int)sizeof(T);   // bytes of one 1024-column chunk
+    static constexpr int STAGE = TMA_NCONS * CHUNK;
+    static constexpr int NS = sizeof(T) == 2 ? 3 : 2;
+    static constexpr int NBARS = 2 * NS + 2 * TMA_MSLOTS + 2 * TMA_MIDS;
+    static constexpr int SMEM = NS * STAGE + TMA_MSLOTS * TMA_SEG * 32 * 4 + NBARS * 8;
 };
 
 // One decode masking pass (classification, mask, apply, greedy key) with the
 // logits streamed through shared memory by TMA bulk copies.  Work item = (row,
-// segment of TMA_SEG chunks).  Warp 0 (producer) copies the item's mask words
-// and every chunk that holds an allowed position into a ring of NS stages
-// (chunks with nothing allowed are not read); warp 1 walks the classifier for
-// the CTA's upcoming rows; warps 2-7 take the chunks round-robin, write -inf
-// where masked and fold allowed values into the row's greedy key.
+// segment of TMA_SEG chunks).  Warp 0 (producer) fetches each item's mask words
+// one item ahead, then for every ring stage copies the stage's chunks that hold
+// an allowed position (runs of neighbouring chunks in one copy; chunks with
+// nothing allowed are not read); warp 1 walks the classifier for the CTA's
+// upcoming rows; consumer warp c takes chunk c of every stage, writes -inf where
+// masked and folds allowed values into the row's greedy key.
 // Requires 16-byte aligned rows; rows' mask rows padded to whole chunks.
 template <typename T>
-__global__ void __launch_bounds__(256, 4) k_step_tma(T* logits, int64_t stride, int B, int V, uint32_t* copy_out,
-                                                     unsigned long long* __restrict__ best_key, DevTables D,
-                                                     DevStates S) {
-    constexpr int NS = TmaShape<T>::NS, TILE = TmaShape<T>::TILE;
-    static_assert(NS % TMA_NCONS == 0, "each ring stage must belong to one consumer warp");
+__global__ void __launch_bounds__(TMA_WARPS * 32, 3) k_step_tma(T* logits, int64_t stride, int B, int V,
+                                                                uint32_t* copy_out,
+                                                                unsigned long long* __restrict__ best_key,
+                                                                DevTables D, DevStates S, int have_mid) {
+    using Sh = TmaShape<T>;
+    constexpr int NS = Sh::NS, CHUNK = Sh::CHUNK, STAGE = Sh::STAGE;
+    static_assert(TMA_SEG == 32, "one lane per chunk of an item");
+    static_assert(TMA_NCONS <= 32 && TMA_SEG % TMA_NCONS == 0, "whole stages per item");
     extern __shared__ __align__(128) uint8_t smem[];
     uint8_t* tiles = smem;
-    uint32_t* mbuf = reinterpret_cast<uint32_t*>(smem + NS * TILE);
-    uint64_t* bars = reinterpret_cast<uint64_t*>(mbuf + 2 * TMA_SEG * 32);
-    __shared__ int s_mid[2];
+    uint32_t* mbuf = reinterpret_cast<uint32_t*>(smem + NS * STAGE);
+    uint64_t* bars = reinterpret_cast<uint64_t*>(mbuf + TMA_MSLOTS * TMA_SEG * 32);
+    __shared__ int s_mid[TMA_MIDS];
     __shared__ uint4 s_lut[256];
     int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     int cpr = (V + 1023) >> 10;
@@ -963,15 +1186,17 @@ __global__ void __launch_bounds__(256, 4) k_step_tma(T* logits, int64_t stride, 
     build_allow_lut<T>(s_lut);
     long items = (long)B * nseg;
     const uint32_t full0 = smem_addr(bars), empty0 = full0 + 8 * NS, mfull0 = empty0 + 8 * NS;
-    const uint32_t mempty0 = mfull0 + 16, midf0 = mfull0 + 32, mide0 = mfull0 + 48;
+    const uint32_t mempty0 = mfull0 + 8 * TMA_MSLOTS, midf0 = mempty0 + 8 * TMA_MSLOTS, mide0 = midf0 + 8 * TMA_MIDS;
     if (threadIdx.x == 0) {
         for (int k = 0; k < NS; k++) {
             mbar_init(full0 + 8 * k, 1);
-            mbar_init(empty0 + 8 * k, 1);
+            mbar_init(empty0 + 8 * k, TMA_NCONS);
         }
-        for (int k = 0; k < 2; k++) {
+        for (int k = 0; k < TMA_MSLOTS; k++) {
             mbar_init(mfull0 + 8 * k, 1);
             mbar_init(mempty0 + 8 * k, TMA_NCONS);
+        }
+        for (int k = 0; k < TMA_MIDS; k++) {
             mbar_init(midf0 + 8 * k, 1);
             mbar_init(mide0 + 8 * k, 1);
         }
@@ -982,46 +1207,69 @@ __global__ void __launch_bounds__(256, 4) k_step_tma(T* logits, int64_t stride, 
     bool failed = false;
     if (warp == 0) {
         // ---------------------------------------------------------- producer
-        long t = 0;
+        long s = 0;            // ring stages issued
+        int issued = -1;       // last item whose mask words were requested
+        const uint64_t stream_policy = l2_evict_first_policy();
+        // request item ii's mask words (its row classified by the walker) into slot ii % TMA_MSLOTS
+        auto fetch_mask = [&](int ii, long itm) -> bool {
+            int b = (int)(itm / nseg), sg = (int)(itm - (long)b * nseg);
+            int c0 = sg * TMA_SEG, nch = min(TMA_SEG, cpr - c0);
+            int ms = ii % TMA_MIDS;
+            if (!__shfl_sync(FULL, (int)mbar_wait(midf0 + 8 * ms, (uint32_t)((ii / TMA_MIDS) & 1)), 0)) return false;
+            int mid = s_mid[ms];
+            __syncwarp();
+            int slot = ii % TMA_MSLOTS, use = ii / TMA_MSLOTS;
+            if (lane == 0) {
+                mbar_arrive(mide0 + 8 * ms);
+                if (sg == 0 && !have_mid) S.mid[b] = mid;
+            }
+            if (use >= 1 && !__shfl_sync(FULL, (int)mbar_wait(mempty0 + 8 * slot, (uint32_t)((use - 1) & 1)), 0))
+                return false;
+            if (lane == 0) {
+                mbar_arrive_tx(mfull0 + 8 * slot, nch * 128);
+                tma_load_1d(smem_addr(mbuf + slot * TMA_SEG * 32), D.masks + (size_t)mid * D.Wp + (size_t)c0 * 32,
+                            nch * 128, mfull0 + 8 * slot);
+            }
+            issued = ii;
+            return true;
+        };
         int i = 0;
-        int issued_mask = -1;
+        if ((long)blockIdx.x < items && !fetch_mask(0, blockIdx.x)) failed = true;
         for (long it = blockIdx.x; it < items && !failed; it += gridDim.x, i++) {
             int b = (int)(it / nseg), sg = (int)(it - (long)b * nseg);
             int c0 = sg * TMA_SEG, nch = min(TMA_SEG, cpr - c0);
-            int slot = i & 1;
-            uint32_t ph = (i >> 1) & 1;
-            if (!__shfl_sync(FULL, (int)mbar_wait(midf0 + 8 * slot, ph), 0)) { failed = true; break; }
-            int mid = s_mid[slot];
-            __syncwarp();
-            if (lane == 0) {
-                mbar_arrive(mide0 + 8 * slot);
-                if (sg == 0) S.mid[b] = mid;
-            }
-            if (i >= 2 && !__shfl_sync(FULL, (int)mbar_wait(mempty0 + 8 * slot, ((i >> 1) - 1) & 1), 0)) {
+            if (it + gridDim.x < items && !fetch_mask(i + 1, it + gridDim.x)) { failed = true; break; }
+            int slot = i % TMA_MSLOTS;
+            if (!__shfl_sync(FULL, (int)mbar_wait(mfull0 + 8 * slot, (uint32_t)((i / TMA_MSLOTS) & 1)), 0)) {
                 failed = true;
                 break;
             }
-            uint32_t* mb = mbuf + slot * TMA_SEG * 32;
-            if (lane == 0) {
-                mbar_arrive_tx(mfull0 + 8 * slot, nch * 128);
-                tma_load_1d(smem_addr(mb), D.masks + (size_t)mid * D.Wp + (size_t)c0 * 32, nch * 128, mfull0 + 8 * slot);
-            }
-            issued_mask = i;
-            if (!__shfl_sync(FULL, (int)mbar_wait(mfull0 + 8 * slot, ph), 0)) { failed = true; break; }
+            // lane k: does chunk k of the item hold an allowed position?  (rotated reads: no bank conflicts)
+            const uint32_t* mb = mbuf + slot * TMA_SEG * 32;
+            uint32_t acc = 0;
+#pragma unroll 8
+            for (int k = 0; k < 32; k++) acc |= mb[lane * 32 + ((k + lane) & 31)];
+            uint32_t load = __ballot_sync(FULL, acc != 0u && lane < nch);
+            if (c0 + nch == cpr && (V & 1023)) load &= ~(1u << (nch - 1));   // the ragged chunk is read directly
             const T* row = logits + (size_t)b * stride;
-            for (int k = 0; k < nch; k++, t++) {
-                int j = c0 + k;
-                int stg = (int)(t % NS);
-                if (t >= NS && !__shfl_sync(FULL, (int)mbar_wait(empty0 + 8 * stg, (uint32_t)(((t / NS) - 1) & 1)), 0)) {
+            for (int g = 0; g * TMA_NCONS < nch; g++, s++) {
+                int stg = (int)(s % NS);
+                if (s >= NS && !__shfl_sync(FULL, (int)mbar_wait(empty0 + 8 * stg, (uint32_t)(((s / NS) - 1) & 1)), 0)) {
                     failed = true;
                     break;
                 }
-                bool any = __ballot_sync(FULL, mb[k * 32 + lane] != 0u) != 0u;
-                bool ragged = (j == cpr - 1) && (V & 1023);
                 if (lane == 0) {
-                    if (any && !ragged) {
-                        mbar_arrive_tx(full0 + 8 * stg, TILE);
-                        tma_load_1d(smem_addr(tiles + stg * TILE), row + (size_t)j * 1024, TILE, full0 + 8 * stg);
+                    uint32_t f = (load >> (g * TMA_NCONS)) & ((1u << TMA_NCONS) - 1u);
+                    if (f) {
+                        mbar_arrive_tx(full0 + 8 * stg, (uint32_t)(__popc(f) * CHUNK));
+                        while (f) {
+                            int a = __ffs(f) - 1;
+                            int len = __ffs(~(f >> a)) - 1;
+                            tma_load_1d_hint(smem_addr(tiles + stg * STAGE + a * CHUNK),
+                                             row + (size_t)(c0 + g * TMA_NCONS + a) * 1024, (uint32_t)(len * CHUNK),
+                                             full0 + 8 * stg, stream_policy);
+                            f &= ~(((1u << len) - 1u) << a);
+                        }
                     } else {
                         mbar_arrive(full0 + 8 * stg);
                     }
@@ -1030,77 +1278,104 @@ __global__ void __launch_bounds__(256, 4) k_step_tma(T* logits, int64_t stride, 
         }
         if (failed && lane == 0) {
             // let this CTA's copies in flight land before it exits (bounded)
-            for (long tt = t > NS ? t - NS : 0; tt < t; tt++) mbar_wait(full0 + 8 * (int)(tt % NS), (uint32_t)((tt / NS) & 1));
-            if (issued_mask >= 0) mbar_wait(mfull0 + 8 * (issued_mask & 1), (issued_mask >> 1) & 1);
+            for (long tt = s > NS ? s - NS : 0; tt < s; tt++) mbar_wait(full0 + 8 * (int)(tt % NS), (uint32_t)((tt / NS) & 1));
+            for (int ii = issued > 0 ? issued - 1 : 0; ii <= issued; ii++)
+                mbar_wait(mfull0 + 8 * (ii % TMA_MSLOTS), (uint32_t)((ii / TMA_MSLOTS) & 1));
         }
     } else if (warp == 1) {
         // ------------------------------------------------------------ walker
+        // lanes 0..TMA_MIDS-1 each classify one of the next TMA_MIDS items' rows, so
+        // the dependent table loads of those walks overlap
         int i = 0;
-        for (long it = blockIdx.x; it < items; it += gridDim.x, i++) {
-            int slot = i & 1;
-            if (i >= 2 && !__shfl_sync(FULL, (int)mbar_wait(mide0 + 8 * slot, ((i >> 1) - 1) & 1), 0)) {
+        for (long it = blockIdx.x; it < items && !failed; it += (long)gridDim.x * TMA_MIDS, i += TMA_MIDS) {
+            if (i >= TMA_MIDS && !__shfl_sync(FULL, (int)mbar_wait(mide0 + 8 * (TMA_MIDS - 1),
+                                                                    ((i / TMA_MIDS) - 1) & 1), 0)) {
                 failed = true;
                 break;
             }
-            int mid = warp_classify(D, S, (int)(it / nseg), lane);
-            if (lane == 0) {
-                s_mid[slot] = mid;
-                mbar_arrive(midf0 + 8 * slot);
+            long my = it + (long)lane * gridDim.x;
+            int mid = 0;
+            if (lane < TMA_MIDS && my < items) {
+                int rb = (int)(my / nseg);
+                mid = have_mid ? S.mid[rb] : thread_classify(D, S, rb);
             }
+            if (lane < TMA_MIDS && my < items) {
+                s_mid[lane] = mid;
+                mbar_arrive(midf0 + 8 * lane);
+            }
+            __syncwarp();
         }
     } else {
         // --------------------------------------------------------- consumers
         int c = warp - 2;
-        long t = 0;
+        long s = 0;
         int i = 0;
         for (long it = blockIdx.x; it < items && !failed; it += gridDim.x, i++) {
             int b = (int)(it / nseg), sg = (int)(it - (long)b * nseg);
             int c0 = sg * TMA_SEG, nch = min(TMA_SEG, cpr - c0);
-            int slot = i & 1;
-            if (!__shfl_sync(FULL, (int)mbar_wait(mfull0 + 8 * slot, (i >> 1) & 1), 0)) { failed = true; break; }
+            int slot = i % TMA_MSLOTS;
+            if (!__shfl_sync(FULL, (int)mbar_wait(mfull0 + 8 * slot, (uint32_t)((i / TMA_MSLOTS) & 1)), 0)) {
+                failed = true;
+                break;
+            }
             const uint32_t* mb = mbuf + slot * TMA_SEG * 32;
             T* row = logits + (size_t)b * stride;
             Best best{0.f, -1};
-            int k0 = (int)((c - (t % TMA_NCONS) + TMA_NCONS) % TMA_NCONS);
-            for (int k = k0; k < nch; k += TMA_NCONS) {
-                long tt = t + k;
-                int stg = (int)(tt % NS);
-                int j = c0 + k;
-                if (!__shfl_sync(FULL, (int)mbar_wait(full0 + 8 * stg, (uint32_t)((tt / NS) & 1)), 0)) {
+            BestPiece bp = best_piece_none();
+            for (int g = 0; g * TMA_NCONS < nch; g++, s++) {
+                int stg = (int)(s % NS);
+                if (!__shfl_sync(FULL, (int)mbar_wait(full0 + 8 * stg, (uint32_t)((s / NS) & 1)), 0)) {
                     failed = true;
                     break;
                 }
-                uint32_t w = mb[k * 32 + lane];
-                if (copy_out) {
-                    int wi = j * 32 + lane;
-                    if (wi < D.W) copy_out[(size_t)b * D.W + wi] = w;
-                }
-                int col0 = j << 10;
-                if ((j == cpr - 1) && (V & 1023)) {
-                    apply_argmax_chunk_scalar<T>(row, col0, V - col0, w, lane, best);
-                } else if (__ballot_sync(FULL, w != 0u) == 0u) {
-                    constexpr int PIECES = TILE / 16 / 32;
-                    uint4 ninf = make_uint4(NegInf<T>::pair, NegInf<T>::pair, NegInf<T>::pair, NegInf<T>::pair);
+                int k = g * TMA_NCONS + c;
+                bool released = false;
+                if (k < nch) {
+                    int j = c0 + k;
+                    uint32_t w = mb[k * 32 + lane];
+                    if (copy_out) {
+                        int wi = j * 32 + lane;
+                        if (wi < D.W) copy_out[(size_t)b * D.W + wi] = w;
+                    }
+                    int col0 = j << 10;
+                    const uint8_t* tile = tiles + stg * STAGE + c * CHUNK;
+                    if ((j == cpr - 1) && (V & 1023)) {
+                        apply_argmax_chunk_scalar<T>(row, col0, V - col0, w, lane, best);
+                    } else if (__ballot_sync(FULL, w != 0u) == 0u) {
+                        constexpr int PIECES = CHUNK / 16 / 32;
+                        uint4 ninf = make_uint4(NegInf<T>::pair, NegInf<T>::pair, NegInf<T>::pair, NegInf<T>::pair);
 #pragma unroll
-                    for (int q = 0; q < PIECES; q++)
-                        st_cs_v4(reinterpret_cast<uint8_t*>(row + col0) + (q * 32 + lane) * 16, ninf);
-                } else if (sizeof(T) == 2) {
-                    apply_argmax_chunk_bf16(reinterpret_cast<const uint16_t*>(tiles + stg * TILE),
-                                            reinterpret_cast<uint16_t*>(row), col0, w, lane, best, s_lut);
-                } else {
-                    apply_argmax_chunk_f32(reinterpret_cast<const uint32_t*>(tiles + stg * TILE),
-                                           reinterpret_cast<uint32_t*>(row), col0, w, lane, best, s_lut);
+                        for (int q = 0; q < PIECES; q++)
+                            st_cs_v4(reinterpret_cast<uint8_t*>(row + col0) + (q * 32 + lane) * 16, ninf);
+                    } else if constexpr (sizeof(T) == 2) {
+                        // the chunk goes to registers and the stage back to the producer
+                        // before the chunk is folded and written out
+                        ChunkRegs r;
+                        load_mask_chunk_bf16(reinterpret_cast<const uint16_t*>(tile), w, lane, s_lut, r);
+                        __syncwarp();
+                        if (lane == 0) mbar_arrive(empty0 + 8 * stg);
+                        released = true;
+                        fold_store_chunk_bf16(reinterpret_cast<uint16_t*>(row), col0, lane, r, bp);
+                    } else {
+                        apply_argmax_chunk_f32(reinterpret_cast<const uint32_t*>(tile), reinterpret_cast<uint32_t*>(row),
+                                               col0, w, lane, best, s_lut);
+                    }
                 }
-                __syncwarp();
-                if (lane == 0) mbar_arrive(empty0 + 8 * stg);
+                if (!released) {
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(empty0 + 8 * stg);
+                }
             }
-            t += nch;
             unsigned long long key = best_key_of(best);
-#pragma unroll
-            for (int off = 16; off; off >>= 1) {
-                unsigned long long o = __shfl_xor_sync(FULL, key, off);
-                key = o > key ? o : key;
+            if constexpr (sizeof(T) == 2) {
+                unsigned long long kp = best_piece_key_bf16(bp);
+                key = kp > key ? kp : key;
             }
+            // warp maximum of the 64-bit keys: the high words, then the low words of the lanes holding it
+            uint32_t khi = (uint32_t)(key >> 32), klo = (uint32_t)key;
+            uint32_t mhi = __reduce_max_sync(FULL, khi);
+            uint32_t mlo = __reduce_max_sync(FULL, khi == mhi ? klo : 0u);
+            key = ((unsigned long long)mhi << 32) | mlo;
             if (lane == 0) {
                 if (key) atomicMax(best_key + b, key);
                 mbar_arrive(mempty0 + 8 * slot);
@@ -1182,6 +1457,33 @@ psc_status launch_apply(void* logits, psc_dtype dtype, int64_t row_stride, const
 
 // Masking + greedy choice with in-kernel classification; leaves each row's
 // key in st->d.best and its mask id in st->d.mid.
+// Algorithm 2 steps 1-2 for every row (the token given, or the fused pass's greedy
+// choice when d_tokens_out is set), then step 3 for the new configurations: the
+// rows' mask ids are current afterwards.
+psc_status launch_advance(const psc_handle* h, psc_states* st, const int32_t* d_tokens, int use_mid,
+                          int32_t* d_row_status, int32_t* d_tokens_out, cudaStream_t cs) {
+    int B = st->d.B;
+    int from_keys = d_tokens_out ? 1 : 0;
+    psc_status s;
+    if (h->d.adv_bytes > 0) {
+        k_advance_warp<<<(B + ADV_WARPS - 1) / ADV_WARPS, ADV_WARPS * 32, adv_smem(h->d), cs>>>(
+            h->d, st->d, d_tokens, B, use_mid, d_row_status, from_keys, d_tokens_out);
+        s = launch_check("k_advance_warp");
+    } else {
+        k_advance<<<(B + 127) / 128, 128, 0, cs>>>(h->d, st->d, d_tokens, B, use_mid, d_row_status, from_keys,
+                                                    d_tokens_out);
+        s = launch_check("k_advance");
+        if (s == PSC_OK) {
+            int threads = 256;
+            k_classify<<<(int)(((size_t)B * 32 + threads - 1) / threads), threads, 0, cs>>>(h->d, st->d, B);
+            s = launch_check("k_classify");
+        }
+    }
+    st->gen++;
+    if (s == PSC_OK) st->mid_gen = st->gen;
+    return s;
+}
+
 psc_status launch_fused(const psc_handle* h, const psc_states* st, void* d_logits, psc_dtype dtype, int64_t row_stride,
                         int V, uint32_t* d_bitmask_out, cudaStream_t cs) {
     int B = st->d.B;
@@ -1189,6 +1491,7 @@ psc_status launch_fused(const psc_handle* h, const psc_states* st, void* d_logit
     size_t esz = dtype == PSC_BF16 ? 2 : 4;
     int vec = aligned16(d_logits) && ((row_stride * (int64_t)esz) % 16 == 0);
     int cpr = (V + 1023) / 1024;
+    int have_mid = st->mid_gen == st->gen ? 1 : 0;   // mask ids current: no classifier walks
     int slots = sm_count(h->device) * 4;   // 4 resident CTAs of 256 threads per SM
     long seg = ((long)cpr * B) / (2L * slots);
     int seg_chunks = (int)std::max(1L, std::min(32L, seg));
@@ -1196,15 +1499,16 @@ psc_status launch_fused(const psc_handle* h, const psc_states* st, void* d_logit
     int grid = (int)std::max(1L, std::min<long>(items, slots));
     psc_status s;
     if (vec) {
-        // TMA pipeline: one item = (row, 32 chunks); 4 CTAs per SM
+        // TMA pipeline: one item = (row, 32 chunks); as many CTAs as are resident at once
         long titems = (long)B * ((cpr + TMA_SEG - 1) / TMA_SEG);
-        int tgrid = (int)std::max(1L, std::min<long>(titems, (long)sm_count(h->device) * 4));
+        long resident = (long)sm_count(h->device) * h->tma_ctas[dtype == PSC_BF16 ? 0 : 1];
+        int tgrid = (int)std::max(1L, std::min<long>(titems, resident));
         if (dtype == PSC_BF16)
-            k_step_tma<uint16_t><<<tgrid, 256, TmaShape<uint16_t>::SMEM, cs>>>(
-                (uint16_t*)d_logits, row_stride, B, V, d_bitmask_out, st->d.best, h->d, st->d);
+            k_step_tma<uint16_t><<<tgrid, TMA_WARPS * 32, TmaShape<uint16_t>::SMEM, cs>>>(
+                (uint16_t*)d_logits, row_stride, B, V, d_bitmask_out, st->d.best, h->d, st->d, have_mid);
         else
-            k_step_tma<uint32_t><<<tgrid, 256, TmaShape<uint32_t>::SMEM, cs>>>(
-                (uint32_t*)d_logits, row_stride, B, V, d_bitmask_out, st->d.best, h->d, st->d);
+            k_step_tma<uint32_t><<<tgrid, TMA_WARPS * 32, TmaShape<uint32_t>::SMEM, cs>>>(
+                (uint32_t*)d_logits, row_stride, B, V, d_bitmask_out, st->d.best, h->d, st->d, have_mid);
         s = launch_check("k_step_tma");
     } else {
         if (dtype == PSC_BF16)
@@ -1246,7 +1550,7 @@ int host_feed(const psc::Tables& T, uint16_t* st, int& depth, int cap, int cls) 
 }  // namespace
 
 namespace {
-// Compact int16 lexer/parser tables for k_advance_smem, or an empty blob when
+// Compact int16 lexer/parser tables for k_advance_warp, or an empty blob when
 // the grammar is too large for shared memory (k_advance then reads global memory).
 std::vector<uint8_t> build_advance_blob(const psc::Tables& t, DevTables& d) {
     std::vector<uint8_t> blob;
@@ -1373,13 +1677,13 @@ psc_status upload_tables(std::unique_ptr<psc_handle>& h, bool global_tables) {
         int optin = 0;
         cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, h->device);
         cudaFuncAttributes fa{};
-        cudaFuncGetAttributes(&fa, k_advance_smem);
+        cudaFuncGetAttributes(&fa, k_advance_warp);
         optin -= (int)fa.sharedSizeBytes;   // the limit covers dynamic memory only
-        if (optin < d.adv_bytes) {
+        if (optin < adv_smem(d)) {
             d.adv_bytes = 0;   // cannot stage: fall back to global tables
-        } else if ((s = cuda_check(cudaFuncSetAttribute(k_advance_smem, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        } else if ((s = cuda_check(cudaFuncSetAttribute(k_advance_warp, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                         optin),
-                                   "cudaFuncSetAttribute(k_advance_smem)")) != PSC_OK) {
+                                   "cudaFuncSetAttribute(k_advance_warp)")) != PSC_OK) {
             for (int i = 0; i < h->n_blocks; i++) cudaFree(h->blocks[i]);
             return s;
         }
@@ -1390,10 +1694,17 @@ psc_status upload_tables(std::unique_ptr<psc_handle>& h, bool global_tables) {
                         "cudaFuncSetAttribute(k_step_tma)")) != PSC_OK ||
         (s = cuda_check(cudaFuncSetAttribute(k_step_tma<uint32_t>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              TmaShape<uint32_t>::SMEM),
-                        "cudaFuncSetAttribute(k_step_tma)")) != PSC_OK) {
+                        "cudaFuncSetAttribute(k_step_tma)")) != PSC_OK ||
+        (s = cuda_check(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&h->tma_ctas[0], k_step_tma<uint16_t>,
+                                                                      TMA_WARPS * 32, TmaShape<uint16_t>::SMEM),
+                        "cudaOccupancyMaxActiveBlocksPerMultiprocessor(k_step_tma)")) != PSC_OK ||
+        (s = cuda_check(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&h->tma_ctas[1], k_step_tma<uint32_t>,
+                                                                      TMA_WARPS * 32, TmaShape<uint32_t>::SMEM),
+                        "cudaOccupancyMaxActiveBlocksPerMultiprocessor(k_step_tma)")) != PSC_OK) {
         for (int i = 0; i < h->n_blocks; i++) cudaFree(h->blocks[i]);
         return s;
     }
+    for (int k = 0; k < 2; k++) h->tma_ctas[k] = std::max(1, h->tma_ctas[k]);
     d.q0 = t.q0;
     d.nq = t.nq;
     d.n_lr = t.n_lr;
@@ -1548,14 +1859,7 @@ psc_status psc_advance(const psc_handle* h, psc_states* st, const int32_t* d_tok
     if (s != PSC_OK) return s;
     if (!st || st->h != h || B != st->d.B || !d_tokens) return fail_with(PSC_ERR_ARG, "psc_advance: bad arguments");
     int use_mid = st->mid_gen == st->gen ? 1 : 0;
-    if (h->d.adv_bytes > 0)
-        k_advance_smem<<<(B + 63) / 64, 64, h->d.adv_bytes, (cudaStream_t)stream>>>(h->d, st->d, d_tokens, B,
-                                                                                  use_mid, d_row_status, 0, nullptr);
-    else
-        k_advance<<<(B + 127) / 128, 128, 0, (cudaStream_t)stream>>>(h->d, st->d, d_tokens, B, use_mid, d_row_status,
-                                                                      0, nullptr);
-    st->gen++;
-    return launch_check("k_advance");
+    return launch_advance(h, st, d_tokens, use_mid, d_row_status, nullptr, (cudaStream_t)stream);
 }
 
 psc_status psc_fill_mask(const psc_handle* h, const psc_states* st, int32_t B, uint32_t* d_bitmask, void* stream) {
@@ -1640,13 +1944,7 @@ psc_status psc_decode_step(const psc_handle* h, psc_states* st, int32_t B, void*
         return fail_with(PSC_ERR_ARG, "psc_decode_step: bad arguments");
     cudaStream_t cs = (cudaStream_t)stream;
     if ((s = launch_fused(h, st, d_logits, dtype, row_stride, V, d_bitmask_out, cs)) != PSC_OK) return s;
-    if (h->d.adv_bytes > 0)
-        k_advance_smem<<<(B + 63) / 64, 64, h->d.adv_bytes, cs>>>(h->d, st->d, nullptr, B, 1, d_row_status, 1,
-                                                                   d_tokens);
-    else
-        k_advance<<<(B + 127) / 128, 128, 0, cs>>>(h->d, st->d, nullptr, B, 1, d_row_status, 1, d_tokens);
-    st->gen++;
-    return launch_check("k_advance");
+    return launch_advance(h, st, nullptr, 1, d_row_status, d_tokens, cs);
 }
 
 psc_status psc_states_download(const psc_states* st, int32_t* h_q, int32_t* h_depth, uint16_t* h_stack,
