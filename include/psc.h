@@ -205,16 +205,32 @@ psc_status psc_fill_apply_argmax(const psc_handle* h, const psc_states* st, int3
                                  int32_t* d_tokens, void* stream);
 
 /* One whole decoding step on the device (Algorithm 2 steps 1-4 plus masking and
- * greedy sampling), in two kernels: the masking pass classifies every row's
- * stack inside the kernel, applies the mask to the logits in place, writes
- * the optional bitmask copy and picks the greedy token per row; the advance
- * kernel then feeds that token to the row's lexer and parser.
+ * greedy sampling), in two kernels: the masking pass applies every row's mask
+ * (step 4) to the logits in place, writes the optional bitmask copy and picks
+ * the greedy token per row; the advance kernel then feeds that token to the
+ * row's lexer and parser (steps 1-2) and classifies the new configuration
+ * (step 3), so the next step's masking pass reads the mask ids directly.  The
+ * masking pass classifies rows itself when the mask ids are not current (after
+ * psc_state_init or psc_state_reset).
  *   d_tokens      : device int32 [B]; receives the chosen tokens (-1 = nothing allowed)
  *   d_row_status  : optional device int32 [B] statuses after the step
- * Other arguments as for psc_fill_apply_argmax. */
+ * Other arguments as for psc_fill_apply_argmax.  Equivalent to
+ * psc_decode_step_mask followed by psc_decode_step_advance. */
 psc_status psc_decode_step(const psc_handle* h, psc_states* st, int32_t B, void* d_logits, psc_dtype dtype,
                            int64_t row_stride, int32_t V, uint32_t* d_bitmask_out, int32_t* d_tokens,
                            int32_t* d_row_status, void* stream);
+
+/* The two halves of psc_decode_step, for callers that interleave work (or
+ * timing) between them.  psc_decode_step_mask runs the masking pass and keeps
+ * each row's greedy choice in the states object; psc_decode_step_advance
+ * consumes those choices: writes them to d_tokens, advances every row and
+ * classifies the new configurations.  Calling psc_decode_step_advance without
+ * a preceding psc_decode_step_mask on the same states object finds no choices
+ * (every token -1, rows unchanged).  Arguments as for psc_decode_step. */
+psc_status psc_decode_step_mask(const psc_handle* h, psc_states* st, int32_t B, void* d_logits, psc_dtype dtype,
+                                int64_t row_stride, int32_t V, uint32_t* d_bitmask_out, void* stream);
+psc_status psc_decode_step_advance(const psc_handle* h, psc_states* st, int32_t B, int32_t* d_tokens,
+                                   int32_t* d_row_status, void* stream);
 
 /* Copies the batch to host memory and synchronises the stream (tests and
  * debugging).  Any output pointer may be NULL.

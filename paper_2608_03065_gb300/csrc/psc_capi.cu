@@ -1947,6 +1947,27 @@ psc_status psc_decode_step(const psc_handle* h, psc_states* st, int32_t B, void*
     return launch_advance(h, st, nullptr, 1, d_row_status, d_tokens, cs);
 }
 
+psc_status psc_decode_step_mask(const psc_handle* h, psc_states* st, int32_t B, void* d_logits, psc_dtype dtype,
+                                int64_t row_stride, int32_t V, uint32_t* d_bitmask_out, void* stream) {
+    psc_status s = check_device(h, "psc_decode_step_mask");
+    if (s != PSC_OK) return s;
+    if (!st || st->h != h || B != st->d.B || !d_logits || V != h->d.V || row_stride < V ||
+        (dtype != PSC_F32 && dtype != PSC_BF16))
+        return fail_with(PSC_ERR_ARG, "psc_decode_step_mask: bad arguments");
+    return launch_fused(h, st, d_logits, dtype, row_stride, V, d_bitmask_out, (cudaStream_t)stream);
+}
+
+psc_status psc_decode_step_advance(const psc_handle* h, psc_states* st, int32_t B, int32_t* d_tokens,
+                                   int32_t* d_row_status, void* stream) {
+    psc_status s = check_device(h, "psc_decode_step_advance");
+    if (s != PSC_OK) return s;
+    if (!st || st->h != h || B != st->d.B || !d_tokens)
+        return fail_with(PSC_ERR_ARG, "psc_decode_step_advance: bad arguments");
+    // the greedy keys were made for the mask ids the masking pass used (current
+    // unless rows changed since): the advance checks tokens against those
+    return launch_advance(h, st, nullptr, 1, d_row_status, d_tokens, (cudaStream_t)stream);
+}
+
 psc_status psc_states_download(const psc_states* st, int32_t* h_q, int32_t* h_depth, uint16_t* h_stack,
                                int32_t* h_status, void* stream) {
     if (!st) return fail_with(PSC_ERR_ARG, "psc_states_download: NULL states");

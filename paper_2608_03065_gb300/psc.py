@@ -26,7 +26,7 @@ EXPORTED = ["psc_compile", "psc_destroy", "psc_last_error", "psc_info", "psc_sta
             "psc_state_destroy", "psc_advance", "psc_fill_mask", "psc_apply_mask", "psc_fill_apply",
             "psc_argmax_masked", "psc_states_download", "psc_host_classify", "psc_host_mask_row",
             "psc_host_advance", "psc_fill_apply_noalloc", "psc_fill_apply_argmax", "psc_save", "psc_load",
-            "psc_decode_step"]
+            "psc_decode_step", "psc_decode_step_mask", "psc_decode_step_advance"]
 NOALLOC_MAX_ROWS = 16384
 
 
@@ -84,6 +84,8 @@ def load(path: str = LIB_PATH):
         "psc_fill_apply_argmax": (i32, [vp, vp, i32, vp, i32, i64, i32, vp, vp, vp]),
         "psc_save": (i32, [vp, ctypes.c_char_p]),
         "psc_decode_step": (i32, [vp, vp, i32, vp, i32, i64, i32, vp, vp, vp, vp]),
+        "psc_decode_step_mask": (i32, [vp, vp, i32, vp, i32, i64, i32, vp, vp]),
+        "psc_decode_step_advance": (i32, [vp, vp, i32, vp, vp, vp]),
         "psc_load": (i32, [ctypes.c_char_p, vp, vp]),
     }
     for name, (res, args) in sig.items():
@@ -329,6 +331,27 @@ def psc_decode_step(h: Handle, st: States, logits, tokens, bitmask_out=None, row
                                   _row_stride(logits), h.V, _ptr(bitmask_out, torch.int32, "bitmask_out"),
                                   _ptr(tokens, torch.int32, "tokens"), _ptr(row_status, torch.int32, "row_status"),
                                   _stream(stream)))
+
+
+def psc_decode_step_mask(h: Handle, st: States, logits, bitmask_out=None, stream=None):
+    """First half of psc_decode_step: masking pass, greedy choices kept in the states."""
+    import torch
+    if logits.shape[0] != st.B or logits.shape[1] < h.V:
+        raise ValueError("logits must be [B, >=V]")
+    if bitmask_out is not None and (bitmask_out.shape != (st.B, h.W) or not bitmask_out.is_contiguous()):
+        raise ValueError("bitmask_out must be a contiguous [B, W] tensor")
+    _check(load().psc_decode_step_mask(h.ptr, st.ptr, st.B, _ptr(logits, None, "logits"), _dtype_code(logits),
+                                       _row_stride(logits), h.V, _ptr(bitmask_out, torch.int32, "bitmask_out"),
+                                       _stream(stream)))
+
+
+def psc_decode_step_advance(h: Handle, st: States, tokens, row_status=None, stream=None):
+    """Second half of psc_decode_step: tokens out, rows advanced and classified."""
+    import torch
+    if tokens.numel() != st.B:
+        raise ValueError("tokens must hold B int32 values")
+    _check(load().psc_decode_step_advance(h.ptr, st.ptr, st.B, _ptr(tokens, torch.int32, "tokens"),
+                                          _ptr(row_status, torch.int32, "row_status"), _stream(stream)))
 
 
 def psc_states_download(st: States, stream=None) -> dict:

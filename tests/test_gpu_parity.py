@@ -245,7 +245,8 @@ def test_large_config_fused_sampled(psc, cfg_id):
 
 
 # ------------------------------------------------------------- decode loop
-@pytest.mark.parametrize("cfg_id,steps,mode", [(2, 6, "separate"), (3, 3, "fused"), (5, 4, "step")])
+@pytest.mark.parametrize("cfg_id,steps,mode", [(2, 6, "separate"), (3, 3, "fused"), (5, 4, "step"),
+                                                (4, 3, "split")])
 def test_decode_loop_advance(psc, cfg_id, steps, mode):
     _decode_loop(psc, case(psc, cfg_id), steps, mode)
 
@@ -257,6 +258,26 @@ def test_decode_loop_table_paths(psc, global_tables):
     c = Case(psc, 2, global_tables=global_tables)
     assert (c.h.info().advance_table_bytes > 0) == (not global_tables)
     _decode_loop(psc, c, 5, "step")
+
+
+def test_decode_step_advance_without_mask(psc):
+    """The advance half with no masking pass before it finds no greedy choices:
+    every token -1 and the rows unchanged."""
+    w = configs.load(2, batch=8)
+    h = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id)
+    st = psc.psc_state_init(h, w.B, 64)
+    tm = torch.from_numpy(w.token_matrix()).cuda()
+    for j in range(min(tm.shape[1], 6)):
+        psc.psc_advance(h, st, tm[:, j].contiguous())
+    before = psc.psc_states_download(st)
+    tok = torch.full((w.B,), 7, dtype=torch.int32, device="cuda")
+    stat = torch.empty(w.B, dtype=torch.int32, device="cuda")
+    psc.psc_decode_step_advance(h, st, tok, stat)
+    after = psc.psc_states_download(st)
+    assert (tok.cpu().numpy() == -1).all()
+    np.testing.assert_array_equal(stat.cpu().numpy(), before["status"])
+    for k in ("q", "depth", "stack", "status"):
+        np.testing.assert_array_equal(after[k], before[k])
 
 
 def _decode_loop(psc, c, steps, mode):
@@ -274,6 +295,9 @@ def _decode_loop(psc, c, steps, mode):
         bm = torch.zeros(B, c.h.W, dtype=torch.int32, device="cuda")
         if mode == "step":
             psc.psc_decode_step(c.h, c.st, x, tok, bm, stat)
+        elif mode == "split":
+            psc.psc_decode_step_mask(c.h, c.st, x, bm)
+            psc.psc_decode_step_advance(c.h, c.st, tok, stat)
         elif mode == "fused":
             psc.psc_fill_apply_argmax(c.h, c.st, x, tok, bm)
         else:
@@ -286,7 +310,7 @@ def _decode_loop(psc, c, steps, mode):
         allowed = bits_of(dev_mask, V)
         np.testing.assert_array_equal(tok.cpu().numpy(), cpu_greedy(logits, allowed))
         np.testing.assert_array_equal(raw_bits(x)[rows], reference_masked(logits[rows], allowed[rows]))
-        if mode != "step":
+        if mode not in ("step", "split"):
             psc.psc_advance(c.h, c.st, tok, stat)
         torch.cuda.synchronize()
         t = tok.cpu().numpy()
