@@ -33,6 +33,7 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 WORKLOAD = 5
+SEQ = 32          # decode steps per sequence of the workload
 METRIC = "masked decode steps/s and µs/step at batch×vocab; HBM GB/s vs GB300 peak"
 UNIT = "steps/s"
 PROFILE_FILE = os.path.join(ROOT, "profiles", "k_step_tma_c5_traffic.txt")
@@ -193,7 +194,9 @@ def config_block(w, n):
     return {"workload": f"config 5: C-like grammar, vocab {w.V}, batch {w.B}, bf16 logits ~N(0,2), "
                         "decode steps (mask+apply+greedy+advance)",
             "batch": w.B, "vocab": w.V, "logit_dtype": "bf16", "grammar": "synthetic C-like (150 rules)",
-            "parallelism": f"replicas x{n}", "l2": "inputs larger than L2 (512 MiB logits per step)"}
+            "parallelism": f"replicas x{n}", "l2": "inputs larger than L2 (512 MiB logits per step)",
+            "decode": f"sequences of {SEQ} greedy steps from the prefix states (restored from a device "
+                      "copy before each sequence, inside the timed region); fresh logits every step"}
 
 
 def traffic_from_profile(kernel_src_hash: str):
@@ -252,6 +255,10 @@ def main():
         psc.psc_advance(h, st, tm[:, j].contiguous())
     torch.cuda.synchronize()
 
+    # the workload's decode sequences: SEQ steps from the prefix states, which are
+    # restored from a device copy before every sequence (the copy is timed too)
+    snap = psc.psc_state_init(h, B, 256)
+    psc.psc_state_copy(snap, st)
     K, Wm = args.steps, args.warmup
     n_buf = K + Wm
     gen = torch.Generator(device=dev).manual_seed(1000 * WORKLOAD + 4 + rank)
@@ -274,6 +281,10 @@ def main():
         if timed is not None:
             ev[timed][2].record(stream)
 
+    def restore():
+        psc.psc_state_copy(st, snap, stream=stream)
+
+    restore()
     for i in range(Wm):
         step(i)
     torch.cuda.synchronize()
@@ -285,6 +296,8 @@ def main():
         torch.cuda.nvtx.range_push("psc_steps")
         t_start.record(stream)
         for i in range(K):
+            if i % SEQ == 0:
+                restore()
             step(Wm + i, timed=i)
         t_end.record(stream)
         torch.cuda.synchronize()
@@ -316,6 +329,8 @@ def main():
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
     for i in range(K):
+        if i % SEQ == 0:
+            restore()
         dbuf.copy_(host[i % n_host], non_blocking=True)
         psc.psc_decode_step(h, st, dbuf, tok, bitmask, stat, stream=stream)
         tok_host.copy_(tok, non_blocking=True)

@@ -146,6 +146,14 @@ psc_status psc_state_reset(psc_states* st, const int32_t* d_rows, int32_t n, voi
 
 void psc_state_destroy(psc_states* st);
 
+/* Copies every row of src into dst: lexer states, depths, statuses, stacks,
+ * mask ids and pending greedy choices (device-to-device, enqueued on stream).
+ * Both objects must belong to the same handle and have the same B and cap
+ * (else PSC_ERR_ARG).  The paper has no counterpart: it serves forking a batch
+ * (beam search, speculative branches) and restoring a saved one, e.g. to
+ * decode again from the same prefixes. */
+psc_status psc_state_copy(psc_states* dst, const psc_states* src, void* stream);
+
 /* Algorithm 2, steps 1-2, done incrementally on the device: for each row b with
  * d_tokens[b] >= 0, first checks the token against the row's current mask; a
  * token outside it sets PSC_ROW_REJECTED; the end-of-sequence token sets

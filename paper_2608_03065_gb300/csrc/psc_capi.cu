@@ -230,10 +230,13 @@ __device__ __forceinline__ void apply_chunk(T* row, int col0, uint32_t word, int
         int wsrc = (c * E) >> 5;
         int sh = (c * E) & 31;
         uint32_t bits = (__shfl_sync(FULL, word, wsrc) >> sh) & FULLBITS;
+        // a 32-byte sector (this lane's 16 bytes and its neighbour's) is written whole or not
+        // at all, so the L2 never holds a partly written sector (read-modify-write on eviction)
+        bool keep = (bits & __shfl_xor_sync(FULL, bits, 1)) == FULLBITS;
         T* p = row + col0 + c * E;
         if (bits == 0) {
             st_cs_v4(p, ninf);
-        } else if (bits != FULLBITS) {
+        } else if (!keep) {
             uint4 v = *reinterpret_cast<const uint4*>(p);
             uint32_t w[4] = {v.x, v.y, v.z, v.w};
             if (sizeof(T) == 2) {
@@ -661,7 +664,8 @@ __device__ __forceinline__ void load_mask_chunk_bf16(const uint16_t* src, uint32
 }
 
 // Folds a masked chunk into the lane's best piece with packed bf16x2 maxima (NaN
-// never wins: the maximum returns the other operand) and writes it to the row.
+// never wins: the maximum returns the other operand) and writes it to the row
+// (32-byte sectors with every token allowed are left as they are).
 // Every lane runs the same instructions for every piece; only a piece whose
 // allowed values are all -inf or NaN, met before any other allowed value, takes
 // a short scalar path.
@@ -692,9 +696,11 @@ __device__ __forceinline__ void fold_store_chunk_bf16(uint16_t* row, int col0, i
         bp.x.y = upd ? x1 : bp.x.y;
         bp.x.z = upd ? x2 : bp.x.z;
         bp.x.w = upd ? x3 : bp.x.w;
-        // every piece is written, also one with every position allowed: a partly written
-        // 32-byte sector costs a read-modify-write when the L2 evicts it
-        st_cs_v4(row + pc, r.x[k]);
+        // a 32-byte sector (this lane's piece and its neighbour's) is written whole or not
+        // at all: a partly written sector costs a read-modify-write when the L2 evicts it.
+        // Only sectors whose 16 tokens are all allowed stay as they are.
+        uint32_t pair = bk & __shfl_xor_sync(FULL, bk, 1);
+        if (pair != 0xFFu) st_cs_v4(row + pc, r.x[k]);
     }
 }
 
@@ -883,7 +889,8 @@ struct StackView {
 
 // Feed one lexeme class to the parser: resolve it to a terminal with the
 // current top (contextual lexing), reduce until it is shifted.  Returns a row status.
-__device__ int feed_class_win(const uint8_t* sm, const DevTables& T, StackView& sv, int& depth, int& top, int cap,
+__device__ __forceinline__ int feed_class_win(const uint8_t* sm, const DevTables& T, StackView& sv, int& depth,
+                                              int& top, int cap,
                               int cls) {
     const int16_t* resolve = reinterpret_cast<const int16_t*>(sm + T.o_resolve);
     const int16_t* action = reinterpret_cast<const int16_t*>(sm + T.o_action);
@@ -918,7 +925,7 @@ __device__ int feed_class_win(const uint8_t* sm, const DevTables& T, StackView& 
 // Classifier walk of a configuration (lexer state q, stack of the given depth
 // read through the view) by a full warp: lanes fetch 32 stack symbols at a time,
 // the walk broadcasts them with shuffles.  Every lane returns the mask id.
-__device__ int warp_walk(const DevTables& T, const StackView& sv, int q, int depth, int lane) {
+__device__ __forceinline__ int warp_walk(const DevTables& T, const StackView& sv, int q, int depth, int lane) {
     if (q < 0 || q >= T.nq || depth < 1) return 0;
     int s = __ldg(T.dfa_start + q);
     if (s < 0) return -s - 1;
@@ -938,7 +945,9 @@ __device__ int warp_walk(const DevTables& T, const StackView& sv, int q, int dep
 
 // Algorithm 2 steps 1-3 for one row per warp: consume the row's token (the
 // given one, or the greedy choice of the fused masking pass when from_keys),
-// then classify the new configuration into S.mid.
+// then classify the new configuration into S.mid.  Everything that needs only
+// global memory (the row's state, its mask word, the token's bytes, the stack
+// window) is loaded while the tables are still being staged.
 __global__ void __launch_bounds__(ADV_WARPS * 32) k_advance_warp(DevTables T, DevStates S, const int32_t* tokens,
                                                                  int B, int use_mid, int32_t* status_out,
                                                                  int from_keys, int32_t* tokens_out) {
@@ -955,92 +964,93 @@ __global__ void __launch_bounds__(ADV_WARPS * 32) k_advance_warp(DevTables T, De
                      ::"r"(smem_addr(sm)), "l"(T.adv), "r"(T.adv_bytes), "r"(bar_a)
                      : "memory");
     }
-    __syncthreads();
-    bool staged = __all_sync(FULL, mbar_wait0(bar_a, 1 << 24));
     int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     int b = blockIdx.x * ADV_WARPS + warp;
+    bool active = b < B;   // warp-uniform
+    StackView sv{reinterpret_cast<uint16_t*>(sm + T.adv_bytes) + warp * ADV_WIN,
+                 S.stack + (size_t)(active ? b : 0) * S.cap, 0x40000000, 0x7FFFFFFF};
+    int tok = -1, status = ROW_OK, q = 0, depth = 0;
+    bool parse = false;
+    uint32_t mword = 0;
+    uint32_t tw[8] = {0, 0, 0, 0, 0, 0, 0, 0};   // the token's bytes (tokens up to 32 bytes)
+    int len = 0;
+    int64_t vlo = 0;
+    if (active) {
+        if (lane == 0) {
+            if (from_keys) {   // the greedy choice of the fused masking pass
+                unsigned long long k = S.best[b];
+                S.best[b] = 0ull;
+                tok = k ? (int32_t)(~(uint32_t)(k & 0xFFFFFFFFu)) : -1;
+                tokens_out[b] = tok;
+            } else {
+                tok = tokens[b];
+            }
+            status = S.status[b];
+        }
+        tok = __shfl_sync(FULL, tok, 0);
+        status = __shfl_sync(FULL, status, 0);
+        q = S.q[b];
+        depth = S.depth[b];
+        if (tok >= 0) {
+            if (status == ROW_DONE) {
+                status = tok == T.eos_id ? ROW_DONE : ROW_REJECTED;
+            } else if (status == ROW_OK) {
+                if (tok >= T.V) {
+                    status = ROW_REJECTED;
+                } else {
+                    int mid;
+                    if (use_mid) {
+                        mid = S.mid[b];
+                    } else {
+                        StackView g{sv.win, sv.st, 0x40000000, 0x7FFFFFFF};   // all of the stack in global memory
+                        mid = depth >= 1 && depth <= S.cap ? warp_walk(T, g, q, depth, lane) : 0;
+                    }
+                    // the token's mask bit; the row is only committed (q, depth) when it is set
+                    mword = __ldg(T.masks + (size_t)mid * T.Wp + (tok >> 5));
+                    if (tok == T.eos_id) status = ((mword >> (tok & 31)) & 1) ? ROW_DONE : ROW_REJECTED;
+                    else if (depth < 1 || depth > S.cap) status = ROW_REJECTED;
+                    else parse = true;
+                }
+            }
+        }
+        if (parse) {
+            // the window of the stack top and the token's bytes, loaded together
+            sv.base = depth > ADV_KEEP ? depth - ADV_KEEP : 0;
+            for (int i = lane; i < depth - sv.base; i += 32) sv.win[i] = sv.st[sv.base + i];
+            if (lane == 0) {
+                vlo = T.vocab_off[tok];
+                len = (int)(T.vocab_off[tok + 1] - vlo);
+#pragma unroll
+                for (int i = 0; i < 32; i++)
+                    if (i < len) tw[i >> 2] |= (uint32_t)T.vocab[vlo + i] << (8 * (i & 3));
+            }
+        }
+    }
+    __syncthreads();
+    bool staged = __all_sync(FULL, mbar_wait0(bar_a, 1 << 24));
     if (!staged) {
         // the copy did not land: give the rows a LIMIT status, wait (bounded) for the copy, return
         if (threadIdx.x == 0) atomicAdd(&g_pipeline_timeouts, 1);
-        if (b < B && lane == 0) {
-            if (S.status[b] == ROW_OK) S.status[b] = ROW_LIMIT;
-            if (from_keys) {
-                tokens_out[b] = -1;
-                S.best[b] = 0ull;
-            }
-            if (status_out) status_out[b] = S.status[b];
+        if (active && lane == 0) {
+            if (status == ROW_OK) status = ROW_LIMIT;
+            S.status[b] = status;
+            if (status_out) status_out[b] = status;
             S.mid[b] = 0;
         }
         mbar_wait0(bar_a, 1 << 24);
         return;
     }
-    if (b >= B) return;
-    const uint8_t* bc = sm + T.o_bc;
-    const int16_t* trans = reinterpret_cast<const int16_t*>(sm + T.o_trans);
-    const int16_t* acc = reinterpret_cast<const int16_t*>(sm + T.o_accept);
-    const uint8_t* ign = sm + T.o_ign;
-    StackView sv{reinterpret_cast<uint16_t*>(sm + T.adv_bytes) + warp * ADV_WIN, S.stack + (size_t)b * S.cap, 0,
-                 0x7FFFFFFF};
-    int tok = 0, status = ROW_OK;
-    if (lane == 0) {
-        if (from_keys) {   // the greedy choice of the fused masking pass
-            unsigned long long k = S.best[b];
-            S.best[b] = 0ull;
-            tok = k ? (int32_t)(~(uint32_t)(k & 0xFFFFFFFFu)) : -1;
-            tokens_out[b] = tok;
-        } else {
-            tok = tokens[b];
-        }
-        status = S.status[b];
-    }
-    tok = __shfl_sync(FULL, tok, 0);
-    status = __shfl_sync(FULL, status, 0);
-    int q = S.q[b], depth = S.depth[b];
-    bool parse = false;
-    uint32_t mword = 0;
-    if (tok >= 0) {
-        if (status == ROW_DONE) {
-            status = tok == T.eos_id ? ROW_DONE : ROW_REJECTED;
-        } else if (status == ROW_OK) {
-            if (tok >= T.V) {
-                status = ROW_REJECTED;
-            } else {
-                int mid;
-                if (use_mid) {
-                    mid = S.mid[b];
-                } else {
-                    StackView g{nullptr, sv.st, 0x40000000, 0x7FFFFFFF};   // all of the stack in global memory
-                    mid = depth >= 1 && depth <= S.cap ? warp_walk(T, g, q, depth, lane) : 0;
-                }
-                // the token's mask bit; the row is only committed (q, depth) when it is set
-                mword = __ldg(T.masks + (size_t)mid * T.Wp + (tok >> 5));
-                if (tok == T.eos_id) status = ((mword >> (tok & 31)) & 1) ? ROW_DONE : ROW_REJECTED;
-                else parse = true;
-            }
-        }
-    }
+    if (!active) return;
     if (parse) {
-        if (depth < 1 || depth > S.cap) {
-            parse = false;
-            status = ROW_REJECTED;
-        }
-    }
-    if (parse) {
-        sv.base = depth > ADV_KEEP ? depth - ADV_KEEP : 0;
-        for (int i = lane; i < depth - sv.base; i += 32) sv.win[i] = sv.st[sv.base + i];
-        __syncwarp();
+        const uint8_t* bc = sm + T.o_bc;
+        const int16_t* trans = reinterpret_cast<const int16_t*>(sm + T.o_trans);
+        const int16_t* acc = reinterpret_cast<const int16_t*>(sm + T.o_accept);
+        const uint8_t* ign = sm + T.o_ign;
         int nq = q, nd = depth;
         if (lane == 0) {
             int top = sv.win[depth - 1 - sv.base];
-            int64_t lo = T.vocab_off[tok], hi = T.vocab_off[tok + 1];
-            int len = (int)(hi - lo);
-            // the token's bytes, fetched together (tokens up to 32 bytes)
-            uint32_t tw[8] = {0, 0, 0, 0, 0, 0, 0, 0};
-#pragma unroll
-            for (int i = 0; i < 32; i++)
-                if (i < len) tw[i >> 2] |= (uint32_t)T.vocab[lo + i] << (8 * (i & 3));
             for (int i = 0; i < len && status == ROW_OK; i++) {
-                int byte = i < 32 ? (int)((tw[i >> 2] >> (8 * (i & 3))) & 0xFFu) : (int)T.vocab[lo + i];
+                int byte = i < 32 ? (int)((tw[i >> 2] >> (8 * (i & 3))) & 0xFFu) : (int)T.vocab[vlo + i];
                 int c = bc[byte];
                 int nx = trans[nq * T.nbc + c];
                 if (nx >= 0) {
@@ -1080,16 +1090,12 @@ __global__ void __launch_bounds__(ADV_WARPS * 32) k_advance_warp(DevTables T, De
         if (tok >= 0) S.status[b] = status;
         if (status_out) status_out[b] = status;
     }
-    // the next masking pass's mask id
+    // the next masking pass's mask id (without a parse the window holds nothing:
+    // sv.base still points past any stack index, so the walk reads global memory)
     int mid;
-    if (status == ROW_DONE) {
-        mid = 1;
-    } else if (status != ROW_OK) {
-        mid = 0;
-    } else {
-        if (!parse) sv.base = 0x40000000;   // window not loaded: read the stack from global memory
-        mid = depth >= 1 && depth <= S.cap ? warp_walk(T, sv, q, depth, lane) : 0;
-    }
+    if (status == ROW_DONE) mid = 1;
+    else if (status != ROW_OK) mid = 0;
+    else mid = depth >= 1 && depth <= S.cap ? warp_walk(T, sv, q, depth, lane) : 0;
     if (lane == 0) S.mid[b] = mid;
 }
 
@@ -1829,6 +1835,36 @@ psc_status psc_state_init(const psc_handle* h, int32_t B, int32_t cap, void* str
         return s;
     }
     *out = st.release();
+    return PSC_OK;
+}
+
+psc_status psc_state_copy(psc_states* dst, const psc_states* src, void* stream) {
+    if (!dst || !src || dst->h != src->h || dst->d.B != src->d.B || dst->d.cap != src->d.cap)
+        return fail_with(PSC_ERR_ARG, "psc_state_copy: states of different handles or shapes");
+    if (dst == src) return PSC_OK;
+    int dev = -1;
+    cudaGetDevice(&dev);
+    if (dev != dst->device) return fail_with(PSC_ERR_ARG, "psc_state_copy: current device differs from the states'");
+    cudaStream_t cs = (cudaStream_t)stream;
+    const DevStates& a = src->d;
+    DevStates& b = dst->d;
+    size_t B = (size_t)a.B;
+    psc_status s;
+    // one copy per array (no batched-copy call)
+    if ((s = cuda_check(cudaMemcpyAsync(b.q, a.q, B * 4, cudaMemcpyDeviceToDevice, cs), "psc_state_copy")) != PSC_OK ||
+        (s = cuda_check(cudaMemcpyAsync(b.depth, a.depth, B * 4, cudaMemcpyDeviceToDevice, cs), "psc_state_copy")) !=
+            PSC_OK ||
+        (s = cuda_check(cudaMemcpyAsync(b.status, a.status, B * 4, cudaMemcpyDeviceToDevice, cs), "psc_state_copy")) !=
+            PSC_OK ||
+        (s = cuda_check(cudaMemcpyAsync(b.stack, a.stack, B * (size_t)a.cap * 2, cudaMemcpyDeviceToDevice, cs),
+                        "psc_state_copy")) != PSC_OK ||
+        (s = cuda_check(cudaMemcpyAsync(b.mid, a.mid, B * 4, cudaMemcpyDeviceToDevice, cs), "psc_state_copy")) !=
+            PSC_OK ||
+        (s = cuda_check(cudaMemcpyAsync(b.best, a.best, B * 8, cudaMemcpyDeviceToDevice, cs), "psc_state_copy")) !=
+            PSC_OK)
+        return s;
+    dst->gen++;
+    dst->mid_gen = src->mid_gen == src->gen ? dst->gen : 0;   // the mask ids are as current as src's
     return PSC_OK;
 }
 

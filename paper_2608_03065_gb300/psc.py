@@ -26,7 +26,7 @@ EXPORTED = ["psc_compile", "psc_destroy", "psc_last_error", "psc_info", "psc_sta
             "psc_state_destroy", "psc_advance", "psc_fill_mask", "psc_apply_mask", "psc_fill_apply",
             "psc_argmax_masked", "psc_states_download", "psc_host_classify", "psc_host_mask_row",
             "psc_host_advance", "psc_fill_apply_noalloc", "psc_fill_apply_argmax", "psc_save", "psc_load",
-            "psc_decode_step", "psc_decode_step_mask", "psc_decode_step_advance"]
+            "psc_decode_step", "psc_decode_step_mask", "psc_decode_step_advance", "psc_state_copy"]
 NOALLOC_MAX_ROWS = 16384
 
 
@@ -85,6 +85,7 @@ def load(path: str = LIB_PATH):
         "psc_save": (i32, [vp, ctypes.c_char_p]),
         "psc_decode_step": (i32, [vp, vp, i32, vp, i32, i64, i32, vp, vp, vp, vp]),
         "psc_decode_step_mask": (i32, [vp, vp, i32, vp, i32, i64, i32, vp, vp]),
+        "psc_state_copy": (i32, [vp, vp, vp]),
         "psc_decode_step_advance": (i32, [vp, vp, i32, vp, vp, vp]),
         "psc_load": (i32, [ctypes.c_char_p, vp, vp]),
     }
@@ -259,6 +260,11 @@ def psc_state_reset(st: States, rows=None, stream=None):
     import torch
     n = st.B if rows is None else rows.numel()
     _check(load().psc_state_reset(st.ptr, _ptr(rows, torch.int32, "rows"), n, _stream(stream)))
+
+
+def psc_state_copy(dst: States, src: States, stream=None):
+    """dst's rows := src's rows (same handle, B and cap), on the device."""
+    _check(load().psc_state_copy(dst.ptr, src.ptr, _stream(stream)))
 
 
 def psc_advance(h: Handle, st: States, tokens, row_status=None, stream=None):

@@ -280,6 +280,38 @@ def test_decode_step_advance_without_mask(psc):
         np.testing.assert_array_equal(after[k], before[k])
 
 
+def test_state_copy_forks_a_batch(psc):
+    """A copied batch decodes exactly like its source (same tokens, statuses and
+    states after several steps); copies between mismatched batches are refused."""
+    w = configs.load(2)
+    h = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id)
+    a = psc.psc_state_init(h, w.B, 128)
+    tm = torch.from_numpy(w.token_matrix()).cuda()
+    for j in range(tm.shape[1]):
+        psc.psc_advance(h, a, tm[:, j].contiguous())
+    b = psc.psc_state_init(h, w.B, 128)
+    psc.psc_state_copy(b, a)
+    ta = torch.empty(w.B, dtype=torch.int32, device="cuda")
+    tb = torch.empty_like(ta)
+    for step in range(4):
+        logits = w.logits(50 + step)
+        xa, xb = logits.cuda(), logits.cuda()
+        psc.psc_decode_step(h, a, xa, ta)
+        psc.psc_decode_step(h, b, xb, tb)
+        torch.cuda.synchronize()
+        np.testing.assert_array_equal(ta.cpu().numpy(), tb.cpu().numpy())
+        np.testing.assert_array_equal(raw_bits(xa), raw_bits(xb))
+    da, db = psc.psc_states_download(a), psc.psc_states_download(b)
+    for k in ("q", "depth", "status"):
+        np.testing.assert_array_equal(da[k], db[k])
+    for r in range(w.B):
+        np.testing.assert_array_equal(da["stack"][r, :da["depth"][r]], db["stack"][r, :db["depth"][r]])
+    small = psc.psc_state_init(h, w.B, 64)
+    with pytest.raises(psc.PscError) as e:
+        psc.psc_state_copy(small, a)
+    assert e.value.code == 1
+
+
 def _decode_loop(psc, c, steps, mode):
     """fill_apply -> argmax -> advance for several steps; after every step the
     device masks equal the oracle's after advancing it by the same tokens
