@@ -218,6 +218,121 @@ def traffic_from_profile(kernel_src_hash: str):
         return None
 
 
+# ------------------------------------------------------------- teacher mode
+def run_teacher(args):
+    """RQ1: whole sentences of configs 2-4 are teacher-forced through the device
+    path (psc_fill_mask, then psc_advance); the pass rate on them must be 1, and
+    sentences with one random token spliced in are mostly stopped.  RQ2: one
+    decoding step at batch 1 on the config-5 tables (mask + advance on the
+    device), beside the same step through the library's host functions (the
+    classifier walk, the mask-row copy and the parser step on the CPU)."""
+    import numpy as np
+    import torch
+    from paper_2608_03065_gb300 import build, psc
+    from workloads import configs, teacher
+    build.build()
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    out = {"metric": "teacher-forced pass rate; batch-1 step latency", "mode": "teacher", "rq1": {}, "rq2": {}}
+
+    def first_rejection(h, w, seqs):
+        B = len(seqs)
+        T = max(len(q) for q in seqs) + 1
+        tokm = np.full((B, T), -1, dtype=np.int32)
+        for b, q in enumerate(seqs):
+            tokm[b, :len(q)] = q
+            tokm[b, len(q)] = w.eos_id
+        st = psc.psc_state_init(h, B, 256)
+        bm = torch.empty(B, h.W, dtype=torch.int32, device=dev)
+        first = np.full(B, -1, dtype=np.int64)
+        for j in range(T):
+            psc.psc_fill_mask(h, st, bm)
+            m = bm.cpu().numpy().view(np.uint32)
+            col = tokm[:, j]
+            for b in np.nonzero((col >= 0) & (first < 0))[0]:
+                v = int(col[b])
+                if not ((m[b, v >> 5] >> (v & 31)) & 1):
+                    first[b] = j
+            psc.psc_advance(h, st, torch.from_numpy(np.where(first < 0, col, -1).astype(np.int32)).to(dev))
+        torch.cuda.synchronize()
+        return first, int(sum(len(q) + 1 for q in seqs))
+
+    for cfg in (2, 3, 4):
+        w = configs.load(cfg, batch=1)
+        ts = teacher.teacher_set(w, 64)
+        h = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id)
+        t0 = time.time()
+        pos, ntok = first_rejection(h, w, ts.positives)
+        neg, _ = first_rejection(h, w, ts.negatives)
+        secs = time.time() - t0
+        out["rq1"][w.spec.name] = {
+            "sentences": len(ts.positives), "tokens": ntok,
+            "positive_pass_rate": float((pos < 0).mean()),
+            "negative_stopped_rate": float((neg >= 0).mean()),
+            "stopped_before_splice": int(sum(1 for r, k in zip(neg, ts.inserted_at) if 0 <= r < k)),
+            "wall_s": round(secs, 2)}
+
+    # RQ2 on config 5's tables, one row
+    w = configs.load(5, batch=1)
+    h = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id)
+    ids = w.prefix_ids[0]
+    n = min(len(ids), 200)
+    st = psc.psc_state_init(h, 1, 256)
+    bm = torch.empty(1, h.W, dtype=torch.int32, device=dev)
+    toks = [torch.tensor([v], dtype=torch.int32, device=dev) for v in ids[:n]]
+    stream = torch.cuda.current_stream()
+    for i in range(5):
+        psc.psc_fill_mask(h, st, bm, stream=stream)
+    torch.cuda.synchronize()
+    st = psc.psc_state_init(h, 1, 256)
+    evs = []
+    for i in range(n):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        psc.psc_fill_mask(h, st, bm, stream=stream)
+        psc.psc_advance(h, st, toks[i], stream=stream)
+        b.record(stream)
+        evs.append((a, b))
+    torch.cuda.synchronize()
+    gpu_us = sorted(a.elapsed_time(b) * 1000.0 for a, b in evs)
+    logits = [(torch.randn(1, w.V, device=dev) * w.spec.sigma).to(torch.bfloat16) for _ in range(8)]
+    tok1 = torch.empty(1, dtype=torch.int32, device=dev)
+    st2 = psc.psc_state_init(h, 1, 256)
+    for v in ids[:20]:
+        psc.psc_advance(h, st2, torch.tensor([v], dtype=torch.int32, device=dev))
+    evs = []
+    for i in range(64):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        psc.psc_decode_step(h, st2, logits[i % 8], tok1, stream=stream)
+        b.record(stream)
+        evs.append((a, b))
+    torch.cuda.synchronize()
+    dec_us = sorted(a.elapsed_time(b) * 1000.0 for a, b in evs)
+    # host: the library's C functions called directly (ctypes call overhead included)
+    lib = psc.load()
+    hh = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id, host_only=True)
+    cap = 256
+    stack = np.zeros(cap, dtype=np.uint16)
+    row = np.zeros(hh.W, dtype=np.uint32)
+    q, depth, status = ctypes.c_int32(0), ctypes.c_int32(1), ctypes.c_int32(0)
+    host_us = []
+    for i in range(n):
+        t0 = time.perf_counter()
+        mid = lib.psc_host_classify(hh.ptr, q.value, stack.ctypes.data, depth.value, status.value)
+        lib.psc_host_mask_row(hh.ptr, mid, row.ctypes.data)
+        lib.psc_host_advance(hh.ptr, ctypes.byref(q), stack.ctypes.data, ctypes.byref(depth), cap,
+                             ctypes.byref(status), int(ids[i]))
+        host_us.append((time.perf_counter() - t0) * 1e6)
+    host_us.sort()
+    med = lambda a: round(a[len(a) // 2], 2)
+    out["rq2"] = {"tables": w.spec.name, "steps": n,
+                  "gpu_fill_mask_plus_advance_b1_us": {"median": med(gpu_us), "p90": round(gpu_us[int(0.9 * len(gpu_us))], 2)},
+                  "gpu_decode_step_b1_us": {"median": med(dec_us), "vocab": w.V},
+                  "host_walk_mask_row_advance_us": {"median": med(host_us), "note": "one CPU thread, ctypes call overhead included"}}
+    print(json.dumps(out))
+
+
 # ------------------------------------------------------------------ main arm
 def main():
     ap = argparse.ArgumentParser()
@@ -226,9 +341,14 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="gb300")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--mode", default="decode", choices=["decode", "teacher"],
+                    help="decode: the benchmark line; teacher: teacher-forcing pass rates and "
+                         "batch-1 step latency (the paper's RQ1/RQ2 measurements on these workloads)")
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)
+    if args.mode == "teacher":
+        return run_teacher(args)
 
     import torch
     import torch.distributed as dist
@@ -343,6 +463,29 @@ def main():
         e2e_ms = float(tt.item())
     e2e_value = world * K / (e2e_ms / 1000.0)
 
+    # the plain mask paths on the same workload (prefix states, mask ids current),
+    # each the median of 50 launches with CUDA events, logits buffers in rotation
+    def median_us(fn, n=50):
+        times = []
+        for i in range(n):
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            fn(bufs[i % n_buf])
+            b.record(stream)
+            times.append((a, b))
+        torch.cuda.synchronize()
+        return statistics.median(a.elapsed_time(b) * 1000.0 for a, b in times)
+
+    restore()
+    no_tokens = torch.full((B,), -1, dtype=torch.int32, device=dev)
+    paths = {
+        "fill_apply_us": median_us(lambda x: psc.psc_fill_apply(h, st, x, bitmask, stream=stream)),
+        "fill_mask_us": median_us(lambda x: psc.psc_fill_mask(h, st, bitmask, stream=stream)),
+        "apply_mask_us": median_us(lambda x: psc.psc_apply_mask(x, bitmask, B, V, stream=stream)),
+        # a no-op advance still classifies every row: the classifier walk alone (+ launch)
+        "classify_us": median_us(lambda x: psc.psc_advance(h, st, no_tokens, stream=stream)),
+    }
+
     if rank != 0:
         if world > 1:
             dist.destroy_process_group()
@@ -380,6 +523,7 @@ def main():
         "gpu_launches": 2 * K,
         "clocks": clocks.summary(),
         "cpu_baseline": cpu,
+        "mask_paths": paths,
         "device_timeouts": h.info().device_timeouts,
         "tables": {"classifier_states": info.n_classifier_states, "masks": info.n_masks,
                    "classifier_bytes": info.classifier_bytes, "mask_bytes": info.mask_bytes,

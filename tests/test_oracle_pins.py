@@ -343,3 +343,20 @@ def test_sampled_sentences_are_sentences():
             assert o.allowed(cf, None)
             n_done += 1
         assert n_done > 0
+
+
+@pytest.mark.parametrize("cfg_id", [2, 4])
+def test_teacher_forced_sentences_never_masked(cfg_id):
+    """RQ1 invariant (Section 4): every token of a whole sentence of the grammar is
+    in the oracle's mask when teacher-forced, and the end of sequence is allowed
+    after it."""
+    from workloads import configs, teacher
+    w = configs.load(cfg_id, batch=1)
+    ts = teacher.teacher_set(w, 8)
+    o = Oracle(w.grammar_text)
+    for ids in ts.positives:
+        c = o.initial()
+        for v in ids:
+            assert o.allowed(c, w.vocab[v])
+            o.advance(c, w.vocab[v])
+        assert o.allowed(c, None)
