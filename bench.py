@@ -388,7 +388,10 @@ def main():
     tok = torch.empty(B, dtype=torch.int32, device=dev)
     stat = torch.empty(B, dtype=torch.int32, device=dev)
     stream = torch.cuda.current_stream()
-    ev = [tuple(torch.cuda.Event(enable_timing=True) for _ in range(3)) for _ in range(K)]
+    # per-launch events on the first sequence only: an event between two kernels stops the
+    # second from starting while the first finishes (programmatic dependent launch)
+    n_ev = min(K, SEQ)
+    ev = [tuple(torch.cuda.Event(enable_timing=True) for _ in range(3)) for _ in range(n_ev)]
 
     def step(i, timed=None):
         x = bufs[i]
@@ -418,7 +421,7 @@ def main():
         for i in range(K):
             if i % SEQ == 0:
                 restore()
-            step(Wm + i, timed=i)
+            step(Wm + i, timed=i if i < n_ev else None)
         t_end.record(stream)
         torch.cuda.synchronize()
         torch.cuda.nvtx.range_pop()

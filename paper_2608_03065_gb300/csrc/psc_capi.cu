@@ -59,6 +59,7 @@ struct DevTables {
     // compact lexer/parser tables for k_advance_warp (adv_bytes = 0: not built)
     const uint8_t* adv;
     int adv_bytes, o_bc, o_trans, o_accept, o_ign, o_resolve, o_action, o_go, o_rlen, o_rlhs, nbc;
+    int adv_packed;   // reduce entries of the compact ACTION hold (rule length << 10 | lhs) instead of the rule
 };
 
 struct DevStates {
@@ -853,6 +854,12 @@ __device__ __forceinline__ uint32_t smem_addr(const void* p) {
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
 
+// Programmatic dependent launch: the next kernel of the stream may be scheduled
+// now (it waits for this grid's results with grid_dep_wait); and the wait for
+// the previous kernel's results (returns at once when there is none to wait for).
+__device__ __forceinline__ void grid_dep_launch() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+__device__ __forceinline__ void grid_dep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 // Bounded wait on phase 0 of an mbarrier; returns false if it did not complete.
 __device__ __forceinline__ bool mbar_wait0(uint32_t bar, int limit) {
     for (int it = 0; it < limit; it++) {
@@ -909,11 +916,12 @@ __device__ __forceinline__ int feed_class_win(const uint8_t* sm, const DevTables
             return ROW_OK;
         }
         if (kind != psc::ACT_REDUCE) return ROW_REJECTED;
-        int k = rlen[val];
+        int k = T.adv_packed ? val >> 10 : rlen[val];
+        int lhs = T.adv_packed ? val & 1023 : rlhs[val];
         if (depth - k < 1) return ROW_REJECTED;
         depth -= k;
         int under = k ? sv.get(depth - 1) : top;
-        int g = go[under * T.n_nts + rlhs[val]];
+        int g = go[under * T.n_nts + lhs];
         if (g < 0) return ROW_REJECTED;
         if (depth >= cap) return ROW_OVERFLOW;
         sv.set(depth++, g);
@@ -964,6 +972,8 @@ __global__ void __launch_bounds__(ADV_WARPS * 32) k_advance_warp(DevTables T, De
                      ::"r"(smem_addr(sm)), "l"(T.adv), "r"(T.adv_bytes), "r"(bar_a)
                      : "memory");
     }
+    grid_dep_launch();
+    grid_dep_wait();   // the greedy keys and rows come from the previous kernel
     int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     int b = blockIdx.x * ADV_WARPS + warp;
     bool active = b < B;   // warp-uniform
@@ -1209,7 +1219,9 @@ __global__ void __launch_bounds__(TMA_WARPS * 32, 3) k_step_tma(T* logits, int64
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     }
+    grid_dep_launch();
     __syncthreads();
+    grid_dep_wait();   // mask ids, greedy keys and rows come from the previous kernel
     bool failed = false;
     if (warp == 0) {
         // ---------------------------------------------------------- producer
@@ -1463,6 +1475,24 @@ psc_status launch_apply(void* logits, psc_dtype dtype, int64_t row_stride, const
 
 // Masking + greedy choice with in-kernel classification; leaves each row's
 // key in st->d.best and its mask id in st->d.mid.
+// Launches a kernel that may start while the previous kernel of the stream finishes
+// (programmatic dependent launch): it waits for that kernel's results itself.
+template <typename... KArgs, typename... Args>
+psc_status launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t cs, const char* what,
+                      Args... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = cs;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cuda_check(cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...), what);
+}
+
 // Algorithm 2 steps 1-2 for every row (the token given, or the fused pass's greedy
 // choice when d_tokens_out is set), then step 3 for the new configurations: the
 // rows' mask ids are current afterwards.
@@ -1472,9 +1502,8 @@ psc_status launch_advance(const psc_handle* h, psc_states* st, const int32_t* d_
     int from_keys = d_tokens_out ? 1 : 0;
     psc_status s;
     if (h->d.adv_bytes > 0) {
-        k_advance_warp<<<(B + ADV_WARPS - 1) / ADV_WARPS, ADV_WARPS * 32, adv_smem(h->d), cs>>>(
-            h->d, st->d, d_tokens, B, use_mid, d_row_status, from_keys, d_tokens_out);
-        s = launch_check("k_advance_warp");
+        s = launch_pdl(k_advance_warp, dim3((B + ADV_WARPS - 1) / ADV_WARPS), dim3(ADV_WARPS * 32), adv_smem(h->d), cs,
+                       "k_advance_warp", h->d, st->d, d_tokens, B, use_mid, d_row_status, from_keys, d_tokens_out);
     } else {
         k_advance<<<(B + 127) / 128, 128, 0, cs>>>(h->d, st->d, d_tokens, B, use_mid, d_row_status, from_keys,
                                                     d_tokens_out);
@@ -1510,12 +1539,13 @@ psc_status launch_fused(const psc_handle* h, const psc_states* st, void* d_logit
         long resident = (long)sm_count(h->device) * h->tma_ctas[dtype == PSC_BF16 ? 0 : 1];
         int tgrid = (int)std::max(1L, std::min<long>(titems, resident));
         if (dtype == PSC_BF16)
-            k_step_tma<uint16_t><<<tgrid, TMA_WARPS * 32, TmaShape<uint16_t>::SMEM, cs>>>(
-                (uint16_t*)d_logits, row_stride, B, V, d_bitmask_out, st->d.best, h->d, st->d, have_mid);
+            s = launch_pdl(k_step_tma<uint16_t>, dim3(tgrid), dim3(TMA_WARPS * 32), TmaShape<uint16_t>::SMEM, cs,
+                           "k_step_tma", (uint16_t*)d_logits, row_stride, B, V, d_bitmask_out, st->d.best, h->d,
+                           st->d, have_mid);
         else
-            k_step_tma<uint32_t><<<tgrid, TMA_WARPS * 32, TmaShape<uint32_t>::SMEM, cs>>>(
-                (uint32_t*)d_logits, row_stride, B, V, d_bitmask_out, st->d.best, h->d, st->d, have_mid);
-        s = launch_check("k_step_tma");
+            s = launch_pdl(k_step_tma<uint32_t>, dim3(tgrid), dim3(TMA_WARPS * 32), TmaShape<uint32_t>::SMEM, cs,
+                           "k_step_tma", (uint32_t*)d_logits, row_stride, B, V, d_bitmask_out, st->d.best, h->d,
+                           st->d, have_mid);
     } else {
         if (dtype == PSC_BF16)
             k_apply_argmax<uint16_t, true><<<grid, 256, 0, cs>>>((uint16_t*)d_logits, row_stride, M, B, V, vec,
@@ -1607,9 +1637,16 @@ std::vector<uint8_t> build_advance_blob(const psc::Tables& t, DevTables& d) {
         blob[d.o_ign + c] = t.cls_ignored[c];
         for (int s = 0; s < t.n_lr; s++) put16(d.o_resolve, (size_t)c * t.n_lr + s, t.resolve[(size_t)c * t.n_lr + s]);
     }
+    // a reduce entry carries its rule's length and left-hand side when they fit in 14 bits
+    // (one dependent shared-memory read less per reduction)
+    int max_len = 0;
+    for (int L : t.rule_len) max_len = std::max(max_len, L);
+    d.adv_packed = (max_len < 16 && t.n_nts <= 1024) ? 1 : 0;
     for (size_t i = 0; i < t.action.size(); i++) {
         int32_t a = t.action[i];
-        put16(d.o_action, i, ((psc::act_val(a) & 0x3FFF) << 2) | psc::act_kind(a));
+        int kind = psc::act_kind(a), val = psc::act_val(a);
+        if (d.adv_packed && kind == psc::ACT_REDUCE) val = (t.rule_len[val] << 10) | t.rule_lhs[val];
+        put16(d.o_action, i, ((val & 0x3FFF) << 2) | kind);
     }
     for (size_t i = 0; i < t.go.size(); i++) put16(d.o_go, i, t.go[i]);
     for (int r = 0; r < n_rules; r++) {
