@@ -448,6 +448,48 @@ def test_nan_payloads_and_infinities_kept(psc):
         np.testing.assert_array_equal(got, want)
 
 
+@pytest.mark.parametrize("global_tables", [False, True])
+def test_deep_stacks_and_long_pushes(psc, global_tables):
+    """Balanced parentheses with tokens of up to 32 brackets: stacks grow to
+    thousands of entries, past the advance kernel's shared-memory window (192
+    entries copied in, 256 held), pushes of one token run beyond the window into
+    global memory, and closing tokens pop below it; masks and statuses after every
+    step equal the oracle's."""
+    g = 'start: s\ns: | s "(" s ")"\n'
+    toks = [b"(" * n for n in (1, 2, 7, 16, 31, 32)] + [b")" * n for n in (1, 3, 16, 32)] + [b"()", b")(", b""]
+    eos = len(toks) - 1
+    h = psc.psc_compile(g, toks, eos, global_tables=global_tables)
+    o = Oracle(g)
+    voc = Vocab.from_list(toks, eos)
+    B, cap = 6, 8192
+    st = psc.psc_state_init(h, B, cap)
+    ocs = [o.initial() for _ in range(B)]
+    rng = np.random.default_rng(77)
+    bm = torch.empty(B, h.W, dtype=torch.int32, device="cuda")
+    stat = torch.empty(B, dtype=torch.int32, device="cuda")
+    for step in range(70):
+        psc.psc_fill_mask(h, st, bm)
+        m = bm.cpu().numpy().view(np.uint32)
+        np.testing.assert_array_equal(m, o.masks(ocs, voc), err_msg=f"step {step}")
+        allowed = bits_of(m, len(toks))
+        tok = np.full(B, -1, dtype=np.int32)
+        for r in range(B):
+            opts = [t for t in np.nonzero(allowed[r])[0] if t != eos]
+            # rows 0-2 mostly open (deep stacks), rows 3-5 open and close at random
+            opens = [t for t in opts if toks[t].startswith(b"((")] if r < 3 else []
+            tok[r] = int(rng.choice(opens)) if opens and rng.random() < 0.8 else int(rng.choice(opts))
+        psc.psc_advance(h, st, torch.from_numpy(tok).cuda(), stat)
+        s_dev = stat.cpu().numpy()
+        for r in range(B):
+            ost = o.advance(ocs[r], toks[tok[r]])
+            want = {ST_OK: psc.ROW_OK, ST_DONE: psc.ROW_DONE, ST_ERROR: psc.ROW_REJECTED}[ost]
+            assert s_dev[r] == want, (step, r, s_dev[r], want)
+    d = psc.psc_states_download(st)
+    assert d["depth"].max() > 1024     # the deep rows went far past the window
+    for r in range(B):
+        assert d["depth"][r] == ocs[r].info()["depth"]
+
+
 def test_state_reset_rows(psc):
     c = case(psc, 2)
     rows = torch.tensor([0, 3, 5], dtype=torch.int32, device="cuda")
