@@ -459,6 +459,64 @@ void Builder::expand(int32_t n, const int32_t* g, int glen) {
 
 }  // namespace
 
+void set_mask_rows(Tables& t, const uint32_t* rows, int n, int W) {
+    int nch = (W + 31) / 32;
+    t.W = W;
+    t.n_masks = n;
+    t.nch = nch;
+    t.mask_rows.assign((size_t)n * nch, 0);
+    t.mask_chunks.clear();
+    // open addressing over chunk contents (64-bit FNV-1a of the 32 words)
+    size_t cap = 1024;
+    while (cap < (size_t)n * nch / 4 + 1024) cap <<= 1;
+    std::vector<int64_t> slot(cap, -1);
+    std::vector<uint64_t> slot_hash(cap, 0);
+    uint32_t chunk[32];
+    for (int m = 0; m < n; m++) {
+        const uint32_t* row = rows + (size_t)m * W;
+        for (int c = 0; c < nch; c++) {
+            int w0 = c * 32, nw = std::min(32, W - w0);
+            std::memcpy(chunk, row + w0, sizeof(uint32_t) * nw);
+            for (int k = nw; k < 32; k++) chunk[k] = 0;
+            uint64_t h = 1469598103934665603ull;
+            for (int k = 0; k < 32; k++) h = (h ^ chunk[k]) * 1099511628211ull;
+            if ((size_t)t.mask_chunks.size() / 32 * 2 >= cap) {   // keep the load factor below 1/2
+                size_t ncap = cap << 1;
+                std::vector<int64_t> ns(ncap, -1);
+                std::vector<uint64_t> nh(ncap, 0);
+                for (size_t i = 0; i < cap; i++) {
+                    if (slot[i] < 0) continue;
+                    size_t j = slot_hash[i] & (ncap - 1);
+                    while (ns[j] >= 0) j = (j + 1) & (ncap - 1);
+                    ns[j] = slot[i];
+                    nh[j] = slot_hash[i];
+                }
+                slot.swap(ns);
+                slot_hash.swap(nh);
+                cap = ncap;
+            }
+            size_t j = h & (cap - 1);
+            int64_t id = -1;
+            while (slot[j] >= 0) {
+                if (slot_hash[j] == h &&
+                    std::memcmp(t.mask_chunks.data() + (size_t)slot[j] * 32, chunk, sizeof(chunk)) == 0) {
+                    id = slot[j];
+                    break;
+                }
+                j = (j + 1) & (cap - 1);
+            }
+            if (id < 0) {
+                id = (int64_t)(t.mask_chunks.size() / 32);
+                t.mask_chunks.insert(t.mask_chunks.end(), chunk, chunk + 32);
+                slot[j] = id;
+                slot_hash[j] = h;
+            }
+            t.mask_rows[(size_t)m * nch + c] = (uint32_t)id;
+        }
+    }
+    t.n_chunks = (int)(t.mask_chunks.size() / 32);
+}
+
 Tables compile_tables(const std::string& text, const uint8_t* vb, const int64_t* vo, int V, int eos_id,
                       const Options& opt) {
     double t0 = now();
@@ -728,12 +786,13 @@ Tables compile_tables(const std::string& text, const uint8_t* vb, const int64_t*
     T.dfa_start.resize(L.nq);
     for (int q = 0; q < L.nq; q++) T.dfa_start[q] = enc(cls[start_state[q]]);
     T.V = V;
-    T.W = W;
-    T.n_masks = n_masks;
-    T.masks.assign((size_t)n_masks * W, 0);
-    for (size_t m = 0; m < mask_new.size(); m++)
-        if (mask_new[m] >= 0)
-            std::memcpy(T.masks.data() + (size_t)mask_new[m] * W, grows.data() + m * W, sizeof(uint32_t) * W);
+    {
+        std::vector<uint32_t> dense((size_t)n_masks * W, 0);
+        for (size_t m = 0; m < mask_new.size(); m++)
+            if (mask_new[m] >= 0)
+                std::memcpy(dense.data() + (size_t)mask_new[m] * W, grows.data() + m * W, sizeof(uint32_t) * W);
+        set_mask_rows(T, dense.data(), n_masks, W);
+    }
 
     // lexer and parser tables for the device
     T.nq = L.nq;

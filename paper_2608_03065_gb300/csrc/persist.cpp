@@ -3,7 +3,9 @@
 // preprocessing overhead); here the flat tables of a compiled handle are
 // written as one binary file: a magic/version header, every table as
 // (element count, raw little-endian bytes), and a 64-bit FNV-1a checksum of
-// everything before it.  No compression (the paper uses zstd).
+// everything before it.  The mask rows are stored as they are held in memory:
+// chunk ids plus the distinct 1024-token chunks (no general-purpose compression;
+// the paper uses zstd).
 #include <cstdio>
 #include <cstring>
 #include <type_traits>
@@ -13,7 +15,7 @@
 namespace psc {
 namespace {
 
-const char MAGIC[8] = {'P', 'S', 'C', 'T', 'A', 'B', '0', '1'};
+const char MAGIC[8] = {'P', 'S', 'C', 'T', 'A', 'B', '0', '2'};
 
 struct Writer {
     FILE* f;
@@ -69,12 +71,12 @@ void fields(S& s, Tables& t) {
     };
     int32_t contextual = t.contextual ? 1 : 0;
     sc(t.nq); sc(t.q0); sc(t.n_classes); sc(t.n_lr); sc(t.n_terms); sc(t.n_nts); sc(t.end_term);
-    sc(contextual); sc(t.S); sc(t.V); sc(t.W); sc(t.n_masks); sc(t.eos_id);
+    sc(contextual); sc(t.S); sc(t.V); sc(t.W); sc(t.n_masks); sc(t.nch); sc(t.n_chunks); sc(t.eos_id);
     sc(t.n_dfa_states_built); sc(t.n_threads); sc(t.n_trie_nodes); sc(t.seconds_total);
     t.contextual = contextual != 0;
     vc(t.lex_trans); vc(t.lex_accept); vc(t.cls_ignored);
     vc(t.action); vc(t.go); vc(t.rule_len); vc(t.rule_lhs); vc(t.resolve);
-    vc(t.dfa); vc(t.dfa_start); vc(t.dfa_mask); vc(t.masks);
+    vc(t.dfa); vc(t.dfa_start); vc(t.dfa_mask); vc(t.mask_rows); vc(t.mask_chunks);
     vc(t.vocab_bytes); vc(t.vocab_off);
 }
 
@@ -87,7 +89,10 @@ void validate(const Tables& t) {
     if (t.resolve.size() != (size_t)t.n_classes * t.n_lr || t.cls_ignored.size() != (size_t)t.n_classes) bad("classes");
     if (t.dfa.size() != (size_t)t.S * t.n_lr || t.dfa_mask.size() != (size_t)t.S || t.dfa_start.size() != (size_t)t.nq)
         bad("classifier");
-    if (t.W != (t.V + 31) / 32 || t.masks.size() != (size_t)t.n_masks * t.W || t.n_masks < 2) bad("masks");
+    if (t.W != (t.V + 31) / 32 || t.nch != (t.W + 31) / 32 || t.n_masks < 2 || t.n_chunks < 1 ||
+        t.mask_rows.size() != (size_t)t.n_masks * t.nch || t.mask_chunks.size() != (size_t)t.n_chunks * 32)
+        bad("masks");
+    for (uint32_t c : t.mask_rows) if (c >= (uint32_t)t.n_chunks) bad("mask chunk id");
     if (t.vocab_off.size() != (size_t)t.V + 1 || (uint64_t)t.vocab_off[t.V] != t.vocab_bytes.size()) bad("vocabulary");
     for (int32_t x : t.lex_trans) if (x < -1 || x >= t.nq) bad("lexer transition");
     for (int32_t c : t.lex_accept) if (c < -1 || c >= t.n_classes) bad("lexer class");

@@ -2,16 +2,17 @@
 //
 // Online step of the paper (Algorithm 2), per decoding step and batch row:
 //   steps 1-2  incremental lexing and LR parsing of the sampled token on the
-//              row's device-resident stack                      -> k_advance
+//              row's device-resident stack                      -> k_advance_warp
 //   step 3     one pass of the classifier DFA over (q, stack from the top),
-//              O(|stack|), stopping at absorbing states          -> k_classify
-//   step 4     the precomputed mask of the reached state         -> k_fill / k_apply_rows
+//              O(|stack|), stopping at absorbing states          -> k_advance_warp / k_classify
+//   step 4     the precomputed mask of the reached state         -> k_step_tma / k_fill / k_apply_rows
 // plus applying the mask to the logits and greedy sampling over the allowed
 // tokens (left to the serving engine in the paper).
 //
 // Memory layout on the device (all tables uploaded once by psc_compile):
 //   dfa      int32 [S][n_lr]      next classifier state, or -(mask+1) when absorbing
-//   masks    uint32 [n_masks][Wp] mask rows, Wp = W rounded up to 32 words (whole 1024-column chunks)
+//   mrows    uint32 [n_masks][nch] mask rows as ids of 1024-token chunks (nch = ceil(W / 32))
+//   mchunks  uint32 [n_chunks][32] the distinct chunks (words past W zero)
 //   stacks   uint16 [B][cap]      parser stacks, bottom first; depth[b] entries used
 //   logits   [B][row_stride]      bf16 or f32, caller-owned, masked in place
 #include <cuda_bf16.h>
@@ -51,11 +52,12 @@ struct DevTables {
     const int32_t* dfa;
     const int32_t* dfa_start;
     const int32_t* dfa_mask;
-    const uint32_t* masks;
+    const uint32_t* mchunks;   // distinct 32-word chunks of the mask rows [n_chunks][32]
+    const uint32_t* mrows;     // mask rows as chunk ids [n_masks][nch]
     const uint8_t* vocab;
     const int64_t* vocab_off;
     int q0, nq, n_lr, n_terms, n_nts, end_term;
-    int V, W, Wp, eos_id, n_masks;
+    int V, W, nch, eos_id, n_masks;
     // compact lexer/parser tables for k_advance_warp (adv_bytes = 0: not built)
     const uint8_t* adv;
     int adv_bytes, o_bc, o_trans, o_accept, o_ign, o_resolve, o_action, o_go, o_rlen, o_rlhs, nbc;
@@ -109,6 +111,12 @@ __device__ __forceinline__ uint4 ld_nc_v4(const void* p) {
                  : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
                  : "l"(p));
     return v;
+}
+
+// Word w of mask row `mid` (the mask of Section 3.5, held as chunk ids + chunks).
+__device__ __forceinline__ uint32_t mask_word(const DevTables& T, int mid, int w) {
+    uint32_t c = __ldg(T.mrows + (size_t)mid * T.nch + (w >> 5));
+    return __ldg(T.mchunks + (size_t)c * 32 + (w & 31));
 }
 
 // Classifier walk for one row (Algorithm 2 step 3), executed by a full warp:
@@ -183,23 +191,24 @@ __global__ void k_classify(DevTables T, DevStates S, int B) {
 }
 
 // out[b][:] = masks[mid[b]][:]   (16-byte vector copies when W % 4 == 0)
-__global__ void k_fill(const uint32_t* __restrict__ masks, int Wp, const int32_t* __restrict__ mid, int B, int W,
-                       uint32_t* __restrict__ out, int vec) {
+__global__ void k_fill(DevTables D, const int32_t* __restrict__ mid, int B, uint32_t* __restrict__ out, int vec) {
     size_t tid = blockIdx.x * (size_t)blockDim.x + threadIdx.x;
     size_t stride = (size_t)gridDim.x * blockDim.x;
+    int W = D.W;
     if (vec) {
         int W4 = W >> 2;
         size_t total = (size_t)B * W4;
         for (size_t i = tid; i < total; i += stride) {
             int b = (int)(i / W4), w = (int)(i % W4);
-            uint4 v = ld_nc_v4(masks + (size_t)mid[b] * Wp + 4 * w);
+            uint32_t c = __ldg(D.mrows + (size_t)__ldg(mid + b) * D.nch + ((4 * w) >> 5));
+            uint4 v = ld_nc_v4(D.mchunks + (size_t)c * 32 + ((4 * w) & 31));
             st_cs_v4(out + (size_t)b * W + 4 * w, v);
         }
     } else {
         size_t total = (size_t)B * W;
         for (size_t i = tid; i < total; i += stride) {
             int b = (int)(i / W), w = (int)(i % W);
-            out[i] = __ldg(masks + (size_t)mid[b] * Wp + w);
+            out[i] = mask_word(D, __ldg(mid + b), w);
         }
     }
 }
@@ -272,12 +281,18 @@ __device__ __forceinline__ void apply_chunk_scalar(T* row, int col0, int ncols, 
 // mask table row picked by the classifier (mid[b]).
 struct MaskSrc {
     const uint32_t* bitmask;   // nullable
-    const uint32_t* table;
+    const uint32_t* chunks;    // the device mask table (chunk ids + chunks)
+    const uint32_t* rows;
     const int32_t* mid;
-    int W, Wp;
+    int W, nch;
     uint32_t* copy_out;        // nullable: also write the words here ([B][W])
-    __device__ __forceinline__ const uint32_t* row(int b) const {
-        return bitmask ? bitmask + (size_t)b * W : table + (size_t)__ldg(mid + b) * Wp;
+    // word `lane` of 1024-column chunk j of row b (0 past W)
+    __device__ __forceinline__ uint32_t word(int b, int j, int lane) const {
+        int wi = j * 32 + lane;
+        if (wi >= W) return 0u;
+        if (bitmask) return __ldg(bitmask + (size_t)b * W + wi);
+        uint32_t c = __ldg(rows + (size_t)__ldg(mid + b) * nch + j);
+        return __ldg(chunks + (size_t)c * 32 + lane);
     }
 };
 
@@ -293,8 +308,7 @@ __global__ void __launch_bounds__(256) k_apply_rows(T* logits, int64_t stride, M
         int j = (int)(c - (long)b * cpr);
         int col0 = j << 10;
         int wi = (col0 >> 5) + lane;
-        const uint32_t* mrow = M.row(b);
-        uint32_t word = wi < M.W ? __ldg(mrow + wi) : 0u;
+        uint32_t word = M.word(b, j, lane);
         if (M.copy_out && wi < M.W) M.copy_out[(size_t)b * M.W + wi] = word;
         T* row = logits + (size_t)b * stride;
         int ncols = V - col0;
@@ -314,7 +328,7 @@ __global__ void __launch_bounds__(256) k_argmax_masked(const T* logits, int64_t 
     int b = blockIdx.x;
     if (b >= B) return;
     int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarp = blockDim.x >> 5;
-    const uint32_t* mrow = D.masks + (size_t)mid[b] * D.Wp;
+    const uint32_t* rowids = D.mrows + (size_t)mid[b] * D.nch;
     const T* row = logits + (size_t)b * stride;
     float best = 0.f;
     int bi = -1;
@@ -330,7 +344,7 @@ __global__ void __launch_bounds__(256) k_argmax_masked(const T* logits, int64_t 
     for (int j = warp; j < cpr; j += nwarp) {
         int col0 = j << 10;
         int wi = (col0 >> 5) + lane;
-        uint32_t word = wi < D.W ? __ldg(mrow + wi) : 0u;
+        uint32_t word = wi < D.W ? __ldg(D.mchunks + (size_t)__ldg(rowids + j) * 32 + lane) : 0u;
         if (__ballot_sync(FULL, word != 0) == 0) continue;
         int ncols = V - col0;
         if (vec && ncols >= 1024) {
@@ -437,7 +451,7 @@ __global__ void k_advance(DevTables T, DevStates S, const int32_t* tokens, int B
                 status = ROW_REJECTED;
             } else {
                 int mid = use_mid ? S.mid[b] : thread_classify(T, S, b);
-                bool allowed = (__ldg(T.masks + (size_t)mid * T.Wp + (tok >> 5)) >> (tok & 31)) & 1;
+                bool allowed = (mask_word(T, mid, tok >> 5) >> (tok & 31)) & 1;
                 if (!allowed) {
                     status = ROW_REJECTED;
                 } else if (tok == T.eos_id) {
@@ -773,14 +787,17 @@ __global__ void __launch_bounds__(256, 4) k_apply_argmax(T* logits, int64_t stri
         int sg = (int)(it - (long)b * nseg);
         int c0 = sg * seg_chunks;
         int c1 = min(c0 + seg_chunks, cpr);
-        const uint32_t* mrow;
+        int wmid = 0;
         if (WALK) {
-            int mid = s_mid[cur];
-            mrow = D.masks + (size_t)mid * D.Wp;
-            if (sg == 0 && threadIdx.x == 0) S.mid[b] = mid;
-        } else {
-            mrow = M.row(b);
+            wmid = s_mid[cur];
+            if (sg == 0 && threadIdx.x == 0) S.mid[b] = wmid;
         }
+        // word `lane` of chunk j of this row's mask
+        auto word_at = [&](int j) -> uint32_t {
+            if (!WALK) return M.word(b, j, lane);
+            int wi = j * 32 + lane;
+            return wi < D.W ? __ldg(D.mchunks + (size_t)__ldg(D.mrows + (size_t)wmid * D.nch + j) * 32 + lane) : 0u;
+        };
         T* row = logits + (size_t)b * stride;
         Best best{0.f, -1};
         if (WALK) {
@@ -796,7 +813,7 @@ __global__ void __launch_bounds__(256, 4) k_apply_argmax(T* logits, int64_t stri
                 if (j >= c1) break;
                 int col0 = j << 10;
                 int wi = (col0 >> 5) + lane;
-                uint32_t word = wi < M.W ? __ldg(mrow + wi) : 0u;
+                uint32_t word = word_at(j);
                 if (M.copy_out && wi < M.W) M.copy_out[(size_t)b * M.W + wi] = word;
                 apply_argmax_any<T>(row, col0, V, word, lane, vec, best, s_lut);
             }
@@ -804,7 +821,7 @@ __global__ void __launch_bounds__(256, 4) k_apply_argmax(T* logits, int64_t stri
             for (int j = c0 + warp; j < c1; j += 8) {
                 int col0 = j << 10;
                 int wi = (col0 >> 5) + lane;
-                uint32_t word = wi < M.W ? __ldg(mrow + wi) : 0u;
+                uint32_t word = word_at(j);
                 if (M.copy_out && wi < M.W) M.copy_out[(size_t)b * M.W + wi] = word;
                 apply_argmax_any<T>(row, col0, V, word, lane, vec, best, s_lut);
             }
@@ -1016,7 +1033,7 @@ __global__ void __launch_bounds__(ADV_WARPS * 32) k_advance_warp(DevTables T, De
                         mid = depth >= 1 && depth <= S.cap ? warp_walk(T, g, q, depth, lane) : 0;
                     }
                     // the token's mask bit; the row is only committed (q, depth) when it is set
-                    mword = __ldg(T.masks + (size_t)mid * T.Wp + (tok >> 5));
+                    mword = mask_word(T, mid, tok >> 5);
                     if (tok == T.eos_id) status = ((mword >> (tok & 31)) & 1) ? ROW_DONE : ROW_REJECTED;
                     else if (depth < 1 || depth > S.cap) status = ROW_REJECTED;
                     else parse = true;
@@ -1243,11 +1260,13 @@ __global__ void __launch_bounds__(TMA_WARPS * 32, 3) k_step_tma(T* logits, int64
             }
             if (use >= 1 && !__shfl_sync(FULL, (int)mbar_wait(mempty0 + 8 * slot, (uint32_t)((use - 1) & 1)), 0))
                 return false;
-            if (lane == 0) {
-                mbar_arrive_tx(mfull0 + 8 * slot, nch * 128);
-                tma_load_1d(smem_addr(mbuf + slot * TMA_SEG * 32), D.masks + (size_t)mid * D.Wp + (size_t)c0 * 32,
-                            nch * 128, mfull0 + 8 * slot);
-            }
+            // the item's chunk ids, then one 128-byte bulk copy per chunk (lane k: chunk k)
+            uint32_t cid = lane < nch ? __ldg(D.mrows + (size_t)mid * D.nch + c0 + lane) : 0u;
+            if (lane == 0) mbar_arrive_tx(mfull0 + 8 * slot, nch * 128);
+            __syncwarp();
+            if (lane < nch)
+                tma_load_1d(smem_addr(mbuf + slot * TMA_SEG * 32 + lane * 32), D.mchunks + (size_t)cid * 32, 128,
+                            mfull0 + 8 * slot);
             issued = ii;
             return true;
         };
@@ -1522,7 +1541,7 @@ psc_status launch_advance(const psc_handle* h, psc_states* st, const int32_t* d_
 psc_status launch_fused(const psc_handle* h, const psc_states* st, void* d_logits, psc_dtype dtype, int64_t row_stride,
                         int V, uint32_t* d_bitmask_out, cudaStream_t cs) {
     int B = st->d.B;
-    MaskSrc M{nullptr, h->d.masks, st->d.mid, h->d.W, h->d.Wp, d_bitmask_out};
+    MaskSrc M{nullptr, h->d.mchunks, h->d.mrows, st->d.mid, h->d.W, h->d.nch, d_bitmask_out};
     size_t esz = dtype == PSC_BF16 ? 2 : 4;
     int vec = aligned16(d_logits) && ((row_stride * (int64_t)esz) % 16 == 0);
     int cpr = (V + 1023) / 1024;
@@ -1690,10 +1709,6 @@ psc_status upload_tables(std::unique_ptr<psc_handle>& h, bool global_tables) {
     psc_status s = cuda_check(cudaGetDevice(&h->device), "cudaGetDevice");
     if (s != PSC_OK) return s;
     DevTables& d = h->d;
-    int Wp = (t.W + 31) & ~31;   // whole 1024-column chunks per row (16-byte and 128-byte aligned rows)
-    std::vector<uint32_t> masks((size_t)t.n_masks * Wp, 0);
-    for (int m = 0; m < t.n_masks; m++)
-        std::memcpy(masks.data() + (size_t)m * Wp, t.masks.data() + (size_t)m * t.W, sizeof(uint32_t) * t.W);
     std::vector<int32_t> dfa = t.dfa;
     if (dfa.empty()) dfa.push_back(0);
     std::vector<int32_t> dfa_mask = t.dfa_mask;
@@ -1703,7 +1718,8 @@ psc_status upload_tables(std::unique_ptr<psc_handle>& h, bool global_tables) {
         (s = upload(h.get(), t.go, &d.go)) || (s = upload(h.get(), t.rule_len, &d.rule_len)) ||
         (s = upload(h.get(), t.rule_lhs, &d.rule_lhs)) || (s = upload(h.get(), t.resolve, &d.resolve)) ||
         (s = upload(h.get(), dfa, &d.dfa)) || (s = upload(h.get(), t.dfa_start, &d.dfa_start)) ||
-        (s = upload(h.get(), dfa_mask, &d.dfa_mask)) || (s = upload(h.get(), masks, &d.masks)) ||
+        (s = upload(h.get(), dfa_mask, &d.dfa_mask)) || (s = upload(h.get(), t.mask_chunks, &d.mchunks)) ||
+        (s = upload(h.get(), t.mask_rows, &d.mrows)) ||
         (s = upload(h.get(), t.vocab_bytes, &d.vocab, 16)) || (s = upload(h.get(), t.vocab_off, &d.vocab_off))) {
         for (int i = 0; i < h->n_blocks; i++) cudaFree(h->blocks[i]);
         return s;
@@ -1756,7 +1772,7 @@ psc_status upload_tables(std::unique_ptr<psc_handle>& h, bool global_tables) {
     d.end_term = t.end_term;
     d.V = t.V;
     d.W = t.W;
-    d.Wp = Wp;
+    d.nch = t.nch;
     d.eos_id = t.eos_id;
     d.n_masks = t.n_masks;
     return PSC_OK;
@@ -1823,7 +1839,7 @@ psc_status psc_info(const psc_handle* h, psc_info_t* out) {
     out->n_masks = t.n_masks;
     out->eos_id = t.eos_id;
     out->classifier_bytes = (int64_t)(t.dfa.size() + t.dfa_start.size() + t.dfa_mask.size()) * 4;
-    out->mask_bytes = (int64_t)t.n_masks * ((t.W + 31) & ~31) * 4;
+    out->mask_bytes = (int64_t)(t.mask_rows.size() + t.mask_chunks.size()) * 4;
     out->states_built = t.n_dfa_states_built;
     out->compile_seconds = t.seconds_total;
     out->advance_table_bytes = h->host_only ? 0 : h->d.adv_bytes;
@@ -1945,7 +1961,7 @@ psc_status psc_fill_mask(const psc_handle* h, const psc_states* st, int32_t B, u
     size_t units = vec ? (size_t)B * (h->d.W / 4) : (size_t)B * h->d.W;
     int blocks = (int)std::min<size_t>((units + 255) / 256, (size_t)sm_count(h->device) * 8);
     if (blocks < 1) blocks = 1;
-    k_fill<<<blocks, 256, 0, cs>>>(h->d.masks, h->d.Wp, st->d.mid, B, h->d.W, d_bitmask, vec);
+    k_fill<<<blocks, 256, 0, cs>>>(h->d, st->d.mid, B, d_bitmask, vec);
     return launch_check("k_fill");
 }
 
@@ -1956,7 +1972,7 @@ psc_status psc_apply_mask(void* d_logits, psc_dtype dtype, int64_t row_stride, c
     if (B == 0) return PSC_OK;
     int dev = 0;
     cudaGetDevice(&dev);
-    MaskSrc M{d_bitmask, nullptr, nullptr, (V + 31) / 32, 0, nullptr};
+    MaskSrc M{d_bitmask, nullptr, nullptr, nullptr, (V + 31) / 32, 0, nullptr};
     return launch_apply(d_logits, dtype, row_stride, M, B, V, (cudaStream_t)stream, dev);
 }
 
@@ -1969,7 +1985,7 @@ psc_status psc_fill_apply(const psc_handle* h, const psc_states* st, int32_t B, 
         return fail_with(PSC_ERR_ARG, "psc_fill_apply: bad arguments");
     cudaStream_t cs = (cudaStream_t)stream;
     if ((s = ensure_mid(h, st, cs)) != PSC_OK) return s;
-    MaskSrc M{nullptr, h->d.masks, st->d.mid, h->d.W, h->d.Wp, d_bitmask_out};
+    MaskSrc M{nullptr, h->d.mchunks, h->d.mrows, st->d.mid, h->d.W, h->d.nch, d_bitmask_out};
     return launch_apply(d_logits, dtype, row_stride, M, B, V, cs, h->device);
 }
 
@@ -2071,7 +2087,7 @@ int32_t psc_host_classify(const psc_handle* h, int32_t q, const uint16_t* h_stac
 
 psc_status psc_host_mask_row(const psc_handle* h, int32_t mask_id, uint32_t* h_row) {
     if (!h || !h_row || mask_id < 0 || mask_id >= h->t.n_masks) return fail_with(PSC_ERR_ARG, "psc_host_mask_row: bad arguments");
-    std::memcpy(h_row, h->t.masks.data() + (size_t)mask_id * h->t.W, sizeof(uint32_t) * h->t.W);
+    for (int w = 0; w < h->t.W; w++) h_row[w] = psc::mask_word(h->t, mask_id, w);
     return PSC_OK;
 }
 
@@ -2092,7 +2108,7 @@ psc_status psc_host_advance(const psc_handle* h, int32_t* q, uint16_t* h_stack, 
         return PSC_OK;
     }
     int mid = psc::classify_host(T, *q, h_stack, *depth, st);
-    if (mid < 0 || !((T.masks[(size_t)mid * T.W + (tok >> 5)] >> (tok & 31)) & 1)) {
+    if (mid < 0 || !((psc::mask_word(T, mid, tok >> 5) >> (tok & 31)) & 1)) {
         *status = ROW_REJECTED;
         return PSC_OK;
     }
@@ -2146,7 +2162,7 @@ psc_status psc_fill_apply_noalloc(const psc_handle* h, const int32_t* d_q, const
     int blocks = (int)(((size_t)B * 32 + threads - 1) / threads);
     k_classify<<<blocks, threads, 0, cs>>>(h->d, S, B);
     if ((s = launch_check("k_classify")) != PSC_OK) return s;
-    MaskSrc M{nullptr, h->d.masks, mid, h->d.W, h->d.Wp, d_bitmask_out};
+    MaskSrc M{nullptr, h->d.mchunks, h->d.mrows, mid, h->d.W, h->d.nch, d_bitmask_out};
     return launch_apply(d_logits, dtype, row_stride, M, B, V, cs, h->device);
 }
 

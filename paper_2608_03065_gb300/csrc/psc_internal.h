@@ -105,9 +105,13 @@ struct Tables {
     std::vector<int32_t> dfa;            // [S][n_lr]: next state, or -(mask+1) when absorbing
     std::vector<int32_t> dfa_start;      // [nq]: first state after reading q (same encoding)
     std::vector<int32_t> dfa_mask;       // [S]: mask id when the stack ends in this state
-    // masks: row 0 = nothing allowed, row 1 = only the end-of-sequence token
-    int V = 0, W = 0, n_masks = 0;
-    std::vector<uint32_t> masks;         // [n_masks][W]
+    // masks: row 0 = nothing allowed, row 1 = only the end-of-sequence token.
+    // A row is stored as nch = ceil(W/32) ids of 32-word chunks (1024 tokens each);
+    // equal chunks are stored once (the table shrinks about tenfold on the C-like
+    // workloads).  Words past W in a row's last chunk are zero.
+    int V = 0, W = 0, n_masks = 0, nch = 0, n_chunks = 0;
+    std::vector<uint32_t> mask_rows;     // [n_masks][nch] chunk ids
+    std::vector<uint32_t> mask_chunks;   // [n_chunks][32]
     // vocabulary
     std::vector<uint8_t> vocab_bytes;
     std::vector<int64_t> vocab_off;      // [V+1]
@@ -116,6 +120,15 @@ struct Tables {
     int64_t n_dfa_states_built = 0, n_threads = 0, n_trie_nodes = 0;
     double seconds_lex = 0, seconds_dfa = 0, seconds_min = 0, seconds_total = 0;
 };
+
+// Word w of mask row m.
+inline uint32_t mask_word(const Tables& t, int m, int w) {
+    return t.mask_chunks[(size_t)t.mask_rows[(size_t)m * t.nch + (w >> 5)] * 32 + (w & 31)];
+}
+
+// Stores n dense mask rows of W words each (row m at rows + m * W) as chunk ids
+// and distinct chunks (ids numbered in the order chunks are first met).
+void set_mask_rows(Tables& t, const uint32_t* rows, int n, int W);
 
 Tables compile_tables(const std::string& grammar, const uint8_t* vocab_bytes, const int64_t* offsets,
                       int V, int eos_id, const Options& opt);
