@@ -83,7 +83,8 @@ typedef struct {
     int32_t n_masks;         /* distinct precomputed masks A_s (Section 3.5) */
     int32_t eos_id;
     int64_t classifier_bytes;  /* device bytes of the classifier tables (cf. Table 7, DFA) */
-    int64_t mask_bytes;        /* device bytes of the mask rows (cf. Table 7, masks) */
+    int64_t mask_bytes;        /* device bytes of the mask table (cf. Table 7, masks): each row is
+                                  held as ids of 1024-token chunks, equal chunks stored once */
     int64_t states_built;      /* classifier states before minimisation */
     double compile_seconds;
     int64_t advance_table_bytes;  /* bytes psc_advance stages in shared memory (0: it reads global memory) */
