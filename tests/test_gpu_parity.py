@@ -312,6 +312,51 @@ def test_state_copy_forks_a_batch(psc):
     assert e.value.code == 1
 
 
+def test_decode_sequence_in_a_cuda_graph(psc):
+    """A decode sequence (restore the batch from a saved copy, then 4 steps of
+    psc_decode_step on fresh logits) captured once in a CUDA graph and replayed
+    gives the same tokens, masked logits and states as running it eagerly."""
+    w = configs.load(3, batch=32)
+    h = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id)
+    snap = psc.psc_state_init(h, w.B, 256)
+    tm = torch.from_numpy(w.token_matrix()).cuda()
+    for j in range(tm.shape[1]):
+        psc.psc_advance(h, snap, tm[:, j].contiguous())
+    steps = 4
+    pristine = [w.logits(70 + i).cuda() for i in range(steps)]
+    # eager
+    st_e = psc.psc_state_init(h, w.B, 256)
+    psc.psc_state_copy(st_e, snap)
+    tok_e, x_e = [], []
+    for i in range(steps):
+        x = pristine[i].clone()
+        t = torch.empty(w.B, dtype=torch.int32, device="cuda")
+        psc.psc_decode_step(h, st_e, x, t)
+        tok_e.append(t)
+        x_e.append(x)
+    torch.cuda.synchronize()
+    # captured
+    st_g = psc.psc_state_init(h, w.B, 256)
+    xs = [torch.empty_like(p) for p in pristine]
+    toks = [torch.empty(w.B, dtype=torch.int32, device="cuda") for _ in range(steps)]
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        psc.psc_state_copy(st_g, snap)
+        for i in range(steps):
+            xs[i].copy_(pristine[i])
+            psc.psc_decode_step(h, st_g, xs[i], toks[i])
+    for rep in range(2):
+        g.replay()
+        torch.cuda.synchronize()
+        for i in range(steps):
+            np.testing.assert_array_equal(toks[i].cpu().numpy(), tok_e[i].cpu().numpy(), err_msg=f"step {i}")
+            np.testing.assert_array_equal(raw_bits(xs[i]), raw_bits(x_e[i]))
+        a, b = psc.psc_states_download(st_e), psc.psc_states_download(st_g)
+        for k in ("q", "depth", "status"):
+            np.testing.assert_array_equal(a[k], b[k])
+
+
 def _decode_loop(psc, c, steps, mode):
     """fill_apply -> argmax -> advance for several steps; after every step the
     device masks equal the oracle's after advancing it by the same tokens
