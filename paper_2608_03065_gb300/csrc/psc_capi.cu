@@ -1172,7 +1172,7 @@ __device__ __forceinline__ uint64_t l2_evict_first_policy() {
 }
 
 
-constexpr int TMA_SEG = 32;     // 1024-column chunks per work item (one per lane of a warp)
+constexpr int TMA_SEG = 32;     // most 1024-column chunks per work item (one per lane of a warp)
 constexpr int TMA_NCONS = 8;    // consumer warps; a ring stage holds one chunk for each of them
 constexpr int TMA_WARPS = TMA_NCONS + 2;   // + producer + walker
 constexpr int TMA_MIDS = 4;     // classified rows the walker may run ahead (it walks them together)
@@ -1191,7 +1191,7 @@ struct TmaShape {
 
 // One decode masking pass (classification, mask, apply, greedy key) with the
 // logits streamed through shared memory by TMA bulk copies.  Work item = (row,
-// segment of TMA_SEG chunks).  Warp 0 (producer) fetches each item's mask words
+// segment of `seg` <= TMA_SEG chunks).  Warp 0 (producer) fetches each item's mask words
 // one item ahead, then for every ring stage copies the stage's chunks that hold
 // an allowed position (runs of neighbouring chunks in one copy; chunks with
 // nothing allowed are not read); warp 1 walks the classifier for the CTA's
@@ -1202,7 +1202,7 @@ template <typename T>
 __global__ void __launch_bounds__(TMA_WARPS * 32, 3) k_step_tma(T* logits, int64_t stride, int B, int V,
                                                                 uint32_t* copy_out,
                                                                 unsigned long long* __restrict__ best_key,
-                                                                DevTables D, DevStates S, int have_mid) {
+                                                                DevTables D, DevStates S, int have_mid, int seg) {
     using Sh = TmaShape<T>;
     constexpr int NS = Sh::NS, CHUNK = Sh::CHUNK, STAGE = Sh::STAGE;
     static_assert(TMA_SEG == 32, "one lane per chunk of an item");
@@ -1215,7 +1215,7 @@ __global__ void __launch_bounds__(TMA_WARPS * 32, 3) k_step_tma(T* logits, int64
     __shared__ uint4 s_lut[256];
     int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     int cpr = (V + 1023) >> 10;
-    int nseg = (cpr + TMA_SEG - 1) / TMA_SEG;
+    int nseg = (cpr + seg - 1) / seg;
     build_allow_lut<T>(s_lut);
     long items = (long)B * nseg;
     const uint32_t full0 = smem_addr(bars), empty0 = full0 + 8 * NS, mfull0 = empty0 + 8 * NS;
@@ -1248,7 +1248,7 @@ __global__ void __launch_bounds__(TMA_WARPS * 32, 3) k_step_tma(T* logits, int64
         // request item ii's mask words (its row classified by the walker) into slot ii % TMA_MSLOTS
         auto fetch_mask = [&](int ii, long itm) -> bool {
             int b = (int)(itm / nseg), sg = (int)(itm - (long)b * nseg);
-            int c0 = sg * TMA_SEG, nch = min(TMA_SEG, cpr - c0);
+            int c0 = sg * seg, nch = min(seg, cpr - c0);
             int ms = ii % TMA_MIDS;
             if (!__shfl_sync(FULL, (int)mbar_wait(midf0 + 8 * ms, (uint32_t)((ii / TMA_MIDS) & 1)), 0)) return false;
             int mid = s_mid[ms];
@@ -1274,7 +1274,7 @@ __global__ void __launch_bounds__(TMA_WARPS * 32, 3) k_step_tma(T* logits, int64
         if ((long)blockIdx.x < items && !fetch_mask(0, blockIdx.x)) failed = true;
         for (long it = blockIdx.x; it < items && !failed; it += gridDim.x, i++) {
             int b = (int)(it / nseg), sg = (int)(it - (long)b * nseg);
-            int c0 = sg * TMA_SEG, nch = min(TMA_SEG, cpr - c0);
+            int c0 = sg * seg, nch = min(seg, cpr - c0);
             if (it + gridDim.x < items && !fetch_mask(i + 1, it + gridDim.x)) { failed = true; break; }
             int slot = i % TMA_MSLOTS;
             if (!__shfl_sync(FULL, (int)mbar_wait(mfull0 + 8 * slot, (uint32_t)((i / TMA_MSLOTS) & 1)), 0)) {
@@ -1349,7 +1349,7 @@ __global__ void __launch_bounds__(TMA_WARPS * 32, 3) k_step_tma(T* logits, int64
         int i = 0;
         for (long it = blockIdx.x; it < items && !failed; it += gridDim.x, i++) {
             int b = (int)(it / nseg), sg = (int)(it - (long)b * nseg);
-            int c0 = sg * TMA_SEG, nch = min(TMA_SEG, cpr - c0);
+            int c0 = sg * seg, nch = min(seg, cpr - c0);
             int slot = i % TMA_MSLOTS;
             if (!__shfl_sync(FULL, (int)mbar_wait(mfull0 + 8 * slot, (uint32_t)((i / TMA_MSLOTS) & 1)), 0)) {
                 failed = true;
@@ -1554,17 +1554,21 @@ psc_status launch_fused(const psc_handle* h, const psc_states* st, void* d_logit
     psc_status s;
     if (vec) {
         // TMA pipeline: one item = (row, 32 chunks); as many CTAs as are resident at once
-        long titems = (long)B * ((cpr + TMA_SEG - 1) / TMA_SEG);
+        // items of 32 chunks; smaller (multiples of a stage) when the batch has too few
+        // chunks to give every resident CTA work
         long resident = (long)sm_count(h->device) * h->tma_ctas[dtype == PSC_BF16 ? 0 : 1];
+        long want = ((long)B * cpr + resident - 1) / resident;
+        int seg = (int)std::min<long>(TMA_SEG, std::max<long>(TMA_NCONS, (want + TMA_NCONS - 1) / TMA_NCONS * TMA_NCONS));
+        long titems = (long)B * ((cpr + seg - 1) / seg);
         int tgrid = (int)std::max(1L, std::min<long>(titems, resident));
         if (dtype == PSC_BF16)
             s = launch_pdl(k_step_tma<uint16_t>, dim3(tgrid), dim3(TMA_WARPS * 32), TmaShape<uint16_t>::SMEM, cs,
                            "k_step_tma", (uint16_t*)d_logits, row_stride, B, V, d_bitmask_out, st->d.best, h->d,
-                           st->d, have_mid);
+                           st->d, have_mid, seg);
         else
             s = launch_pdl(k_step_tma<uint32_t>, dim3(tgrid), dim3(TMA_WARPS * 32), TmaShape<uint32_t>::SMEM, cs,
                            "k_step_tma", (uint32_t*)d_logits, row_stride, B, V, d_bitmask_out, st->d.best, h->d,
-                           st->d, have_mid);
+                           st->d, have_mid, seg);
     } else {
         if (dtype == PSC_BF16)
             k_apply_argmax<uint16_t, true><<<grid, 256, 0, cs>>>((uint16_t*)d_logits, row_stride, M, B, V, vec,
