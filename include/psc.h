@@ -160,14 +160,17 @@ psc_status psc_state_copy(psc_states* dst, const psc_states* src, void* stream);
  * token outside it sets PSC_ROW_REJECTED; the end-of-sequence token sets
  * PSC_ROW_DONE; any other allowed token is lexed from the row's lexer state and
  * the emitted terminals are fed to the LALR(1) parser on the row's stack.
+ * Afterwards every row is classified (step 3) and its mask id kept in the
+ * states object, so the next mask call reads it without walking the stack.
  * d_tokens[b] < 0 leaves row b unchanged.  B must equal the batch size.
  *   d_row_status : optional device int32[B] copy of the statuses after the step. */
 psc_status psc_advance(const psc_handle* h, psc_states* st, const int32_t* d_tokens, int32_t B,
                        int32_t* d_row_status, void* stream);
 
 /* Algorithm 2, steps 3-4: classifies every row's (q, alpha) with the classifier
- * DFA (one pass over the stack from the top, stopping at absorbing states) and
- * writes the precomputed mask of the resulting state as a packed bitmask.
+ * DFA (one pass over the stack from the top, stopping at absorbing states;
+ * skipped when the last psc_advance or decode step already did it) and writes
+ * the precomputed mask of the resulting state as a packed bitmask.
  *   d_bitmask : device uint32 [B][W], W = ceil(V/32), row-contiguous.
  * Rows with status DONE get the end-of-sequence-only mask, failed rows the
  * empty mask. */
@@ -201,11 +204,12 @@ psc_status psc_argmax_masked(const psc_handle* h, const psc_states* st, int32_t 
                              psc_dtype dtype, int64_t row_stride, int32_t V, int32_t* d_tokens,
                              void* stream);
 
-/* psc_fill_apply and psc_argmax_masked in one pass over the logits: every
- * 16-byte chunk is touched once (written with -inf when fully masked, read
- * when it holds an allowed position, read and rewritten when mixed) and the
- * greedy choice among allowed tokens is merged per row with a 64-bit atomic
- * maximum (value order, then the lowest index).  d_tokens[b] = chosen token or
+/* psc_fill_apply and psc_argmax_masked in one pass over the logits: each
+ * 1024-token chunk holding an allowed position is read once (a chunk with none
+ * is only written), every 32-byte sector that holds a masked position is
+ * written once with -inf in the masked places, and the greedy choice among
+ * allowed tokens is merged per row with a 64-bit atomic maximum (value order,
+ * then the lowest index).  d_tokens[b] = chosen token or
  * -1 when row b allows nothing; d_bitmask_out as in psc_fill_apply.  The
  * per-row keys live in the states object; calls on the same states object
  * must not overlap. */
