@@ -950,8 +950,17 @@ __device__ __forceinline__ int feed_class_win(const uint8_t* sm, const DevTables
 // Classifier walk of a configuration (lexer state q, stack of the given depth
 // read through the view) by a full warp: lanes fetch 32 stack symbols at a time,
 // the walk broadcasts them with shuffles.  Every lane returns the mask id.
+// 4-byte read-only load with an L2 cache policy (the classifier table: its lines are
+// kept in L2 ahead of the logits the masking pass streams through it).
+__device__ __forceinline__ int ld_keep(const int32_t* p, uint64_t pol) {
+    int v;
+    asm volatile("ld.global.nc.L2::cache_hint.b32 %0, [%1], %2;" : "=r"(v) : "l"(p), "l"(pol));
+    return v;
+}
 __device__ __forceinline__ int warp_walk(const DevTables& T, const StackView& sv, int q, int depth, int lane) {
     if (q < 0 || q >= T.nq || depth < 1) return 0;
+    uint64_t pol;
+    asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(pol));
     int s = __ldg(T.dfa_start + q);
     if (s < 0) return -s - 1;
     for (int top = depth - 1; top >= 0; top -= 32) {
@@ -960,7 +969,7 @@ __device__ __forceinline__ int warp_walk(const DevTables& T, const StackView& sv
         int n = top + 1 < 32 ? top + 1 : 32;
         for (int j = 0; j < n; j++) {
             int X = __shfl_sync(FULL, x, j);
-            int nx = __ldg(T.dfa + (size_t)s * T.n_lr + X);
+            int nx = ld_keep(T.dfa + (size_t)s * T.n_lr + X, pol);
             if (nx < 0) return -nx - 1;
             s = nx;
         }
@@ -1003,21 +1012,28 @@ __global__ void __launch_bounds__(ADV_WARPS * 32) k_advance_warp(DevTables T, De
     int len = 0;
     int64_t vlo = 0;
     if (active) {
-        if (lane == 0) {
-            if (from_keys) {   // the greedy choice of the fused masking pass
-                unsigned long long k = S.best[b];
-                S.best[b] = 0ull;
-                tok = k ? (int32_t)(~(uint32_t)(k & 0xFFFFFFFFu)) : -1;
-                tokens_out[b] = tok;
-            } else {
-                tok = tokens[b];
-            }
-            status = S.status[b];
-        }
-        tok = __shfl_sync(FULL, tok, 0);
-        status = __shfl_sync(FULL, status, 0);
+        // the loads that need nothing but the row index go first, together
         q = S.q[b];
         depth = S.depth[b];
+        status = S.status[b];
+        int mid = use_mid ? S.mid[b] : 0;
+        if (from_keys) {   // the greedy choice of the fused masking pass
+            unsigned long long k = S.best[b];
+            tok = k ? (int32_t)(~(uint32_t)(k & 0xFFFFFFFFu)) : -1;
+            __syncwarp();
+            if (lane == 0) {
+                S.best[b] = 0ull;
+                tokens_out[b] = tok;
+            }
+        } else {
+            tok = tokens[b];
+        }
+        // the window of the stack top: for the parse and for the classifier walk after it
+        bool live = status == ROW_OK && depth >= 1 && depth <= S.cap;
+        if (live) {
+            sv.base = depth > ADV_KEEP ? depth - ADV_KEEP : 0;
+            for (int i = lane; i < depth - sv.base; i += 32) sv.win[i] = sv.st[sv.base + i];
+        }
         if (tok >= 0) {
             if (status == ROW_DONE) {
                 status = tok == T.eos_id ? ROW_DONE : ROW_REJECTED;
@@ -1025,32 +1041,25 @@ __global__ void __launch_bounds__(ADV_WARPS * 32) k_advance_warp(DevTables T, De
                 if (tok >= T.V) {
                     status = ROW_REJECTED;
                 } else {
-                    int mid;
-                    if (use_mid) {
-                        mid = S.mid[b];
-                    } else {
-                        StackView g{sv.win, sv.st, 0x40000000, 0x7FFFFFFF};   // all of the stack in global memory
+                    if (!use_mid) {
+                        StackView g{sv.win, sv.st, 0x40000000, 0x7FFFFFFF};   // the stack in global memory
                         mid = depth >= 1 && depth <= S.cap ? warp_walk(T, g, q, depth, lane) : 0;
                     }
-                    // the token's mask bit; the row is only committed (q, depth) when it is set
+                    // the token's mask bit (in flight while the token is parsed); the row is
+                    // only committed (q, depth) when it is set
                     mword = mask_word(T, mid, tok >> 5);
                     if (tok == T.eos_id) status = ((mword >> (tok & 31)) & 1) ? ROW_DONE : ROW_REJECTED;
-                    else if (depth < 1 || depth > S.cap) status = ROW_REJECTED;
+                    else if (!live) status = ROW_REJECTED;
                     else parse = true;
                 }
             }
         }
-        if (parse) {
-            // the window of the stack top and the token's bytes, loaded together
-            sv.base = depth > ADV_KEEP ? depth - ADV_KEEP : 0;
-            for (int i = lane; i < depth - sv.base; i += 32) sv.win[i] = sv.st[sv.base + i];
-            if (lane == 0) {
-                vlo = T.vocab_off[tok];
-                len = (int)(T.vocab_off[tok + 1] - vlo);
+        if (parse && lane == 0) {   // the token's bytes
+            vlo = T.vocab_off[tok];
+            len = (int)(T.vocab_off[tok + 1] - vlo);
 #pragma unroll
-                for (int i = 0; i < 32; i++)
-                    if (i < len) tw[i >> 2] |= (uint32_t)T.vocab[vlo + i] << (8 * (i & 3));
-            }
+            for (int i = 0; i < 32; i++)
+                if (i < len) tw[i >> 2] |= (uint32_t)T.vocab[vlo + i] << (8 * (i & 3));
         }
     }
     __syncthreads();
@@ -1077,7 +1086,10 @@ __global__ void __launch_bounds__(ADV_WARPS * 32) k_advance_warp(DevTables T, De
         if (lane == 0) {
             int top = sv.win[depth - 1 - sv.base];
             for (int i = 0; i < len && status == ROW_OK; i++) {
-                int byte = i < 32 ? (int)((tw[i >> 2] >> (8 * (i & 3))) & 0xFFu) : (int)T.vocab[vlo + i];
+                uint32_t wsel = tw[0];   // tw[i >> 2] by selects (registers, not local memory)
+#pragma unroll
+                for (int k = 1; k < 8; k++) wsel = (i >> 2) == k ? tw[k] : wsel;
+                int byte = i < 32 ? (int)((wsel >> (8 * (i & 3))) & 0xFFu) : (int)T.vocab[vlo + i];
                 int c = bc[byte];
                 int nx = trans[nq * T.nbc + c];
                 if (nx >= 0) {
@@ -1117,8 +1129,8 @@ __global__ void __launch_bounds__(ADV_WARPS * 32) k_advance_warp(DevTables T, De
         if (tok >= 0) S.status[b] = status;
         if (status_out) status_out[b] = status;
     }
-    // the next masking pass's mask id (without a parse the window holds nothing:
-    // sv.base still points past any stack index, so the walk reads global memory)
+    // the next masking pass's mask id (the window holds the stack top of every live
+    // row; for the others sv.base still points past any stack index)
     int mid;
     if (status == ROW_DONE) mid = 1;
     else if (status != ROW_OK) mid = 0;
