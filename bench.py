@@ -190,6 +190,30 @@ def run_reference(args):
     }))
 
 
+# ------------------------------------------------------------- multi-rank
+def max_over_ranks(x: float, device) -> float:
+    """The largest x of all ranks (x itself with one process)."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return x
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(world: int, steps: int, elapsed_ms: float) -> float:
+    """Steps/s of the whole job: every rank runs its own replica of the workload for
+    the same number of steps; the slowest rank's time (max over ranks) counts."""
+    return world * steps / (elapsed_ms / 1000.0)
+
+
+def barrier():
+    import torch.distributed as dist
+    if dist.is_available() and dist.is_initialized() and dist.get_world_size() > 1:
+        dist.barrier()
+
+
 def config_block(w, n):
     return {"workload": f"config 5: C-like grammar, vocab {w.V}, batch {w.B}, bf16 logits ~N(0,2), "
                         "decode steps (mask+apply+greedy+advance)",
@@ -411,8 +435,7 @@ def main():
     for i in range(Wm):
         step(i)
     torch.cuda.synchronize()
-    if world > 1:
-        dist.barrier()
+    barrier()
     torch.cuda.synchronize()
     t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with ClockSampler(index=local) as clocks:
@@ -425,18 +448,14 @@ def main():
         t_end.record(stream)
         torch.cuda.synchronize()
         torch.cuda.nvtx.range_pop()
-    if world > 1:
-        dist.barrier()
+    barrier()
     torch.cuda.synchronize()
     elapsed_ms = t_start.elapsed_time(t_end)
     mask_ms = [a.elapsed_time(b) for a, b, _ in ev]      # k_step_tma alone
     step_ms = [a.elapsed_time(c) for a, _, c in ev]      # the whole decode step
-    if world > 1:
-        tt = torch.tensor([elapsed_ms], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        elapsed_ms = float(tt.item())
+    elapsed_ms = max_over_ranks(elapsed_ms, dev)
     ms_per_step = elapsed_ms / K
-    value = world * K / (elapsed_ms / 1000.0)
+    value = whole_job_rate(world, K, elapsed_ms)
 
     # end to end through the public API with host buffers: H2D of each step's
     # logits from pinned memory, the step, D2H of the chosen tokens
@@ -447,8 +466,7 @@ def main():
     tok_host = torch.empty(B, dtype=torch.int32, pin_memory=True)
     dbuf = bufs[0]
     torch.cuda.synchronize()
-    if world > 1:
-        dist.barrier()
+    barrier()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
     for i in range(K):
@@ -459,12 +477,8 @@ def main():
         tok_host.copy_(tok, non_blocking=True)
     e1.record(stream)
     torch.cuda.synchronize()
-    e2e_ms = e0.elapsed_time(e1)
-    if world > 1:
-        tt = torch.tensor([e2e_ms], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        e2e_ms = float(tt.item())
-    e2e_value = world * K / (e2e_ms / 1000.0)
+    e2e_ms = max_over_ranks(e0.elapsed_time(e1), dev)
+    e2e_value = whole_job_rate(world, K, e2e_ms)
 
     # the plain mask paths on the same workload (prefix states, mask ids current),
     # each the median of 50 launches with CUDA events, logits buffers in rotation
