@@ -533,6 +533,10 @@ def main():
         "k_step_tma_us": mask_avg_ms * 1000.0,
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "traffic": traffic,
+                     # the same duration over the DRAM bytes ncu measured for one launch (the
+                     # kernel skips bytes the formula counts: frac can pass 1, this cannot)
+                     "dram_achieved": traffic / (mask_avg_ms / 1000.0) / 1e9 if traffic else None,
+                     "dram_frac": traffic / (mask_avg_ms / 1000.0) / 1e9 / peak if traffic else None,
                      "kernel": "k_step_tma (masking pass + greedy choice, CUDA events around each launch)",
                      "algorithmic_bytes": alg_bytes, "peak_kind": peak_kind},
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": B * V * 2,
