@@ -2103,7 +2103,12 @@ int32_t psc_host_classify(const psc_handle* h, int32_t q, const uint16_t* h_stac
 
 psc_status psc_host_mask_row(const psc_handle* h, int32_t mask_id, uint32_t* h_row) {
     if (!h || !h_row || mask_id < 0 || mask_id >= h->t.n_masks) return fail_with(PSC_ERR_ARG, "psc_host_mask_row: bad arguments");
-    for (int w = 0; w < h->t.W; w++) h_row[w] = psc::mask_word(h->t, mask_id, w);
+    const psc::Tables& t = h->t;
+    for (int c = 0; c < t.nch; c++) {   // chunk by chunk
+        int nw = std::min(32, t.W - c * 32);
+        std::memcpy(h_row + c * 32, t.mask_chunks.data() + (size_t)t.mask_rows[(size_t)mask_id * t.nch + c] * 32,
+                    sizeof(uint32_t) * nw);
+    }
     return PSC_OK;
 }
 
