@@ -470,22 +470,40 @@ def main():
     value = whole_job_rate(world, K, elapsed_ms)
 
     # end to end through the public API with host buffers: H2D of each step's
-    # logits from pinned memory, the step, D2H of the chosen tokens
+    # logits from pinned memory, the step, D2H of the chosen tokens.  Two device
+    # buffers: the next step's logits are copied (on a second stream) while the
+    # current step runs, as a serving loop would overlap them.
     n_host = 2
     host = [torch.empty(B, V, dtype=torch.bfloat16, pin_memory=True) for _ in range(n_host)]
     for k in range(n_host):
         host[k].copy_(bufs[k])
     tok_host = torch.empty(B, dtype=torch.int32, pin_memory=True)
-    dbuf = bufs[0]
+    dbufs = [bufs[0], bufs[1]]
+    copy_stream = torch.cuda.Stream(device=dev)
+    ready = [torch.cuda.Event() for _ in range(2)]
+    free = [torch.cuda.Event() for _ in range(2)]
     torch.cuda.synchronize()
     barrier()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
+    for k in range(2):
+        free[k].record(stream)
+    copy_stream.wait_stream(stream)
+    with torch.cuda.stream(copy_stream):
+        dbufs[0].copy_(host[0], non_blocking=True)
+    ready[0].record(copy_stream)
     for i in range(K):
+        cur, nxt = i % 2, (i + 1) % 2
+        if i + 1 < K:   # the next step's logits, into the buffer the previous step used
+            copy_stream.wait_event(free[nxt])
+            with torch.cuda.stream(copy_stream):
+                dbufs[nxt].copy_(host[(i + 1) % n_host], non_blocking=True)
+            ready[nxt].record(copy_stream)
         if i % SEQ == 0:
             restore()
-        dbuf.copy_(host[i % n_host], non_blocking=True)
-        psc.psc_decode_step(h, st, dbuf, tok, bitmask, stat, stream=stream)
+        stream.wait_event(ready[cur])
+        psc.psc_decode_step(h, st, dbufs[cur], tok, bitmask, stat, stream=stream)
+        free[cur].record(stream)
         tok_host.copy_(tok, non_blocking=True)
     e1.record(stream)
     torch.cuda.synchronize()
