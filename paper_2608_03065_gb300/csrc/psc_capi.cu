@@ -1558,14 +1558,9 @@ psc_status launch_fused(const psc_handle* h, const psc_states* st, void* d_logit
     int vec = aligned16(d_logits) && ((row_stride * (int64_t)esz) % 16 == 0);
     int cpr = (V + 1023) / 1024;
     int have_mid = st->mid_gen == st->gen ? 1 : 0;   // mask ids current: no classifier walks
-    int slots = sm_count(h->device) * 4;   // 4 resident CTAs of 256 threads per SM
-    long seg = ((long)cpr * B) / (2L * slots);
-    int seg_chunks = (int)std::max(1L, std::min(32L, seg));
-    long items = (long)B * ((cpr + seg_chunks - 1) / seg_chunks);
-    int grid = (int)std::max(1L, std::min<long>(items, slots));
     psc_status s;
     if (vec) {
-        // TMA pipeline: one item = (row, 32 chunks); as many CTAs as are resident at once
+        // the pipelined pass (rows 16-byte aligned): as many CTAs as are resident at once;
         // items of 32 chunks; smaller (multiples of a stage) when the batch has too few
         // chunks to give every resident CTA work
         long resident = (long)sm_count(h->device) * h->tma_ctas[dtype == PSC_BF16 ? 0 : 1];
@@ -1582,6 +1577,12 @@ psc_status launch_fused(const psc_handle* h, const psc_states* st, void* d_logit
                            "k_step_tma", (uint32_t*)d_logits, row_stride, B, V, d_bitmask_out, st->d.best, h->d,
                            st->d, have_mid, seg);
     } else {
+        // rows not 16-byte aligned: warp-per-chunk pass, 4 resident CTAs of 256 threads per SM
+        int slots = sm_count(h->device) * 4;
+        long seg = ((long)cpr * B) / (2L * slots);
+        int seg_chunks = (int)std::max(1L, std::min(32L, seg));
+        long items = (long)B * ((cpr + seg_chunks - 1) / seg_chunks);
+        int grid = (int)std::max(1L, std::min<long>(items, slots));
         if (dtype == PSC_BF16)
             k_apply_argmax<uint16_t, true><<<grid, 256, 0, cs>>>((uint16_t*)d_logits, row_stride, M, B, V, vec,
                                                                   seg_chunks, st->d.best, h->d, st->d);
