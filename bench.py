@@ -369,6 +369,56 @@ def run_teacher(args):
     print(json.dumps(out))
 
 
+# --------------------------------------------------------------- sweep mode
+def run_sweep(args):
+    """psc_decode_step on config 5's tables at several batch sizes (rows of the
+    workload's prefix states, repeated) and both logit types: µs per step (median
+    of 16 steps, each on fresh logits, from the same prefix states) and the rate of
+    the formula's bytes."""
+    import torch
+    from paper_2608_03065_gb300 import build, psc
+    from workloads import configs
+    build.build()
+    dev = torch.device("cuda", 0)
+    w = configs.load(WORKLOAD)
+    h = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id)
+    V = w.V
+    tm = torch.from_numpy(w.token_matrix()).to(dev)
+    peak, _ = measured_peaks()
+    out = {"metric": "decode step over batch size and logit type", "mode": "sweep", "vocab": V, "points": []}
+    stream = torch.cuda.current_stream()
+    snaps = {}
+    for B in (1, 16, 128, 1024):   # rows 0..B-1 of the prefix states
+        snaps[B] = psc.psc_state_init(h, B, 256)
+        for j in range(tm.shape[1]):
+            psc.psc_advance(h, snaps[B], tm[:B, j].contiguous())
+    for dt, esz in ((torch.bfloat16, 2), (torch.float32, 4)):
+        for B in (1, 16, 128, 1024):
+            st = psc.psc_state_init(h, B, 256)
+            tok = torch.empty(B, dtype=torch.int32, device=dev)
+            n = 16
+            gen = torch.Generator(device=dev).manual_seed(B)
+            xs = [(torch.randn(B, V, generator=gen, device=dev) * w.spec.sigma).to(dt) for _ in range(n)]
+            times = []
+            for i in range(n):
+                psc.psc_state_copy(st, snaps[B], stream=stream)
+                a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                a.record(stream)
+                psc.psc_decode_step(h, st, xs[i], tok, stream=stream)
+                b.record(stream)
+                torch.cuda.synchronize()
+                times.append(a.elapsed_time(b) * 1000.0)
+            times.sort()
+            us = times[n // 2]
+            alg = B * V // 8 + 2 * B * V * esz
+            out["points"].append({"dtype": "bf16" if esz == 2 else "f32", "batch": B, "us_per_step": round(us, 1),
+                                  "algorithmic_GBps": round(alg / (us * 1e-6) / 1e9, 1),
+                                  "frac": round(alg / (us * 1e-6) / 1e9 / peak, 3)})
+            del xs
+            torch.cuda.empty_cache()
+    print(json.dumps(out))
+
+
 # ------------------------------------------------------------------ main arm
 def main():
     ap = argparse.ArgumentParser()
@@ -377,14 +427,17 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="gb300")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--mode", default="decode", choices=["decode", "teacher"],
+    ap.add_argument("--mode", default="decode", choices=["decode", "teacher", "sweep"],
                     help="decode: the benchmark line; teacher: teacher-forcing pass rates and "
-                         "batch-1 step latency (the paper's RQ1/RQ2 measurements on these workloads)")
+                         "batch-1 step latency (the paper's RQ1/RQ2 measurements on these workloads); "
+                         "sweep: decode-step time over batch sizes and logit types on config 5's tables")
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)
     if args.mode == "teacher":
         return run_teacher(args)
+    if args.mode == "sweep":
+        return run_sweep(args)
 
     import torch
     import torch.distributed as dist
