@@ -72,6 +72,10 @@ typedef struct {
     int32_t host_only;       /* 1: build host tables only (no GPU needed; device calls fail) */
     int32_t global_tables;   /* 1: psc_advance reads its tables from global memory even when they
                                 would fit in shared memory (0 = stage them when they fit) */
+    int64_t max_bottom_up_bytes;  /* host memory for building the bottom-up classifier (0 = 8 GiB);
+                                     negative: not built (psc_load: dropped), and the device walks
+                                     every stack from the top.  Over the limit it is not built
+                                     (no error). */
 } psc_options;
 
 typedef struct {
@@ -90,6 +94,8 @@ typedef struct {
     int64_t advance_table_bytes;  /* bytes psc_advance stages in shared memory (0: it reads global memory) */
     int64_t device_timeouts;      /* bounded in-kernel waits that gave up since the library was loaded
                                      (process-wide; non-zero means a pipeline fault; reading it synchronises) */
+    int64_t bottom_up_states;     /* states of the bottom-up classifier (0: not built) */
+    int64_t bottom_up_bytes;      /* its device bytes (blocks, edge slots, final table) */
 } psc_info_t;
 
 /* Offline construction (Algorithm 1, Section 3).  Reads the grammar text (a
@@ -148,7 +154,8 @@ psc_status psc_state_reset(psc_states* st, const int32_t* d_rows, int32_t n, voi
 void psc_state_destroy(psc_states* st);
 
 /* Copies every row of src into dst: lexer states, depths, statuses, stacks,
- * mask ids and pending greedy choices (device-to-device, enqueued on stream).
+ * mask ids, pending greedy choices and the bottom-up classifier's kept states
+ * (device-to-device, enqueued on stream).
  * Both objects must belong to the same handle and have the same B and cap
  * (else PSC_ERR_ARG).  The paper has no counterpart: it serves forking a batch
  * (beam search, speculative branches) and restoring a saved one, e.g. to
@@ -162,6 +169,9 @@ psc_status psc_state_copy(psc_states* dst, const psc_states* src, void* stream);
  * the emitted terminals are fed to the LALR(1) parser on the row's stack.
  * Afterwards every row is classified (step 3) and its mask id kept in the
  * states object, so the next mask call reads it without walking the stack.
+ * With the bottom-up classifier (psc_options.max_bottom_up_bytes >= 0, the
+ * default) the classification re-reads only the stack entries the step
+ * pushed; without it the stack is walked from the top.
  * d_tokens[b] < 0 leaves row b unchanged.  B must equal the batch size.
  *   d_row_status : optional device int32[B] copy of the statuses after the step. */
 psc_status psc_advance(const psc_handle* h, psc_states* st, const int32_t* d_tokens, int32_t B,
@@ -257,6 +267,16 @@ psc_status psc_states_download(const psc_states* st, int32_t* h_q, int32_t* h_de
  * row `mask_id` (W words) to h_row. */
 int32_t psc_host_classify(const psc_handle* h, int32_t q, const uint16_t* h_stack, int32_t depth,
                           int32_t status);
+
+/* The same classification through the bottom-up classifier (the classifier
+ * DFA reversed, reading the stack from the bottom; the regularity theorem of
+ * Section 3.5 is what makes this automaton exist): returns the mask id, -1 on
+ * bad arguments, or -2 when the handle has no bottom-up classifier or the
+ * stack is not a path of the LR automaton (no parser builds such a stack).
+ * States objects keep this automaton's state after every stack prefix of
+ * every row, so a decode step re-reads only the entries it pushed. */
+int32_t psc_host_classify_bottom_up(const psc_handle* h, int32_t q, const uint16_t* h_stack, int32_t depth,
+                                    int32_t status);
 psc_status psc_host_mask_row(const psc_handle* h, int32_t mask_id, uint32_t* h_row);
 
 /* Host-side lexer+parser step of one configuration (tests and prefix set-up

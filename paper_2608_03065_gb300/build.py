@@ -13,7 +13,7 @@ BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libpsc_gb300.so")
 INCLUDE = os.path.join(os.path.dirname(HERE), "include")
 
-CXX_SOURCES = ["grammar.cpp", "lexer.cpp", "lalr.cpp", "classifier.cpp", "persist.cpp"]
+CXX_SOURCES = ["grammar.cpp", "lexer.cpp", "lalr.cpp", "classifier.cpp", "bottomup.cpp", "persist.cpp"]
 CU_SOURCES = ["psc_capi.cu"]
 GENCODE = "arch=compute_103a,code=sm_103a"
 

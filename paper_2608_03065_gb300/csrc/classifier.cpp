@@ -819,6 +819,7 @@ Tables compile_tables(const std::string& text, const uint8_t* vb, const int64_t*
     T.seconds_lex = t2 - t1;
     T.seconds_dfa = t3 - t2;
     T.seconds_min = t4 - t3;
+    build_bottom_up(T, opt);   // empty tables when a size limit stops it: the device walks from the top
     T.seconds_total = now() - t0;
     return T;
 }

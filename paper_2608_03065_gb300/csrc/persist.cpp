@@ -3,7 +3,8 @@
 // preprocessing overhead); here the flat tables of a compiled handle are
 // written as one binary file: a magic/version header, every table as
 // (element count, raw little-endian bytes), and a 64-bit FNV-1a checksum of
-// everything before it.  The mask rows are stored as they are held in memory:
+// everything before it (format 03: with the bottom-up classifier's tables).
+// The mask rows are stored as they are held in memory:
 // chunk ids plus the distinct 1024-token chunks (no general-purpose compression;
 // the paper uses zstd).
 #include <cstdio>
@@ -15,7 +16,7 @@
 namespace psc {
 namespace {
 
-const char MAGIC[8] = {'P', 'S', 'C', 'T', 'A', 'B', '0', '2'};
+const char MAGIC[8] = {'P', 'S', 'C', 'T', 'A', 'B', '0', '3'};
 
 struct Writer {
     FILE* f;
@@ -78,6 +79,8 @@ void fields(S& s, Tables& t) {
     vc(t.action); vc(t.go); vc(t.rule_len); vc(t.rule_lhs); vc(t.resolve);
     vc(t.dfa); vc(t.dfa_start); vc(t.dfa_mask); vc(t.mask_rows); vc(t.mask_chunks);
     vc(t.vocab_bytes); vc(t.vocab_off);
+    sc(t.bu_root); sc(t.n_bu); sc(t.n_frow);
+    vc(t.bu); vc(t.bu_slot); vc(t.bu_F); vc(t.bu_t);
 }
 
 void validate(const Tables& t) {
@@ -110,6 +113,45 @@ void validate(const Tables& t) {
     for (int32_t s : t.dfa_start) if (!state_ok(s)) bad("classifier start");
     for (int32_t m : t.dfa_mask) if (m < 0 || m >= t.n_masks) bad("classifier mask id");
     if (t.eos_id < -1 || t.eos_id >= t.V) bad("end-of-sequence id");
+    // bottom-up classifier: absent, or every block's successors are block starts
+    if (t.bu_root < 0) {
+        if (!t.bu.empty() || !t.bu_slot.empty() || !t.bu_F.empty() || !t.bu_t.empty() || t.n_bu || t.n_frow)
+            bad("bottom-up classifier");
+        return;
+    }
+    if (t.bu_slot.size() != (size_t)t.n_lr * t.n_lr || t.n_bu < 1 || t.bu_t.size() != (size_t)t.n_bu ||
+        t.n_frow < 1 || t.bu_F.size() != (size_t)t.n_frow * t.nq)
+        bad("bottom-up classifier");
+    std::vector<int> deg(t.n_lr, 0);
+    for (int a = 0; a < t.n_lr; a++)
+        for (int u = 0; u < t.n_lr; u++) {
+            int k = t.bu_slot[(size_t)a * t.n_lr + u];
+            if (k < -1 || k >= t.n_lr) bad("bottom-up slot");
+            if (k >= 0) deg[a]++;
+        }
+    for (int a = 0; a < t.n_lr; a++)   // slots of a state are 0 .. deg-1, each once
+        for (int u = 0; u < t.n_lr; u++) {
+            int k = t.bu_slot[(size_t)a * t.n_lr + u];
+            if (k >= deg[a]) bad("bottom-up slot");
+        }
+    std::vector<uint8_t> is_base(t.bu.size() + 1, 0);
+    size_t len = 0;
+    for (int32_t r = 0; r < t.n_bu; r++) {
+        if (t.bu_t[r] < 0 || t.bu_t[r] >= t.n_lr) bad("bottom-up state");
+        if (len >= t.bu.size()) bad("bottom-up blocks");
+        is_base[len] = 1;
+        len += 1 + (size_t)deg[t.bu_t[r]];
+    }
+    if (len != t.bu.size() || t.bu_root != 0 || t.bu_t[0] != 0) bad("bottom-up blocks");
+    len = 0;
+    for (int32_t r = 0; r < t.n_bu; r++) {
+        const int32_t* blk = t.bu.data() + len;
+        if (blk[0] < 0 || blk[0] >= t.n_frow) bad("bottom-up row id");
+        for (int k = 0; k < deg[t.bu_t[r]]; k++)
+            if (blk[1 + k] < 0 || (size_t)blk[1 + k] >= t.bu.size() || !is_base[blk[1 + k]]) bad("bottom-up successor");
+        len += 1 + (size_t)deg[t.bu_t[r]];
+    }
+    for (int32_t m : t.bu_F) if (m < 0 || m >= t.n_masks) bad("bottom-up mask id");
 }
 
 }  // namespace

@@ -62,6 +62,11 @@ struct DevTables {
     const uint8_t* adv;
     int adv_bytes, o_bc, o_trans, o_accept, o_ign, o_resolve, o_action, o_go, o_rlen, o_rlhs, nbc;
     int adv_packed;   // reduce entries of the compact ACTION hold (rule length << 10 | lhs) instead of the rule
+    // bottom-up classifier (bu = nullptr: not built; the root block, for the stack [0], is at 0)
+    const int32_t* bu;        // blocks [final row, next block per successor slot]
+    const int16_t* bu_slot;   // [n_lr][n_lr] slot of the LR edge t -> u, -1 none
+    const int32_t* bu_F;      // [n_frow][nq] mask ids
+    int bu_len, n_frow;
 };
 
 struct DevStates {
@@ -72,6 +77,7 @@ struct DevStates {
     int32_t* mid;
     int B, cap;
     unsigned long long* best;   // per-row greedy-choice key (nullable)
+    int32_t* rmemo;             // [B][cap] bottom-up classifier block after each stack prefix (nullable)
 };
 
 }  // namespace
@@ -81,7 +87,7 @@ struct psc_handle {
     bool host_only = true;
     int device = -1;
     DevTables d{};
-    void* blocks[16] = {};
+    void* blocks[32] = {};
     int n_blocks = 0;
     int tma_ctas[2] = {1, 1};   // resident k_step_tma CTAs per SM (bf16, f32)
 };
@@ -119,6 +125,22 @@ __device__ __forceinline__ uint32_t mask_word(const DevTables& T, int mid, int w
     return __ldg(T.mchunks + (size_t)c * 32 + (w & 31));
 }
 
+// Mask id of a configuration from the bottom-up classifier's block e for its
+// whole stack (final table row, then the lexer state's column); -1 when e is
+// not a usable block (the caller walks the stack instead).
+__device__ __forceinline__ int memo_mask(const DevTables& T, int e, int q) {
+    if (e < 0 || e >= T.bu_len) return -1;
+    int fr = __ldg(T.bu + e);
+    if (fr < 0 || fr >= T.n_frow) return -1;
+    return __ldg(T.bu_F + (size_t)fr * T.nq + q);
+}
+
+// The row's mask id from its kept bottom-up state, or -1 (not kept / not built).
+__device__ __forceinline__ int memo_classify(const DevTables& T, const DevStates& S, int b, int q, int depth) {
+    if (!S.rmemo || !T.bu) return -1;
+    return memo_mask(T, S.rmemo[(size_t)b * S.cap + depth - 1], q);
+}
+
 // Classifier walk for one row (Algorithm 2 step 3), executed by a full warp:
 // lanes load 32 stack symbols at a time (coalesced), the walk broadcasts them
 // with shuffles and follows the DFA; every lane ends with the same mask id.
@@ -129,6 +151,8 @@ __device__ int warp_classify(const DevTables& T, const DevStates& S, int b, int 
     int q = S.q[b];
     int depth = S.depth[b];
     if (q < 0 || q >= T.nq || depth < 1 || depth > S.cap) return 0;
+    int m = memo_classify(T, S, b, q, depth);
+    if (m >= 0) return m;
     int s = __ldg(T.dfa_start + q);
     if (s < 0) return -s - 1;
     const uint16_t* st = S.stack + (size_t)b * S.cap;
@@ -154,6 +178,8 @@ __device__ int thread_classify(const DevTables& T, const DevStates& S, int b) {
     int q = S.q[b];
     int depth = S.depth[b];
     if (q < 0 || q >= T.nq || depth < 1 || depth > S.cap) return 0;
+    int m = memo_classify(T, S, b, q, depth);
+    if (m >= 0) return m;
     int s = __ldg(T.dfa_start + q);
     if (s < 0) return -s - 1;
     const uint16_t* st = S.stack + (size_t)b * S.cap;
@@ -177,6 +203,7 @@ __global__ void k_state_init(DevStates S, int q0, const int32_t* rows, int n) {
     S.stack[(size_t)b * S.cap] = 0;
     S.mid[b] = 0;
     if (S.best) S.best[b] = 0ull;
+    if (S.rmemo) S.rmemo[(size_t)b * S.cap] = 0;   // the bottom-up classifier's block for [0]
 }
 
 __global__ void k_classify(DevTables T, DevStates S, int B) {
@@ -403,8 +430,9 @@ __global__ void __launch_bounds__(256) k_argmax_masked(const T* logits, int64_t 
 }
 
 // Feed one lexeme class to the parser on a row's stack: resolve the class to a
-// terminal with the current top, reduce until it is shifted.  Returns a row status.
-__device__ int feed_class(const DevTables& T, uint16_t* st, int& depth, int cap, int cls) {
+// terminal with the current top, reduce until it is shifted.  Returns a row
+// status; `low` becomes the lowest stack index written.
+__device__ int feed_class(const DevTables& T, uint16_t* st, int& depth, int cap, int cls, int& low) {
     int top = st[depth - 1];
     int t = T.resolve[(size_t)cls * T.n_lr + top];
     if (t < 0) return ROW_REJECTED;
@@ -413,6 +441,7 @@ __device__ int feed_class(const DevTables& T, uint16_t* st, int& depth, int cap,
         int kind = a & 3, val = a >> 2;
         if (kind == psc::ACT_SHIFT) {
             if (depth >= cap) return ROW_OVERFLOW;
+            low = depth < low ? depth : low;
             st[depth++] = (uint16_t)val;
             return ROW_OK;
         }
@@ -423,9 +452,32 @@ __device__ int feed_class(const DevTables& T, uint16_t* st, int& depth, int cap,
         int go = T.go[(size_t)st[depth - 1] * T.n_nts + T.rule_lhs[val]];
         if (go < 0) return ROW_REJECTED;
         if (depth >= cap) return ROW_OVERFLOW;
+        low = depth < low ? depth : low;
         st[depth++] = (uint16_t)go;
     }
     return ROW_LIMIT;
+}
+
+// Re-reads stack entries [from, depth) of one row through the bottom-up
+// classifier, keeping its block after every prefix (memo[i]: stack [0, i]);
+// returns the block of the whole stack, or -1 (unknown: the stack is then
+// walked from the top).  Entries below `from` are unchanged since they were kept.
+__device__ int memo_extend(const DevTables& T, const uint16_t* st, int32_t* memo, int from, int depth) {
+    int e;
+    if (from <= 0) {
+        e = st[0] == 0 ? 0 : -1;
+        memo[0] = e;
+        from = 1;
+    } else {
+        e = memo[from - 1];
+    }
+    for (int i = from; i < depth; i++) {
+        int t = st[i - 1], u = st[i];
+        int k = t < T.n_lr && u < T.n_lr ? T.bu_slot[(size_t)t * T.n_lr + u] : -1;
+        e = e >= 0 && k >= 0 && e + 1 + k < T.bu_len ? __ldg(T.bu + e + 1 + k) : -1;
+        memo[i] = e;
+    }
+    return e;
 }
 
 // Algorithm 2 steps 1-2 for one row per thread.
@@ -457,7 +509,7 @@ __global__ void k_advance(DevTables T, DevStates S, const int32_t* tokens, int B
                 } else if (tok == T.eos_id) {
                     status = ROW_DONE;
                 } else {
-                    int q = S.q[b], depth = S.depth[b];
+                    int q = S.q[b], depth = S.depth[b], low = 0x7FFFFFFF;
                     uint16_t* st = S.stack + (size_t)b * S.cap;
                     int64_t lo = T.vocab_off[tok], hi = T.vocab_off[tok + 1];
                     for (int64_t i = lo; i < hi && status == ROW_OK; i++) {
@@ -472,13 +524,15 @@ __global__ void k_advance(DevTables T, DevStates S, const int32_t* tokens, int B
                             status = ROW_REJECTED;
                             break;
                         }
-                        if (!T.cls_ignored[cls]) status = feed_class(T, st, depth, S.cap, cls);
+                        if (!T.cls_ignored[cls]) status = feed_class(T, st, depth, S.cap, cls, low);
                         q = T.lex_trans[(size_t)T.q0 * 256 + c];
                         if (q < 0) status = ROW_REJECTED;
                     }
                     if (status == ROW_OK) {
                         S.q[b] = q;
                         S.depth[b] = depth;
+                        if (S.rmemo && T.bu)
+                            memo_extend(T, st, S.rmemo + (size_t)b * S.cap, low < depth ? low : depth, depth);
                     }
                 }
             }
@@ -892,8 +946,8 @@ __device__ __forceinline__ bool mbar_wait0(uint32_t bar, int limit) {
 }
 
 // A row's stack seen through its window: indices in [base, base + ADV_WIN) live
-// in shared memory, the others in global memory.  `lo` tracks the lowest window
-// index written (for the write-back).
+// in shared memory, the others in global memory.  `lo` tracks the lowest index
+// written (for the write-back and the bottom-up classifier).
 struct StackView {
     uint16_t* win;
     uint16_t* st;
@@ -902,12 +956,9 @@ struct StackView {
     __device__ __forceinline__ bool in_win(int i) const { return i >= base && i < base + ADV_WIN; }
     __device__ __forceinline__ int get(int i) const { return in_win(i) ? win[i - base] : st[i]; }
     __device__ __forceinline__ void set(int i, int v) {
-        if (in_win(i)) {
-            win[i - base] = (uint16_t)v;
-            lo = i < lo ? i : lo;
-        } else {
-            st[i] = (uint16_t)v;
-        }
+        if (in_win(i)) win[i - base] = (uint16_t)v;
+        else st[i] = (uint16_t)v;
+        lo = i < lo ? i : lo;
     }
 };
 
@@ -977,6 +1028,39 @@ __device__ __forceinline__ int warp_walk(const DevTables& T, const StackView& sv
     return __ldg(T.dfa_mask + s);
 }
 
+// memo_extend by a full warp: lanes fetch the edge slots of 32 entries at a
+// time, the chain of block loads follows them (broadcast by shuffles), and each
+// lane stores the block of its own entry.  e_below = block of stack [0, from-1]
+// (ignored when from == 0).  Every lane returns the block of the whole stack.
+__device__ __forceinline__ int warp_memo_extend(const DevTables& T, const StackView& sv, int32_t* memo, int from,
+                                                int depth, int e_below, int lane) {
+    uint64_t pol;
+    asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(pol));
+    int e = e_below;
+    if (from <= 0) {
+        e = sv.get(0) == 0 ? 0 : -1;
+        if (lane == 0) memo[0] = e;
+        from = 1;
+    }
+    for (int i0 = from; i0 < depth; i0 += 32) {
+        int i = i0 + lane;
+        int k = -1;
+        if (i < depth) {
+            int t = sv.get(i - 1), u = sv.get(i);
+            k = t < T.n_lr && u < T.n_lr ? __ldg(T.bu_slot + (size_t)t * T.n_lr + u) : -1;
+        }
+        int n = depth - i0 < 32 ? depth - i0 : 32;
+        int mine = -1;
+        for (int j = 0; j < n; j++) {
+            int kj = __shfl_sync(FULL, k, j);
+            e = e >= 0 && kj >= 0 && e + 1 + kj < T.bu_len ? ld_keep(T.bu + e + 1 + kj, pol) : -1;
+            mine = lane == j ? e : mine;
+        }
+        if (i < depth) memo[i] = mine;
+    }
+    return e;
+}
+
 // Algorithm 2 steps 1-3 for one row per warp: consume the row's token (the
 // given one, or the greedy choice of the fused masking pass when from_keys),
 // then classify the new configuration into S.mid.  Everything that needs only
@@ -1007,6 +1091,8 @@ __global__ void __launch_bounds__(ADV_WARPS * 32) k_advance_warp(DevTables T, De
                  S.stack + (size_t)(active ? b : 0) * S.cap, 0x40000000, 0x7FFFFFFF};
     int tok = -1, status = ROW_OK, q = 0, depth = 0;
     bool parse = false;
+    int32_t* memo = active && S.rmemo && T.bu ? S.rmemo + (size_t)b * S.cap : nullptr;
+    int memo_top = -1, depth0 = 0;
     uint32_t mword = 0;
     uint32_t tw[8] = {0, 0, 0, 0, 0, 0, 0, 0};   // the token's bytes (tokens up to 32 bytes)
     int len = 0;
@@ -1015,6 +1101,7 @@ __global__ void __launch_bounds__(ADV_WARPS * 32) k_advance_warp(DevTables T, De
         // the loads that need nothing but the row index go first, together
         q = S.q[b];
         depth = S.depth[b];
+        depth0 = depth;
         status = S.status[b];
         int mid = use_mid ? S.mid[b] : 0;
         if (from_keys) {   // the greedy choice of the fused masking pass
@@ -1033,6 +1120,8 @@ __global__ void __launch_bounds__(ADV_WARPS * 32) k_advance_warp(DevTables T, De
         if (live) {
             sv.base = depth > ADV_KEEP ? depth - ADV_KEEP : 0;
             for (int i = lane; i < depth - sv.base; i += 32) sv.win[i] = sv.st[sv.base + i];
+            // the kept bottom-up blocks of the top 32 prefixes (lane l: stack [0, depth-1-l])
+            if (memo && depth - 1 - lane >= 0) memo_top = memo[depth - 1 - lane];
         }
         if (tok >= 0) {
             if (status == ROW_DONE) {
@@ -1041,9 +1130,11 @@ __global__ void __launch_bounds__(ADV_WARPS * 32) k_advance_warp(DevTables T, De
                 if (tok >= T.V) {
                     status = ROW_REJECTED;
                 } else {
-                    if (!use_mid) {
-                        StackView g{sv.win, sv.st, 0x40000000, 0x7FFFFFFF};   // the stack in global memory
-                        mid = depth >= 1 && depth <= S.cap ? warp_walk(T, g, q, depth, lane) : 0;
+                    if (!use_mid) {   // the kept bottom-up block, else a walk of the stack in global memory
+                        int e = __shfl_sync(FULL, memo_top, 0);
+                        mid = memo && live && q >= 0 && q < T.nq ? memo_mask(T, e, q) : -1;
+                        StackView g{sv.win, sv.st, 0x40000000, 0x7FFFFFFF};
+                        if (mid < 0) mid = depth >= 1 && depth <= S.cap ? warp_walk(T, g, q, depth, lane) : 0;
                     }
                     // the token's mask bit (in flight while the token is parsed); the row is
                     // only committed (q, depth) when it is set
@@ -1132,9 +1223,27 @@ __global__ void __launch_bounds__(ADV_WARPS * 32) k_advance_warp(DevTables T, De
     // the next masking pass's mask id (the window holds the stack top of every live
     // row; for the others sv.base still points past any stack index)
     int mid;
-    if (status == ROW_DONE) mid = 1;
-    else if (status != ROW_OK) mid = 0;
-    else mid = depth >= 1 && depth <= S.cap ? warp_walk(T, sv, q, depth, lane) : 0;
+    if (status == ROW_DONE) {
+        mid = 1;
+    } else if (status != ROW_OK) {
+        mid = 0;
+    } else if (depth < 1 || depth > S.cap || q < 0 || q >= T.nq) {
+        mid = 0;
+    } else {
+        mid = -1;
+        if (memo) {
+            // bottom-up classifier: re-read the entries from the lowest one written
+            // (none written: the stack is as kept) and look the lexer state up
+            int from = parse && sv.lo < depth ? sv.lo : depth;
+            int below = from - 1;                    // block of stack [0, below] as kept
+            int d = depth0 - 1 - below;              // its lane in the prefetched top
+            int e_below = -1;
+            if (below >= 0) e_below = d >= 0 && d < 32 ? __shfl_sync(FULL, memo_top, d) : memo[below];
+            int e = warp_memo_extend(T, sv, memo, from, depth, e_below, lane);
+            mid = memo_mask(T, e, q);
+        }
+        if (mid < 0) mid = warp_walk(T, sv, q, depth, lane);
+    }
     if (lane == 0) S.mid[b] = mid;
 }
 
@@ -1456,6 +1565,10 @@ psc_status upload(psc_handle* h, const std::vector<V>& v, const V** dst, size_t 
     void* p = nullptr;
     psc_status s = cuda_check(cudaMalloc(&p, bytes), "cudaMalloc(tables)");
     if (s != PSC_OK) return s;
+    if (h->n_blocks >= (int)(sizeof(h->blocks) / sizeof(h->blocks[0]))) {
+        cudaFree(p);
+        return fail_with(PSC_ERR_OOM, "too many device table blocks");
+    }
     h->blocks[h->n_blocks++] = p;
     if (!v.empty()) {
         s = cuda_check(cudaMemcpy(p, v.data(), v.size() * sizeof(V), cudaMemcpyHostToDevice), "cudaMemcpy(tables)");
@@ -1741,6 +1854,19 @@ psc_status upload_tables(std::unique_ptr<psc_handle>& h, bool global_tables) {
         for (int i = 0; i < h->n_blocks; i++) cudaFree(h->blocks[i]);
         return s;
     }
+    d.bu = nullptr;
+    d.bu_slot = nullptr;
+    d.bu_F = nullptr;
+    d.bu_len = d.n_frow = 0;
+    if (t.n_bu > 0) {
+        if ((s = upload(h.get(), t.bu, &d.bu)) || (s = upload(h.get(), t.bu_slot, &d.bu_slot)) ||
+            (s = upload(h.get(), t.bu_F, &d.bu_F))) {
+            for (int i = 0; i < h->n_blocks; i++) cudaFree(h->blocks[i]);
+            return s;
+        }
+        d.bu_len = (int)t.bu.size();
+        d.n_frow = t.n_frow;
+    }
     std::vector<uint8_t> blob;
     if (!global_tables) blob = build_advance_blob(t, d);
     if (!blob.empty()) {
@@ -1817,6 +1943,7 @@ psc_status psc_compile(const char* grammar, size_t grammar_len, const uint8_t* v
         if (opts->max_states > 0) o.max_states = opts->max_states;
         if (opts->max_mask_bytes > 0) o.max_mask_bytes = opts->max_mask_bytes;
         o.threads = opts->threads;
+        o.max_bottom_up_bytes = opts->max_bottom_up_bytes;
         host_only = opts->host_only != 0;
         global_tables = opts->global_tables != 0;
     }
@@ -1860,6 +1987,8 @@ psc_status psc_info(const psc_handle* h, psc_info_t* out) {
     out->states_built = t.n_dfa_states_built;
     out->compile_seconds = t.seconds_total;
     out->advance_table_bytes = h->host_only ? 0 : h->d.adv_bytes;
+    out->bottom_up_states = t.n_bu;
+    out->bottom_up_bytes = (int64_t)(t.bu.size() + t.bu_F.size()) * 4 + (int64_t)t.bu_slot.size() * 2;
     out->device_timeouts = 0;
     if (!h->host_only) {
         int v = 0;
@@ -1881,10 +2010,12 @@ psc_status psc_state_init(const psc_handle* h, int32_t B, int32_t cap, void* str
     DevStates& d = st->d;
     d.B = B;
     d.cap = cap;
-    void* p[6] = {};
-    size_t sz[6] = {sizeof(int32_t) * B, sizeof(int32_t) * B, sizeof(int32_t) * B, sizeof(uint16_t) * (size_t)B * cap,
-                    sizeof(int32_t) * B, sizeof(unsigned long long) * B};
-    for (int i = 0; i < 6; i++) {
+    // the bottom-up classifier's kept blocks only when the handle has that classifier
+    const int n_arr = h->d.bu ? 7 : 6;
+    void* p[7] = {};
+    size_t sz[7] = {sizeof(int32_t) * B, sizeof(int32_t) * B, sizeof(int32_t) * B, sizeof(uint16_t) * (size_t)B * cap,
+                    sizeof(int32_t) * B, sizeof(unsigned long long) * B, sizeof(int32_t) * (size_t)B * cap};
+    for (int i = 0; i < n_arr; i++) {
         s = cuda_check(cudaMalloc(&p[i], sz[i]), "cudaMalloc(states)");
         if (s != PSC_OK) {
             for (int j = 0; j < i; j++) cudaFree(p[j]);
@@ -1897,11 +2028,12 @@ psc_status psc_state_init(const psc_handle* h, int32_t B, int32_t cap, void* str
     d.stack = (uint16_t*)p[3];
     d.mid = (int32_t*)p[4];
     d.best = (unsigned long long*)p[5];
+    d.rmemo = (int32_t*)p[6];
     cudaStream_t cs = (cudaStream_t)stream;
     k_state_init<<<(B + 255) / 256, 256, 0, cs>>>(d, h->d.q0, nullptr, B);
     s = launch_check("k_state_init");
     if (s != PSC_OK) {
-        for (int j = 0; j < 6; j++) cudaFree(p[j]);
+        for (int j = 0; j < n_arr; j++) cudaFree(p[j]);
         return s;
     }
     *out = st.release();
@@ -1933,6 +2065,10 @@ psc_status psc_state_copy(psc_states* dst, const psc_states* src, void* stream) 
         (s = cuda_check(cudaMemcpyAsync(b.best, a.best, B * 8, cudaMemcpyDeviceToDevice, cs), "psc_state_copy")) !=
             PSC_OK)
         return s;
+    if (a.rmemo && b.rmemo &&
+        (s = cuda_check(cudaMemcpyAsync(b.rmemo, a.rmemo, B * (size_t)a.cap * 4, cudaMemcpyDeviceToDevice, cs),
+                        "psc_state_copy")) != PSC_OK)
+        return s;
     dst->gen++;
     dst->mid_gen = src->mid_gen == src->gen ? dst->gen : 0;   // the mask ids are as current as src's
     return PSC_OK;
@@ -1956,6 +2092,7 @@ void psc_state_destroy(psc_states* st) {
     cudaFree(st->d.stack);
     cudaFree(st->d.mid);
     cudaFree(st->d.best);
+    cudaFree(st->d.rmemo);
     delete st;
 }
 
@@ -2102,6 +2239,14 @@ int32_t psc_host_classify(const psc_handle* h, int32_t q, const uint16_t* h_stac
     return psc::classify_host(h->t, q, h_stack, depth, status);
 }
 
+int32_t psc_host_classify_bottom_up(const psc_handle* h, int32_t q, const uint16_t* h_stack, int32_t depth,
+                                    int32_t status) {
+    if (!h || (depth > 0 && !h_stack) || depth < 0) return -1;
+    for (int i = 0; i < depth; i++)
+        if (h_stack[i] >= h->t.n_lr) return -1;
+    return psc::classify_host_bottom_up(h->t, q, h_stack, depth, status);
+}
+
 psc_status psc_host_mask_row(const psc_handle* h, int32_t mask_id, uint32_t* h_row) {
     if (!h || !h_row || mask_id < 0 || mask_id >= h->t.n_masks) return fail_with(PSC_ERR_ARG, "psc_host_mask_row: bad arguments");
     const psc::Tables& t = h->t;
@@ -2211,6 +2356,15 @@ psc_status psc_load(const char* path, const psc_options* opts, psc_handle** out)
         return fail_with((psc_status)e.code, e.what());
     } catch (const std::bad_alloc&) {
         return fail_with(PSC_ERR_OOM, "psc_load: out of host memory");
+    }
+    if (opts && opts->max_bottom_up_bytes < 0) {   // drop the bottom-up classifier
+        psc::Tables& t = h->t;
+        t.bu.clear();
+        t.bu_slot.clear();
+        t.bu_F.clear();
+        t.bu_t.clear();
+        t.bu_root = -1;
+        t.n_bu = t.n_frow = 0;
     }
     h->host_only = opts && opts->host_only;
     if (!h->host_only) {

@@ -86,6 +86,8 @@ struct Options {
     int64_t max_states = 4000000;     // classifier states before PSC_ERR_LIMIT
     int64_t max_mask_bytes = int64_t(24) << 30;
     int threads = 0;                  // 0 = hardware concurrency
+    int64_t max_bottom_up_bytes = 0;  // construction memory of the bottom-up classifier
+                                      // (0 = 8 GiB; < 0 = not built; over the limit: not built)
 };
 
 struct Tables {
@@ -112,6 +114,14 @@ struct Tables {
     int V = 0, W = 0, n_masks = 0, nch = 0, n_chunks = 0;
     std::vector<uint32_t> mask_rows;     // [n_masks][nch] chunk ids
     std::vector<uint32_t> mask_chunks;   // [n_chunks][32]
+    // bottom-up classifier (the same classification, reading the stack from the
+    // bottom; empty when not built): blocks [F row, next block per successor slot],
+    // slot of an LR edge t -> u, final mask ids [F row][nq], LR state of each block
+    int bu_root = -1, n_bu = 0, n_frow = 0;
+    std::vector<int32_t> bu;
+    std::vector<int16_t> bu_slot;        // [n_lr][n_lr], -1: no edge
+    std::vector<int32_t> bu_F;           // [n_frow][nq]
+    std::vector<int32_t> bu_t;           // [n_bu] (host only: validation)
     // vocabulary
     std::vector<uint8_t> vocab_bytes;
     std::vector<int64_t> vocab_off;      // [V+1]
@@ -139,5 +149,12 @@ Tables load_tables(const std::string& path);
 
 // host-side walk of the flattened classifier (inspection / tests): mask id of (q, stack)
 int classify_host(const Tables& t, int q, const uint16_t* stack, int depth, int status);
+
+// Builds the bottom-up classifier tables from the forward classifier (false, and
+// empty tables, when a size limit stops it).
+bool build_bottom_up(Tables& t, const Options& opt);
+// The same classification through the bottom-up tables; -2 when they are not
+// built or the stack is not a path of the LR automaton.
+int classify_host_bottom_up(const Tables& t, int q, const uint16_t* stack, int depth, int status);
 
 }  // namespace psc

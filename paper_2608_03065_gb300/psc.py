@@ -26,7 +26,8 @@ EXPORTED = ["psc_compile", "psc_destroy", "psc_last_error", "psc_info", "psc_sta
             "psc_state_destroy", "psc_advance", "psc_fill_mask", "psc_apply_mask", "psc_fill_apply",
             "psc_argmax_masked", "psc_states_download", "psc_host_classify", "psc_host_mask_row",
             "psc_host_advance", "psc_fill_apply_noalloc", "psc_fill_apply_argmax", "psc_save", "psc_load",
-            "psc_decode_step", "psc_decode_step_mask", "psc_decode_step_advance", "psc_state_copy"]
+            "psc_decode_step", "psc_decode_step_mask", "psc_decode_step_advance", "psc_state_copy",
+            "psc_host_classify_bottom_up"]
 NOALLOC_MAX_ROWS = 16384
 
 
@@ -39,7 +40,7 @@ class PscError(RuntimeError):
 class Options(ctypes.Structure):
     _fields_ = [("max_states", ctypes.c_int64), ("max_mask_bytes", ctypes.c_int64),
                 ("threads", ctypes.c_int32), ("host_only", ctypes.c_int32),
-                ("global_tables", ctypes.c_int32)]
+                ("global_tables", ctypes.c_int32), ("max_bottom_up_bytes", ctypes.c_int64)]
 
 
 class InfoT(ctypes.Structure):
@@ -48,7 +49,8 @@ class InfoT(ctypes.Structure):
                 ("n_classifier_states", ctypes.c_int32), ("n_masks", ctypes.c_int32), ("eos_id", ctypes.c_int32),
                 ("classifier_bytes", ctypes.c_int64), ("mask_bytes", ctypes.c_int64),
                 ("states_built", ctypes.c_int64), ("compile_seconds", ctypes.c_double),
-                ("advance_table_bytes", ctypes.c_int64), ("device_timeouts", ctypes.c_int64)]
+                ("advance_table_bytes", ctypes.c_int64), ("device_timeouts", ctypes.c_int64),
+                ("bottom_up_states", ctypes.c_int64), ("bottom_up_bytes", ctypes.c_int64)]
 
 
 _lib = None
@@ -78,6 +80,7 @@ def load(path: str = LIB_PATH):
         "psc_argmax_masked": (i32, [vp, vp, i32, vp, i32, i64, i32, vp, vp]),
         "psc_states_download": (i32, [vp, vp, vp, vp, vp, vp]),
         "psc_host_classify": (i32, [vp, i32, vp, i32, i32]),
+        "psc_host_classify_bottom_up": (i32, [vp, i32, vp, i32, i32]),
         "psc_host_mask_row": (i32, [vp, i32, vp]),
         "psc_host_advance": (i32, [vp, vp, vp, vp, i32, vp, i32]),
         "psc_fill_apply_noalloc": (i32, [vp, vp, vp, vp, vp, i32, i32, vp, i32, i64, i32, vp, vp]),
@@ -152,6 +155,8 @@ class Info:
     compile_seconds: float
     advance_table_bytes: int
     device_timeouts: int
+    bottom_up_states: int
+    bottom_up_bytes: int
 
 
 class Handle:
@@ -176,6 +181,13 @@ class Handle:
     def host_classify(self, q: int, stack, status: int = ROW_OK) -> int:
         st = np.ascontiguousarray(np.asarray(stack, dtype=np.uint16))
         return load().psc_host_classify(self.ptr, q, st.ctypes.data if len(st) else None, len(st), status)
+
+    def host_classify_bottom_up(self, q: int, stack, status: int = ROW_OK) -> int:
+        """The same mask id through the bottom-up classifier (-2: not built, or
+        the stack is not a path of the LR automaton)."""
+        st = np.ascontiguousarray(np.asarray(stack, dtype=np.uint16))
+        return load().psc_host_classify_bottom_up(self.ptr, q, st.ctypes.data if len(st) else None, len(st),
+                                                  status)
 
     def host_mask_row(self, mask_id: int) -> np.ndarray:
         row = np.zeros(self.W, dtype=np.uint32)
@@ -215,8 +227,9 @@ class States:
 # ------------------------------------------------------------------- the ABI
 def psc_compile(grammar: str, vocab: list[bytes] | tuple, eos_id: int, host_only: bool = False,
                 threads: int = 0, max_states: int = 0, max_mask_bytes: int = 0,
-                global_tables: bool = False) -> Handle:
-    """vocab: list of token byte strings, or (blob uint8 array, offsets int64[V+1])."""
+                global_tables: bool = False, bottom_up: bool = True, max_bottom_up_bytes: int = 0) -> Handle:
+    """vocab: list of token byte strings, or (blob uint8 array, offsets int64[V+1]).
+    bottom_up=False builds no bottom-up classifier (every stack is walked from the top)."""
     if isinstance(vocab, tuple):
         blob, offs = vocab
         blob = np.ascontiguousarray(blob, dtype=np.uint8)
@@ -228,7 +241,8 @@ def psc_compile(grammar: str, vocab: list[bytes] | tuple, eos_id: int, host_only
     if blob.size == 0:
         blob = np.zeros(1, dtype=np.uint8)
     V = len(offs) - 1
-    opts = Options(max_states, max_mask_bytes, threads, 1 if host_only else 0, 1 if global_tables else 0)
+    opts = Options(max_states, max_mask_bytes, threads, 1 if host_only else 0, 1 if global_tables else 0,
+                   max_bottom_up_bytes if bottom_up else -1)
     g = grammar.encode("utf-8")
     out = ctypes.c_void_p()
     _check(load().psc_compile(g, len(g), blob.ctypes.data, offs.ctypes.data, V, eos_id, ctypes.byref(opts),
@@ -240,8 +254,8 @@ def psc_save(h: Handle, path: str):
     _check(load().psc_save(h.ptr, os.fsencode(path)))
 
 
-def psc_load(path: str, host_only: bool = False, global_tables: bool = False) -> Handle:
-    opts = Options(0, 0, 0, 1 if host_only else 0, 1 if global_tables else 0)
+def psc_load(path: str, host_only: bool = False, global_tables: bool = False, bottom_up: bool = True) -> Handle:
+    opts = Options(0, 0, 0, 1 if host_only else 0, 1 if global_tables else 0, 0 if bottom_up else -1)
     out = ctypes.c_void_p()
     _check(load().psc_load(os.fsencode(path), ctypes.byref(opts), ctypes.byref(out)))
     h = Handle(out.value, 0)

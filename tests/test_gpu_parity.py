@@ -535,6 +535,54 @@ def test_deep_stacks_and_long_pushes(psc, global_tables):
         assert d["depth"][r] == ocs[r].info()["depth"]
 
 
+@pytest.mark.parametrize("cfg_id,global_tables", [(4, False), (2, True)])
+def test_bottom_up_and_top_down_classification_agree(psc, cfg_id, global_tables):
+    """Decoding with the bottom-up classifier (each advance re-reads only the
+    stack entries it pushed, from the blocks kept per stack prefix) and with
+    top-down walks of the whole stack gives the same tokens, masked logits,
+    statuses and stacks, also after a batch is forked (psc_state_copy) and some
+    of its rows are reset."""
+    w = configs.load(cfg_id, batch=64)
+    hb = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id, global_tables=global_tables)
+    ht = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id, global_tables=global_tables, bottom_up=False)
+    assert hb.info().bottom_up_states > 0 and ht.info().bottom_up_states == 0
+    B, cap = w.B, 512
+    sb0, st = psc.psc_state_init(hb, B, cap), psc.psc_state_init(ht, B, cap)
+    tm = torch.from_numpy(w.token_matrix()).cuda()
+    for j in range(tm.shape[1]):
+        psc.psc_advance(hb, sb0, tm[:, j].contiguous())
+        psc.psc_advance(ht, st, tm[:, j].contiguous())
+    sb = psc.psc_state_init(hb, B, cap)
+    psc.psc_state_copy(sb, sb0)
+    rows = torch.tensor([1, 5, B - 1], dtype=torch.int32, device="cuda")
+    psc.psc_state_reset(sb, rows)
+    psc.psc_state_reset(st, rows)
+    tb, tt = (torch.empty(B, dtype=torch.int32, device="cuda") for _ in range(2))
+    sbs, sts = (torch.empty(B, dtype=torch.int32, device="cuda") for _ in range(2))
+    mb, mt = (torch.zeros(B, hb.W, dtype=torch.int32, device="cuda") for _ in range(2))
+    for step in range(8):
+        logits = w.logits(90 + step)
+        xb, xt = logits.cuda(), logits.cuda()
+        psc.psc_decode_step(hb, sb, xb, tb, mb, sbs)
+        psc.psc_decode_step(ht, st, xt, tt, mt, sts)
+        torch.cuda.synchronize()
+        np.testing.assert_array_equal(mb.cpu().numpy(), mt.cpu().numpy(), err_msg=f"step {step}")
+        np.testing.assert_array_equal(tb.cpu().numpy(), tt.cpu().numpy(), err_msg=f"step {step}")
+        np.testing.assert_array_equal(sbs.cpu().numpy(), sts.cpu().numpy(), err_msg=f"step {step}")
+        np.testing.assert_array_equal(raw_bits(xb), raw_bits(xt))
+    psc.psc_fill_mask(hb, sb, mb)
+    psc.psc_fill_mask(ht, st, mt)
+    np.testing.assert_array_equal(mb.cpu().numpy(), mt.cpu().numpy())
+    db, dt = psc.psc_states_download(sb), psc.psc_states_download(st)
+    for k in ("q", "depth", "status"):
+        np.testing.assert_array_equal(db[k], dt[k])
+    for r in range(B):
+        np.testing.assert_array_equal(db["stack"][r, :db["depth"][r]], dt["stack"][r, :dt["depth"][r]])
+        if db["status"][r] == psc.ROW_OK:   # the host's bottom-up tables agree on the final stacks
+            stack = db["stack"][r, :db["depth"][r]]
+            assert hb.host_classify_bottom_up(int(db["q"][r]), stack) == ht.host_classify(int(db["q"][r]), stack)
+
+
 def test_state_reset_rows(psc):
     c = case(psc, 2)
     rows = torch.tensor([0, 3, 5], dtype=torch.int32, device="cuda")

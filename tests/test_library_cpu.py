@@ -49,10 +49,20 @@ def _host_mask(h, c):
     return h.host_mask_row(h.host_classify(c["q"], c["stack"], c["status"]))
 
 
+_handles = {}
+
+
+def _handle(psc, cfg_id, batch):
+    """Host-only handle of a workload (compiled once per test session)."""
+    if cfg_id not in _handles:
+        w = configs.load(cfg_id, batch=batch)
+        _handles[cfg_id] = (w, psc.psc_compile(w.grammar_text, w.vocab, w.eos_id, host_only=True))
+    return _handles[cfg_id]
+
+
 @pytest.mark.parametrize("cfg_id,batch", [(1, 8), (2, 24), (3, 6)])
 def test_host_tables_match_oracle(psc, cfg_id, batch):
-    w = configs.load(cfg_id, batch=batch)
-    h = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id, host_only=True)
+    w, h = _handle(psc, cfg_id, batch)
     o = Oracle(w.grammar_text)
     voc = Vocab.from_list(w.vocab, w.eos_id)
     cfgs, ocs = [], []
@@ -65,6 +75,42 @@ def test_host_tables_match_oracle(psc, cfg_id, batch):
     for b, c in enumerate(cfgs):
         assert c["status"] == psc.ROW_OK
         np.testing.assert_array_equal(_host_mask(h, c), om[b], err_msg=f"row {b}")
+
+
+@pytest.mark.parametrize("cfg_id,batch", [(1, 8), (2, 24), (3, 6)])
+def test_bottom_up_classifier_agrees_with_the_walk(psc, cfg_id, batch):
+    """The bottom-up classifier (the classifier DFA reversed, reading the stack
+    from the bottom; it exists by the regularity theorem of Section 3.5) gives
+    the top-down walk's mask id at every token of every prefix, and refuses
+    stacks that no parser builds."""
+    w, h = _handle(psc, cfg_id, batch)
+    assert h.info().bottom_up_states > 0
+    n = 0
+    for ids in w.prefix_ids:
+        c = h.host_initial()
+        for v in ids:
+            c = h.host_advance(c, v)
+            assert c["status"] == psc.ROW_OK
+            want = h.host_classify(c["q"], c["stack"])
+            assert h.host_classify_bottom_up(c["q"], c["stack"]) == want, (ids, c)
+            n += 1
+        for st in (psc.ROW_DONE, psc.ROW_REJECTED):   # statuses decide before any table
+            assert h.host_classify_bottom_up(c["q"], c["stack"], st) == h.host_classify(c["q"], c["stack"], st)
+    assert n > 50
+    assert h.host_classify_bottom_up(0, [0, 0]) == -2        # nothing enters the LR start state
+    assert h.host_classify_bottom_up(0, [1]) == -2           # every stack starts with state 0
+
+
+def test_bottom_up_classifier_limits(psc):
+    """Not built on request or over its memory limit (compilation still succeeds;
+    the device then walks stacks from the top)."""
+    w = configs.load(2, batch=2)
+    for kw in ({"bottom_up": False}, {"max_bottom_up_bytes": 4096}):
+        h = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id, host_only=True, **kw)
+        assert h.info().bottom_up_states == 0 and h.info().bottom_up_bytes == 0
+        c = _host_cfg(h, w.prefix_ids[0])
+        assert h.host_classify_bottom_up(c["q"], c["stack"]) == -2
+        assert h.host_classify(c["q"], c["stack"]) >= 0
 
 
 def test_host_tables_deep_parentheses(psc):
@@ -80,9 +126,11 @@ def test_host_tables_deep_parentheses(psc):
         o.advance(oc, b"(")
         if d % 37 == 0 or d == 199:
             np.testing.assert_array_equal(_host_mask(h, c), o.masks([oc], voc)[0])
+        assert h.host_classify_bottom_up(c["q"], c["stack"]) == h.host_classify(c["q"], c["stack"])
     for d in range(200):
         c = h.host_advance(c, 1, cap=512)
         o.advance(oc, b")")
+        assert h.host_classify_bottom_up(c["q"], c["stack"]) == h.host_classify(c["q"], c["stack"])
     np.testing.assert_array_equal(_host_mask(h, c), o.masks([oc], voc)[0])
     assert (_host_mask(h, c)[0] >> 7) & 1   # end of sequence allowed at depth 0
 

@@ -26,8 +26,11 @@ def test_round_trip_gives_identical_masks(psc, tmp_path):
     h2 = psc.psc_load(path, host_only=True)
     i1, i2 = h.info(), h2.info()
     for f in ("V", "W", "n_lexer_states", "n_parser_states", "n_classifier_states", "n_masks", "eos_id",
-              "classifier_bytes", "mask_bytes"):
+              "classifier_bytes", "mask_bytes", "bottom_up_states", "bottom_up_bytes"):
         assert getattr(i1, f) == getattr(i2, f), f
+    assert i2.bottom_up_states > 0
+    h3 = psc.psc_load(path, host_only=True, bottom_up=False)   # loaded without the bottom-up classifier
+    assert h3.info().bottom_up_states == 0
     for ids in w.prefix_ids:
         c1, c2 = h.host_initial(), h2.host_initial()
         for v in ids:
@@ -36,6 +39,8 @@ def test_round_trip_gives_identical_masks(psc, tmp_path):
         m1 = h.host_mask_row(h.host_classify(c1["q"], c1["stack"], c1["status"]))
         m2 = h2.host_mask_row(h2.host_classify(c2["q"], c2["stack"], c2["status"]))
         np.testing.assert_array_equal(m1, m2)
+        assert h2.host_classify_bottom_up(c2["q"], c2["stack"]) == h.host_classify(c1["q"], c1["stack"])
+        assert h3.host_classify_bottom_up(c2["q"], c2["stack"]) == -2
 
 
 def test_corrupt_and_truncated_files_are_refused(psc, tmp_path):
@@ -53,3 +58,27 @@ def test_corrupt_and_truncated_files_are_refused(psc, tmp_path):
         with pytest.raises(psc.PscError) as e:
             psc.psc_load(path + suffix, host_only=True)
         assert e.value.code == 8, suffix
+
+
+def _fnv1a64(data: bytes) -> int:
+    h = 1469598103934665603
+    for b in data:
+        h = ((h ^ b) * 1099511628211) & 0xFFFFFFFFFFFFFFFF
+    return h
+
+
+def test_inconsistent_bottom_up_tables_are_refused(psc, tmp_path):
+    """A file whose checksum is right but whose bottom-up classifier names an LR
+    state out of range (the last table of the file) fails validation."""
+    w = configs.load(1, batch=2)
+    h = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id, host_only=True)
+    path = str(tmp_path / "a.psc")
+    psc.psc_save(h, path)
+    data = bytearray(open(path, "rb").read())
+    body = data[:-8]
+    body[-4:] = (0x7FFF0000).to_bytes(4, "little")      # LR state of the last bottom-up block
+    bad = bytes(body) + _fnv1a64(bytes(body)).to_bytes(8, "little")
+    open(path + ".bad", "wb").write(bad)
+    with pytest.raises(psc.PscError) as e:
+        psc.psc_load(path + ".bad", host_only=True)
+    assert e.value.code == 8 and "bottom-up" in str(e.value)
