@@ -963,10 +963,12 @@ struct StackView {
 };
 
 // Feed one lexeme class to the parser: resolve it to a terminal with the
-// current top (contextual lexing), reduce until it is shifted.  Returns a row status.
+// current top (contextual lexing), reduce until it is shifted.  Returns a row
+// status.  `top` and `below` hold the two topmost entries in registers: a
+// reduction of one symbol (the chains of unit rules) uncovers `below`, so it
+// reads no stack entry.
 __device__ __forceinline__ int feed_class_win(const uint8_t* sm, const DevTables& T, StackView& sv, int& depth,
-                                              int& top, int cap,
-                              int cls) {
+                                              int& top, int& below, int cap, int cls) {
     const int16_t* resolve = reinterpret_cast<const int16_t*>(sm + T.o_resolve);
     const int16_t* action = reinterpret_cast<const int16_t*>(sm + T.o_action);
     const int16_t* go = reinterpret_cast<const int16_t*>(sm + T.o_go);
@@ -980,6 +982,7 @@ __device__ __forceinline__ int feed_class_win(const uint8_t* sm, const DevTables
         if (kind == psc::ACT_SHIFT) {
             if (depth >= cap) return ROW_OVERFLOW;
             sv.set(depth++, val);
+            below = top;
             top = val;
             return ROW_OK;
         }
@@ -988,11 +991,14 @@ __device__ __forceinline__ int feed_class_win(const uint8_t* sm, const DevTables
         int lhs = T.adv_packed ? val & 1023 : rlhs[val];
         if (depth - k < 1) return ROW_REJECTED;
         depth -= k;
-        int under = k ? sv.get(depth - 1) : top;
+        // the entry the reduction uncovers: the top itself (k = 0), the one below it
+        // (k = 1), else read from the stack
+        int under = k == 0 ? top : k == 1 ? below : sv.get(depth - 1);
         int g = go[under * T.n_nts + lhs];
         if (g < 0) return ROW_REJECTED;
         if (depth >= cap) return ROW_OVERFLOW;
         sv.set(depth++, g);
+        below = under;
         top = g;
     }
     return ROW_LIMIT;
@@ -1176,6 +1182,7 @@ __global__ void __launch_bounds__(ADV_WARPS * 32) k_advance_warp(DevTables T, De
         int nq = q, nd = depth;
         if (lane == 0) {
             int top = sv.win[depth - 1 - sv.base];
+            int below = depth >= 2 ? sv.get(depth - 2) : 0;
             for (int i = 0; i < len && status == ROW_OK; i++) {
                 uint32_t wsel = tw[0];   // tw[i >> 2] by selects (registers, not local memory)
 #pragma unroll
@@ -1192,7 +1199,7 @@ __global__ void __launch_bounds__(ADV_WARPS * 32) k_advance_warp(DevTables T, De
                     status = ROW_REJECTED;
                     break;
                 }
-                if (!ign[cls]) status = feed_class_win(sm, T, sv, nd, top, S.cap, cls);
+                if (!ign[cls]) status = feed_class_win(sm, T, sv, nd, top, below, S.cap, cls);
                 nq = trans[T.q0 * T.nbc + c];
                 if (nq < 0) status = ROW_REJECTED;
             }
