@@ -101,6 +101,29 @@ def test_bottom_up_classifier_agrees_with_the_walk(psc, cfg_id, batch):
     assert h.host_classify_bottom_up(0, [1]) == -2           # every stack starts with state 0
 
 
+@pytest.mark.parametrize("cfg_id,batch", [(1, 8), (2, 24)])
+def test_host_advance_tokenwise_equals_bytewise(psc, cfg_id, batch):
+    """The compiled lexer and parser tables keep the state a function of the bytes:
+    advancing by the prefix's tokens or by the single-byte tokens of its bytes
+    gives the same lexer state, stack and mask id (prefixes whose bytes all have
+    single-byte tokens)."""
+    w, h = _handle(psc, cfg_id, batch)
+    single = {t[0]: i for i, t in enumerate(w.vocab) if len(t) == 1}
+    n = 0
+    for ids in w.prefix_ids:
+        if not all(b in single for v in ids for b in w.vocab[v]):
+            continue
+        a, b = h.host_initial(), h.host_initial()
+        for v in ids:
+            a = h.host_advance(a, v)
+            for byte in w.vocab[v]:
+                b = h.host_advance(b, single[byte])
+            assert a == b
+        assert h.host_classify(a["q"], a["stack"]) == h.host_classify(b["q"], b["stack"])
+        n += 1
+    assert n >= 4
+
+
 def test_bottom_up_classifier_limits(psc):
     """Not built on request or over its memory limit (compilation still succeeds;
     the device then walks stacks from the top)."""

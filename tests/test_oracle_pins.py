@@ -309,6 +309,31 @@ def test_invariants_on_workloads(cfg_id):
     assert np.array_equal(m2, m[perm])                 # rows are independent
 
 
+@pytest.mark.parametrize("cfg_id", [1, 2, 3])
+def test_tokenwise_equals_bytewise(cfg_id):
+    """The configuration (q, alpha) is a function of the bytes consumed (Section
+    3.2): a prefix advanced token by token and byte by byte reaches the same
+    status, pending lexeme, stack and mask (the lexer looks one byte ahead and
+    never backtracks, so where a token boundary falls changes nothing)."""
+    w = configs.load(cfg_id, batch=8)
+    o = Oracle(w.grammar_text)
+    voc = Vocab.from_list(w.vocab, w.eos_id)
+    tokwise, bytewise = [], []
+    for ids in w.prefix_ids:
+        a, b = o.initial(), o.initial()
+        for k, v in enumerate(ids):
+            t = w.vocab[v]
+            assert o.advance(a, t) == ST_OK
+            for byte in t:
+                assert o.advance(b, bytes([byte])) == ST_OK
+            if k % 5 == 0:
+                assert a.info() == b.info()
+        assert a.info() == b.info()
+        tokwise.append(a)
+        bytewise.append(b)
+    np.testing.assert_array_equal(o.masks(tokwise, voc), o.masks(bytewise, voc))
+
+
 def test_eos_only_after_complete_sentence():
     o = Oracle(grammars.json_grammar().text())
     voc = Vocab.from_list([b"{", b"}", b"1", b" "] + [b""], eos_id=4)
