@@ -602,9 +602,13 @@ def main():
     if world == 1 and not args.no_cpu_baseline:
         threads = os.cpu_count() or 1
         rate, rows, secs = oracle_rate(w, 10.0, threads)
+        rate1, rows1, secs1 = oracle_rate(w, 3.0, 1)
         cpu = {"value": rate, "unit": UNIT, "cores": threads, "kind": "oracle",
                "sample": f"oracle masks of the first {rows} of {w.B} rows x all {V} tokens "
-                         f"({secs:.1f} s wall on {threads} threads), scaled to one {w.B}-row step"}
+                         f"({secs:.1f} s wall on {threads} threads), scaled to one {w.B}-row step",
+               "us_per_row": secs / rows * 1e6,
+               "single_thread": {"value": rate1, "unit": UNIT, "cores": 1, "us_per_row": secs1 / rows1 * 1e6,
+                                 "sample": f"the first {rows1} rows ({secs1:.1f} s wall on 1 thread)"}}
 
     out = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K, "warmup": Wm,
