@@ -819,7 +819,15 @@ Tables compile_tables(const std::string& text, const uint8_t* vb, const int64_t*
     T.seconds_lex = t2 - t1;
     T.seconds_dfa = t3 - t2;
     T.seconds_min = t4 - t3;
-    build_bottom_up(T, opt);   // empty tables when a size limit stops it: the device walks from the top
+    // optional: empty tables when a size limit or the host's memory stops it (the device
+    // then walks stacks from the top)
+    try {
+        build_bottom_up(T, opt);
+    } catch (const std::bad_alloc&) {
+        Options off = opt;
+        off.max_bottom_up_bytes = -1;
+        build_bottom_up(T, off);   // clears the partial tables
+    }
     T.seconds_total = now() - t0;
     return T;
 }
