@@ -124,6 +124,39 @@ def test_host_advance_tokenwise_equals_bytewise(psc, cfg_id, batch):
     assert n >= 4
 
 
+def test_bottom_up_classifier_c_like_random_walks(psc):
+    """The C-like grammar (150 rules, 15 precedence levels, contextual lexer) with a
+    4,000-token slice of its vocabulary: along random decodes that favour opening
+    brackets, the bottom-up classifier gives the walk's mask id at every step."""
+    w = configs.load(4, batch=1)
+    singles = [bytes([b]) for b in list(range(0x20, 0x7F)) + [9, 10, 13]]
+    vocab = sorted(set(singles) | {t for t in w.vocab[:4000] if t}) + [b""]
+    eos = len(vocab) - 1
+    h = psc.psc_compile(w.grammar_text, vocab, eos, host_only=True)
+    assert h.info().bottom_up_states > 0
+    opens = np.array([t[:1] in (b"(", b"{", b"[") for t in vocab])
+    rng = np.random.default_rng(3)
+    n = deepest = 0
+    for _ in range(12):
+        c = h.host_initial()
+        for _ in range(200):
+            mid = h.host_classify(c["q"], c["stack"])
+            assert h.host_classify_bottom_up(c["q"], c["stack"]) == mid
+            n += 1
+            bits = np.unpackbits(h.host_mask_row(mid).view(np.uint8), bitorder="little")[:len(vocab)].astype(bool)
+            bits[eos] = False
+            allowed = np.nonzero(bits)[0]
+            if len(allowed) == 0:
+                break
+            deep = allowed[opens[allowed]]
+            v = int(rng.choice(deep)) if len(deep) and rng.random() < 0.7 else int(rng.choice(allowed))
+            c = h.host_advance(c, v, cap=4096)
+            deepest = max(deepest, len(c["stack"]))
+            if c["status"] != psc.ROW_OK:
+                break
+    assert n > 1000 and deepest > 16
+
+
 def test_bottom_up_classifier_limits(psc):
     """Not built on request or over its memory limit (compilation still succeeds;
     the device then walks stacks from the top)."""
