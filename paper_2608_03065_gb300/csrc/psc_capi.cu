@@ -2270,6 +2270,9 @@ psc_status psc_host_advance(const psc_handle* h, int32_t* q, uint16_t* h_stack, 
     if (!h || !q || !h_stack || !depth || !status || cap < 2 || *depth < 1 || *depth > cap)
         return fail_with(PSC_ERR_ARG, "psc_host_advance: bad arguments");
     const psc::Tables& T = h->t;
+    if (*q < 0 || *q >= T.nq) return fail_with(PSC_ERR_ARG, "psc_host_advance: lexer state out of range");
+    for (int i = 0; i < *depth; i++)
+        if (h_stack[i] >= T.n_lr) return fail_with(PSC_ERR_ARG, "psc_host_advance: stack entry out of range");
     if (tok < 0) return PSC_OK;
     int st = *status;
     if (st == ROW_DONE) {

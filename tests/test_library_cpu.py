@@ -237,6 +237,26 @@ def test_state_limit(psc):
     assert e.value.code == 5
 
 
+def test_host_calls_check_their_arguments(psc):
+    """Host inspection calls refuse out-of-range lexer states, stack entries and
+    mask ids instead of reading past their tables."""
+    w, h = _handle(psc, 1, 8)
+    n_lr = h.info().n_parser_states
+    assert h.host_classify(0, [0, n_lr]) == -1
+    assert h.host_classify_bottom_up(0, [0, n_lr]) == -1
+    with pytest.raises(psc.PscError) as e:
+        h.host_mask_row(h.info().n_masks)
+    assert e.value.code == 1
+    for bad in ({"q": h.info().n_lexer_states, "stack": [0], "status": psc.ROW_OK},
+                {"q": 0, "stack": [0, n_lr + 3], "status": psc.ROW_OK},
+                {"q": 0, "stack": [], "status": psc.ROW_OK}):
+        with pytest.raises(psc.PscError) as e:
+            h.host_advance(bad, 0)
+        assert e.value.code == 1, bad
+    c = h.host_advance(h.host_initial(), -1)          # a negative token leaves the row as it is
+    assert c == h.host_initial()
+
+
 def test_device_calls_refuse_host_only_handle(psc):
     h = psc.psc_compile(grammars.arithmetic().text(), [b"1", b""], 1, host_only=True)
     with pytest.raises(psc.PscError) as e:
