@@ -169,6 +169,33 @@ def test_bottom_up_classifier_limits(psc):
         assert h.host_classify(c["q"], c["stack"]) >= 0
 
 
+@pytest.mark.parametrize("fixture", ["arith_micro_masks.txt", "json_micro_masks.txt"])
+def test_host_tables_match_golden_masks(psc, fixture):
+    """The compiled tables give the hand-enumerated masks of the golden fixtures."""
+    from workloads.sample import TrieTokenizer
+    from .test_oracle_pins import JSON_MICRO, MICRO
+    if fixture.startswith("arith"):
+        text, vocab = grammars.arithmetic().text(), MICRO
+    else:
+        text, vocab = grammars.json_grammar().text(), JSON_MICRO
+    eos = len(vocab) - 1
+    h = psc.psc_compile(text, vocab, eos, host_only=True)
+    tok = TrieTokenizer(vocab)
+    n = 0
+    with open(os.path.join(ROOT, "tests", "golden", fixture)) as f:
+        for line in f:
+            if not line.strip() or line.startswith("#"):
+                continue
+            m = re.match(r'"(.*)"\s+([\d,]+)$', line.strip())
+            prefix, allowed = m.group(1).encode(), {int(x) for x in m.group(2).split(",")}
+            c = _host_cfg(h, tok.encode(prefix) if prefix else [])
+            assert c["status"] == psc.ROW_OK
+            bits = np.unpackbits(_host_mask(h, c).view(np.uint8), bitorder="little")[:len(vocab)]
+            assert set(np.nonzero(bits)[0].tolist()) == allowed, prefix
+            n += 1
+    assert n >= 7
+
+
 def test_host_tables_deep_parentheses(psc):
     """Balanced parentheses to depth 200: the classifier walk reads deep stacks."""
     g = 'start: s\ns: | s "(" s ")"\n'

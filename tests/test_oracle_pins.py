@@ -1,6 +1,6 @@
 """Pins for the CPU oracle: it is checked against things other than itself.
 
-* hand-enumerated masks (tests/golden/arith_micro_masks.txt);
+* hand-enumerated masks (tests/golden/arith_micro_masks.txt, json_micro_masks.txt);
 * closed forms: balanced parentheses, a single literal, any byte string;
 * Eq. (1) by brute force: search for completions y with x v y in the language;
 * an independent parser: Python lexer + Earley recognizer vs the C lexer + LR(1);
@@ -60,6 +60,29 @@ def test_golden_hand_enumerated_masks():
             assert o.mask_set(cf, voc) == allowed, prefix
             n += 1
     assert n == 7
+
+
+JSON_MICRO = [b"{", b"}", b'"a"', b'"', b":", b"1", b"0", b".5", b"-", b"e", b"tr", b"true", b",", b" ", b"\\",
+              b"]", b"[", b'"a":', b""]
+
+
+def test_golden_json_micro_masks():
+    """Hand-enumerated masks on the JSON grammar: number lexing with one byte of
+    lookahead, string escapes, ignored whitespace, the end-of-sequence rule."""
+    o = Oracle(grammars.json_grammar().text())
+    voc = Vocab.from_list(JSON_MICRO, eos_id=18)
+    n = 0
+    with open(os.path.join(HERE, "golden", "json_micro_masks.txt")) as f:
+        for line in f:
+            if not line.strip() or line.startswith("#"):
+                continue
+            m = re.match(r'"(.*)"\s+([\d,]+)$', line.strip())
+            prefix, allowed = m.group(1).encode(), {int(x) for x in m.group(2).split(",")}
+            cf, st = _cfg(o, voc, prefix)
+            assert st == ST_OK, prefix
+            assert o.mask_set(cf, voc) == allowed, (prefix, sorted(o.mask_set(cf, voc)))
+            n += 1
+    assert n == 13
 
 
 # -------------------------------------------------------------- closed forms
