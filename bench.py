@@ -223,15 +223,41 @@ def config_block(w, n):
                       "copy before each sequence, inside the timed region); fresh logits every step"}
 
 
+def code_only(src: str) -> str:
+    """C/C++/CUDA source without its comments and blank lines (string and
+    character literals kept as they are)."""
+    out, i, n = [], 0, len(src)
+    while i < n:
+        c = src[i]
+        if c in "\"'":
+            j = i + 1
+            while j < n and src[j] != c:
+                j += 2 if src[j] == "\\" else 1
+            out.append(src[i:j + 1])
+            i = j + 1
+        elif src.startswith("//", i):
+            j = src.find("\n", i)
+            i = n if j < 0 else j
+        elif src.startswith("/*", i):
+            j = src.find("*/", i + 2)
+            i = n if j < 0 else j + 2
+            out.append(" ")
+        else:
+            out.append(c)
+            i += 1
+    return "\n".join(line.rstrip() for line in "".join(out).splitlines() if line.strip())
+
+
 def device_source_hash() -> str:
     """sha256 of the device code of the library: psc_capi.cu up to its host glue
-    (and the headers it includes), so host-only edits keep the recorded traffic."""
+    and the headers it includes, comments left out, so host-only and comment-only
+    edits keep the recorded traffic."""
     csrc = os.path.join(ROOT, "paper_2608_03065_gb300", "csrc")
-    src = open(os.path.join(csrc, "psc_capi.cu"), "rb").read()
-    cut = src.find(b"// ----------------------------------------------------------------- host glue")
-    h = hashlib.sha256(src[:cut] if cut > 0 else src)
-    h.update(open(os.path.join(csrc, "psc_internal.h"), "rb").read())
-    h.update(open(os.path.join(ROOT, "include", "psc.h"), "rb").read())
+    src = open(os.path.join(csrc, "psc_capi.cu"), encoding="utf-8").read()
+    cut = src.find("// ----------------------------------------------------------------- host glue")
+    h = hashlib.sha256(code_only(src[:cut] if cut > 0 else src).encode())
+    for path in (os.path.join(csrc, "psc_internal.h"), os.path.join(ROOT, "include", "psc.h")):
+        h.update(code_only(open(path, encoding="utf-8").read()).encode())
     return h.hexdigest()
 
 

@@ -602,11 +602,14 @@ Tables compile_tables(const std::string& text, const uint8_t* vb, const int64_t*
                 // move this part's masks into the global pool
                 int nm = (int)(B.rows.size() / W);
                 std::vector<int32_t> gid(nm);
+                std::vector<uint64_t> row_hash(nm);   // hashed before taking the pool's lock
+                for (int m = 0; m < nm; m++)
+                    row_hash[m] = hash_span((const int32_t*)B.rows.data() + (size_t)m * W, W, 99);
                 {
                     std::lock_guard<std::mutex> lk(pool_mu);
                     for (int m = 0; m < nm; m++) {
                         const uint32_t* r = B.rows.data() + (size_t)m * W;
-                        uint64_t h = hash_span((const int32_t*)r, W, 99);
+                        uint64_t h = row_hash[m];
                         int32_t found = -1;
                         auto range = gindex.equal_range(h);
                         for (auto it = range.first; it != range.second; ++it)
