@@ -3,8 +3,10 @@
 // Online step of the paper (Algorithm 2), per decoding step and batch row:
 //   steps 1-2  incremental lexing and LR parsing of the sampled token on the
 //              row's device-resident stack                      -> k_advance_warp
-//   step 3     one pass of the classifier DFA over (q, stack from the top),
-//              O(|stack|), stopping at absorbing states          -> k_advance_warp / k_classify
+//   step 3     the classifier DFA over (q, stack from the top), O(|stack|),
+//              stopping at absorbing states; kept incremental by the bottom-up
+//              classifier (its state per stack prefix, so a step re-reads only
+//              the entries it changed, then one lookup by q)    -> k_advance_warp / k_classify
 //   step 4     the precomputed mask of the reached state         -> k_step_tma / k_fill / k_apply_rows
 // plus applying the mask to the logits and greedy sampling over the allowed
 // tokens (left to the serving engine in the paper).
@@ -13,7 +15,11 @@
 //   dfa      int32 [S][n_lr]      next classifier state, or -(mask+1) when absorbing
 //   mrows    uint32 [n_masks][nch] mask rows as ids of 1024-token chunks (nch = ceil(W / 32))
 //   mchunks  uint32 [n_chunks][32] the distinct chunks (words past W zero)
+//   bu       int32 [...]          bottom-up classifier blocks [final row, next block per edge slot]
+//   bu_slot  int16 [n_lr][n_lr]   slot of the LR edge t -> u among t's successors, -1 none
+//   bu_F     int32 [n_frow][nq]   mask id per final row and lexer state
 //   stacks   uint16 [B][cap]      parser stacks, bottom first; depth[b] entries used
+//   rmemo    int32 [B][cap]       bottom-up block of stack prefix [0, i] of every row
 //   logits   [B][row_stride]      bf16 or f32, caller-owned, masked in place
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -141,9 +147,10 @@ __device__ __forceinline__ int memo_classify(const DevTables& T, const DevStates
     return memo_mask(T, S.rmemo[(size_t)b * S.cap + depth - 1], q);
 }
 
-// Classifier walk for one row (Algorithm 2 step 3), executed by a full warp:
-// lanes load 32 stack symbols at a time (coalesced), the walk broadcasts them
-// with shuffles and follows the DFA; every lane ends with the same mask id.
+// Classification of one row (Algorithm 2 step 3) by a full warp: from the kept
+// bottom-up block when there is one, else the walk of the classifier DFA: lanes
+// load 32 stack symbols at a time (coalesced), the walk broadcasts them with
+// shuffles and follows the DFA; every lane ends with the same mask id.
 __device__ int warp_classify(const DevTables& T, const DevStates& S, int b, int lane) {
     int status = S.status[b];
     if (status == ROW_DONE) return 1;
@@ -170,7 +177,7 @@ __device__ int warp_classify(const DevTables& T, const DevStates& S, int b, int 
     return __ldg(T.dfa_mask + s);
 }
 
-// the same walk by one thread
+// the same classification by one thread
 __device__ int thread_classify(const DevTables& T, const DevStates& S, int b) {
     int status = S.status[b];
     if (status == ROW_DONE) return 1;
@@ -912,8 +919,9 @@ __global__ void k_finalize_tokens(unsigned long long* __restrict__ best_key, int
 // classes for the lexer) are staged in shared memory by one bulk copy per CTA,
 // and the top ADV_KEEP entries of the row's stack are copied into a per-warp
 // window, so the parser's dependent reads are shared-memory reads.  After the
-// token is consumed the warp walks the classifier for the new configuration
-// (Algorithm 2 step 3) and stores the row's mask id for the next masking pass.
+// token is consumed the warp classifies the new configuration (Algorithm 2 step
+// 3: the bottom-up classifier from the lowest stack entry written, or a walk when
+// it is not built) and stores the row's mask id for the next masking pass.
 constexpr int ADV_WARPS = 8;     // rows per CTA
 constexpr int ADV_WIN = 256;     // stack entries held per row
 constexpr int ADV_KEEP = 192;    // entries copied in (the rest is room for pushes)
@@ -1322,8 +1330,8 @@ struct TmaShape {
 // segment of `seg` <= TMA_SEG chunks).  Warp 0 (producer) fetches each item's mask words
 // one item ahead, then for every ring stage copies the stage's chunks that hold
 // an allowed position (runs of neighbouring chunks in one copy; chunks with
-// nothing allowed are not read); warp 1 walks the classifier for the CTA's
-// upcoming rows; consumer warp c takes chunk c of every stage, writes -inf where
+// nothing allowed are not read); warp 1 reads (or, when they are not current,
+// computes) the mask ids of the CTA's upcoming rows; consumer warp c takes chunk c of every stage, writes -inf where
 // masked and folds allowed values into the row's greedy key.
 // Requires 16-byte aligned rows; rows' mask rows padded to whole chunks.
 template <typename T>
@@ -1450,7 +1458,7 @@ __global__ void __launch_bounds__(TMA_WARPS * 32, 3) k_step_tma(T* logits, int64
     } else if (warp == 1) {
         // ------------------------------------------------------------ walker
         // lanes 0..TMA_MIDS-1 each classify one of the next TMA_MIDS items' rows, so
-        // the dependent table loads of those walks overlap
+        // the dependent table loads of those classifications overlap
         int i = 0;
         for (long it = blockIdx.x; it < items && !failed; it += (long)gridDim.x * TMA_MIDS, i += TMA_MIDS) {
             if (i >= TMA_MIDS && !__shfl_sync(FULL, (int)mbar_wait(mide0 + 8 * (TMA_MIDS - 1),
