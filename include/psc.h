@@ -12,7 +12,9 @@
  * every classifier state; the online step (Algorithm 2) walks each sequence's
  * stack once through that DFA and returns the precomputed mask.  Here the
  * online step runs in CUDA kernels on the GPU that also applies the mask to
- * the logits.
+ * the logits, and the classification is kept incremental: the same classifier
+ * is also built reading the stack from the bottom, its state is kept for every
+ * stack prefix, and a step re-reads only the stack entries it changed.
  *
  * Conventions for every call:
  *  - Pointers named d_* are device memory owned by the caller (for example the
@@ -178,9 +180,10 @@ psc_status psc_advance(const psc_handle* h, psc_states* st, const int32_t* d_tok
                        int32_t* d_row_status, void* stream);
 
 /* Algorithm 2, steps 3-4: classifies every row's (q, alpha) with the classifier
- * DFA (one pass over the stack from the top, stopping at absorbing states;
- * skipped when the last psc_advance or decode step already did it) and writes
- * the precomputed mask of the resulting state as a packed bitmask.
+ * DFA (from the bottom-up classifier's kept state when it is built, else one
+ * pass over the stack from the top, stopping at absorbing states; skipped when
+ * the last psc_advance or decode step already did it) and writes the
+ * precomputed mask of the resulting state as a packed bitmask.
  *   d_bitmask : device uint32 [B][W], W = ceil(V/32), row-contiguous.
  * Rows with status DONE get the end-of-sequence-only mask, failed rows the
  * empty mask. */
@@ -197,8 +200,8 @@ psc_status psc_fill_mask(const psc_handle* h, const psc_states* st, int32_t B, u
 psc_status psc_apply_mask(void* d_logits, psc_dtype dtype, int64_t row_stride, const uint32_t* d_bitmask,
                           int32_t B, int32_t V, void* stream);
 
-/* psc_fill_mask and psc_apply_mask fused: the classifier walk picks each row's
- * mask row, which is applied to the logits straight from the device mask table
+/* psc_fill_mask and psc_apply_mask fused: the row's classification (as in
+ * psc_fill_mask) picks its mask row, which is applied to the logits straight from the device mask table
  * (the bitmask does not round-trip through memory).  V must equal the
  * handle's vocabulary size.
  *   d_bitmask_out : optional device uint32 [B][W] copy of the masks (NULL = none). */
