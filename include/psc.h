@@ -103,9 +103,10 @@ typedef struct {
 /* Offline construction (Algorithm 1, Section 3).  Reads the grammar text (a
  * Lark-like notation, see the library's documentation), builds the lexer DFA,
  * the LALR(1) tables, the realizable terminal sequences R_q(v) of every token
- * from every lexer state (Section 3.1), the stack classifier of Eq. (9) and the
- * mask of every classifier state, and uploads the tables to the current CUDA
- * device unless opts->host_only.
+ * from every lexer state (Section 3.1), the stack classifier of Eq. (9), its
+ * bottom-up form (unless opts say otherwise) and the mask of every classifier
+ * state, and uploads the tables to the current CUDA device unless
+ * opts->host_only.
  *   grammar/grammar_len : grammar text (not NUL-terminated necessarily)
  *   vocab_bytes         : all token byte strings concatenated (host)
  *   vocab_offsets       : V+1 int64 offsets; token v = vocab_bytes[off[v], off[v+1])
@@ -125,8 +126,8 @@ void psc_destroy(psc_handle* h);
 
 /* Writes the handle's compiled tables to a binary file (the paper ships its
  * preprocessing results to decoding users as files, Section 5).  The file holds
- * the lexer, parser, classifier and mask tables and the vocabulary, with a
- * checksum.  Errors: PSC_ERR_IO, PSC_ERR_ARG. */
+ * the lexer, parser, classifier (both forms) and mask tables and the
+ * vocabulary, with a checksum.  Errors: PSC_ERR_IO, PSC_ERR_ARG. */
 psc_status psc_save(const psc_handle* h, const char* path);
 
 /* Reads a file written by psc_save, checks its checksum and the consistency of
