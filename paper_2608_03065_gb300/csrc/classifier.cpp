@@ -55,6 +55,17 @@ uint64_t hash_span(const int32_t* p, size_t n, uint64_t seed) {
     return h;
 }
 
+// Hash of a mask row: the XOR of one mixed value per non-zero word (mix64 is a
+// bijection, so distinct (index, word) pairs give distinct values).  Setting
+// bits in a few words updates it in O(words changed) instead of O(W).
+uint64_t word_hash(size_t i, uint32_t w) { return w ? mix64(((uint64_t)i << 32) ^ w ^ 0x5bd1e995u) : 0; }
+
+uint64_t row_hash(const uint32_t* r, int W) {
+    uint64_t h = 0;
+    for (int i = 0; i < W; i++) h ^= word_hash((size_t)i, r[i]);
+    return h;
+}
+
 // ----------------------------------------------------------------- tries
 struct Trie {
     std::vector<int32_t> child_off{0}, child_cls, child_node;
@@ -217,6 +228,7 @@ struct Builder {
     std::vector<int32_t> res_th, res_acc;
     // masks
     std::vector<uint32_t> rows;                    // [n_masks][W]
+    std::vector<uint64_t> row_hashes;              // row_hash of each row
     std::unordered_multimap<uint64_t, int32_t> row_index;
     std::unordered_map<uint64_t, int32_t> mask_memo;   // (mask, acc list id) -> mask
     ListPool acc_lists;
@@ -253,8 +265,7 @@ struct Builder {
         rows.assign(2 * (size_t)W, 0);
     }
 
-    int32_t add_row(const uint32_t* r) {
-        uint64_t h = hash_span((const int32_t*)r, W, 99);
+    int32_t add_row(const uint32_t* r, uint64_t h) {   // h = row_hash(r)
         auto range = row_index.equal_range(h);
         for (auto it = range.first; it != range.second; ++it)
             if (!memcmp(rows.data() + (size_t)it->second * W, r, sizeof(uint32_t) * W)) return it->second;
@@ -262,6 +273,7 @@ struct Builder {
         if ((int64_t)(rows.size() + W) * 4 > opt.max_mask_bytes)
             throw Error(ST_ERR_LIMIT, "mask rows exceed the memory limit");
         rows.insert(rows.end(), r, r + W);
+        row_hashes.push_back(h);
         row_index.emplace(h, id);
         return id;
     }
@@ -359,12 +371,17 @@ struct Builder {
         int32_t out = m;
         if (fresh) {
             std::vector<uint32_t> row(base, base + W);
+            uint64_t h = row_hashes[m];
             for (int32_t n : acc)
                 for (int32_t k = tr.tok_off[n]; k < tr.tok_off[n + 1]; k++) {
                     int v = tr.toks[k];
-                    row[v >> 5] |= 1u << (v & 31);
+                    uint32_t old = row[v >> 5], now = old | (1u << (v & 31));
+                    if (now != old) {
+                        h ^= word_hash((size_t)(v >> 5), old) ^ word_hash((size_t)(v >> 5), now);
+                        row[v >> 5] = now;
+                    }
                 }
-            out = add_row(row.data());
+            out = add_row(row.data(), h);
         }
         mask_memo.emplace(key, out);
         return out;
@@ -555,8 +572,8 @@ Tables compile_tables(const std::string& text, const uint8_t* vb, const int64_t*
     std::vector<uint32_t> grows(2 * (size_t)W, 0);
     std::copy(eos_row.begin(), eos_row.end(), grows.begin() + W);
     std::unordered_multimap<uint64_t, int32_t> gindex;
-    gindex.emplace(hash_span((const int32_t*)grows.data(), W, 99), 0);
-    gindex.emplace(hash_span((const int32_t*)grows.data() + W, W, 99), 1);
+    gindex.emplace(row_hash(grows.data(), W), 0);
+    gindex.emplace(row_hash(grows.data() + W, W), 1);
     struct Part {
         std::vector<int32_t> st_mask, st_def, exc_y, exc_t;
         std::vector<int64_t> exc_off;
@@ -587,8 +604,9 @@ Tables compile_tables(const std::string& text, const uint8_t* vb, const int64_t*
                 Builder B(L, P, tr, resolve, end_cls, V, opt);
                 std::copy(eos_row.begin(), eos_row.end(), B.rows.begin() + W);
                 B.row_index.clear();
-                B.row_index.emplace(hash_span((const int32_t*)B.rows.data(), W, 99), 0);
-                B.row_index.emplace(hash_span((const int32_t*)B.rows.data() + W, W, 99), 1);
+                B.row_hashes = {row_hash(B.rows.data(), W), row_hash(B.rows.data() + W, W)};
+                B.row_index.emplace(B.row_hashes[0], 0);
+                B.row_index.emplace(B.row_hashes[1], 1);
                 B.state(0, {});
                 int32_t th = B.thread({tr.root[q], -1, 0, -1});
                 Part& pt = parts[q];
@@ -602,14 +620,11 @@ Tables compile_tables(const std::string& text, const uint8_t* vb, const int64_t*
                 // move this part's masks into the global pool
                 int nm = (int)(B.rows.size() / W);
                 std::vector<int32_t> gid(nm);
-                std::vector<uint64_t> row_hash(nm);   // hashed before taking the pool's lock
-                for (int m = 0; m < nm; m++)
-                    row_hash[m] = hash_span((const int32_t*)B.rows.data() + (size_t)m * W, W, 99);
                 {
                     std::lock_guard<std::mutex> lk(pool_mu);
                     for (int m = 0; m < nm; m++) {
                         const uint32_t* r = B.rows.data() + (size_t)m * W;
-                        uint64_t h = row_hash[m];
+                        uint64_t h = B.row_hashes[m];
                         int32_t found = -1;
                         auto range = gindex.equal_range(h);
                         for (auto it = range.first; it != range.second; ++it)
@@ -659,6 +674,13 @@ Tables compile_tables(const std::string& text, const uint8_t* vb, const int64_t*
     }
     if (first_code) throw Error(first_code, first_error);
     if (getenv("PSC_LOG")) {
+        double busy = 0, longest = 0;
+        for (int q = 0; q < L.nq; q++) {
+            busy += parts[q].seconds;
+            longest = std::max(longest, parts[q].seconds);
+        }
+        fprintf(stderr, "psc: %d lexer states on %d threads: %.2f s of builder time, longest %.2f s\n", L.nq,
+                threads, busy, longest);
         for (int k = 0; k < std::min(L.nq, 12); k++) {
             int q = qorder[k];
             fprintf(stderr, "psc: lexer state %d: %zu classifier states, %lld threads, %.2f s\n", q,
