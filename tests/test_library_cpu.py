@@ -9,7 +9,7 @@ import re
 import numpy as np
 import pytest
 
-from oracle import Oracle, Vocab
+from oracle import ST_DONE, ST_ERROR, ST_OK, Oracle, Vocab
 from workloads import configs, grammars
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
@@ -194,6 +194,97 @@ def test_host_tables_match_golden_masks(psc, fixture):
             assert set(np.nonzero(bits)[0].tolist()) == allowed, prefix
             n += 1
     assert n >= 7
+
+
+@pytest.mark.parametrize("which", ["arith", "json"])
+def test_host_tables_exhaustive_small_configurations(psc, which):
+    """Every configuration the micro vocabularies reach in up to 6 tokens
+    (breadth first, deduplicated by lexer state and stack): the compiled tables'
+    mask equals the oracle's, and so does the status of every next token."""
+    from .test_oracle_pins import JSON_MICRO, MICRO
+    text, vocab = ((grammars.arithmetic().text(), MICRO) if which == "arith"
+                   else (grammars.json_grammar().text(), JSON_MICRO))
+    eos = len(vocab) - 1
+    h = psc.psc_compile(text, vocab, eos, host_only=True)
+    o = Oracle(text)
+    voc = Vocab.from_list(vocab, eos)
+    seen = {}
+    frontier = [((), h.host_initial())]
+    for _ in range(6):
+        nxt = []
+        for seq, c in frontier:
+            for v in range(eos):
+                c2 = h.host_advance(c, v, cap=64)
+                key = (c2["q"], tuple(c2["stack"]))
+                if c2["status"] != psc.ROW_OK or key in seen:
+                    continue
+                seen[key] = seq + (v,)
+                nxt.append((seq + (v,), c2))
+        frontier = nxt
+    assert len(seen) > 100
+    cfgs, ocs = [], []
+    for (q, stack), seq in seen.items():
+        oc = o.initial()
+        assert o.advance_tokens(oc, voc, seq) == ST_OK
+        cfgs.append({"q": q, "stack": list(stack), "status": psc.ROW_OK})
+        ocs.append(oc)
+    om = o.masks(ocs, voc)
+    want_status = {ST_OK: psc.ROW_OK, ST_DONE: psc.ROW_DONE, ST_ERROR: psc.ROW_REJECTED}
+    for c, oc, m in zip(cfgs, ocs, om):
+        np.testing.assert_array_equal(_host_mask(h, c), m, err_msg=str(c))
+        for v in range(len(vocab)):
+            oc2 = oc.copy()
+            st = o.advance(oc2, None if v == eos else vocab[v])
+            assert h.host_advance(c, v, cap=64)["status"] == want_status[st], (c, v)
+
+
+@pytest.mark.parametrize("cfg_id", [1, 2, 3, 4])
+def test_host_tables_on_sentences_and_mutations(psc, cfg_id):
+    """Whole sentences of each workload grammar and copies with one byte
+    inserted, deleted or replaced, fed byte by byte (a vocabulary of the 256
+    single bytes): the compiled LALR(1) tables and lexer stop at the same byte
+    as the oracle's canonical LR(1) parser and Thompson-NFA lexer, and accept the
+    same strings at the end of sequence."""
+    from workloads.sample import SentenceSampler
+    spec = configs.grammar_spec(cfg_id)
+    text = spec.text()
+    vocab = [bytes([b]) for b in range(256)] + [b""]
+    h = psc.psc_compile(text, vocab, 256, host_only=True)
+    o = Oracle(text)
+    want_status = {ST_OK: psc.ROW_OK, ST_DONE: psc.ROW_DONE, ST_ERROR: psc.ROW_REJECTED}
+    rng = np.random.default_rng([cfg_id, 11])
+    sampler = SentenceSampler(spec, max_depth=10)
+    n = stopped = tries = 0
+    while n < 60 and tries < 2000:
+        tries += 1
+        txt, finished = sampler.text(rng, 4000)
+        if not finished or not txt:
+            continue
+        b = bytearray(txt)
+        if n % 4:   # three in four mutated, one in four kept whole
+            kind, pos, ch = int(rng.integers(0, 3)), int(rng.integers(0, len(b))), int(rng.integers(0x20, 0x7F))
+            if kind == 0:
+                b.insert(pos, ch)
+            elif kind == 1:
+                del b[pos]
+            else:
+                b[pos] = ch
+        c, oc = h.host_initial(), o.initial()
+        st = ST_OK
+        for byte in bytes(b):
+            st = o.advance(oc, bytes([byte]))
+            c = h.host_advance(c, byte, cap=1024)
+            assert c["status"] == want_status[st], (bytes(b), byte)
+            if st != ST_OK:
+                break
+        if st == ST_OK:
+            st = o.advance(oc, None)
+            assert h.host_advance(c, 256, cap=1024)["status"] == want_status[st], bytes(b)
+        if n % 4 == 0:
+            assert st == ST_DONE, bytes(b)   # whole sentences are accepted
+        stopped += st != ST_DONE
+        n += 1
+    assert n == 60 and stopped > 10
 
 
 def test_host_tables_deep_parentheses(psc):
