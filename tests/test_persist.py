@@ -60,6 +60,23 @@ def test_corrupt_and_truncated_files_are_refused(psc, tmp_path):
         assert e.value.code == 8, suffix
 
 
+def test_tables_without_bottom_up_round_trip(psc, tmp_path):
+    """A handle compiled without the bottom-up classifier saves and loads (the
+    loaded handle has none either) and classifies as before."""
+    w = configs.load(1, batch=4)
+    h = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id, host_only=True, bottom_up=False)
+    path = str(tmp_path / "plain.psc")
+    psc.psc_save(h, path)
+    h2 = psc.psc_load(path, host_only=True)
+    assert h2.info().bottom_up_states == 0
+    for ids in w.prefix_ids:
+        c = h.host_initial()
+        for v in ids:
+            c = h.host_advance(c, v)
+        assert h2.host_classify(c["q"], c["stack"]) == h.host_classify(c["q"], c["stack"])
+        assert h2.host_classify_bottom_up(c["q"], c["stack"]) == -2
+
+
 def _fnv1a64(data: bytes) -> int:
     h = 1469598103934665603
     for b in data:
