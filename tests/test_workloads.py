@@ -1,0 +1,61 @@
+"""The seeded input recipe of the five workloads: sizes, vocabulary structure,
+prefix lengths and tokenization, logits distribution, and determinism (every
+input is a pure function of the config id and its seed streams)."""
+from __future__ import annotations
+
+import numpy as np
+import pytest
+
+from workloads import configs
+
+torch = pytest.importorskip("torch")
+
+SINGLES = {bytes([b]) for b in list(range(0x20, 0x7F)) + [9, 10, 13]}
+
+
+@pytest.mark.parametrize("cfg_id,batch", [(1, None), (2, None), (3, 16), (4, 16), (5, 16)])
+def test_vocabulary_and_prefixes(cfg_id, batch):
+    w = configs.load(cfg_id, batch=batch)
+    s = configs.SPECS[cfg_id]
+    assert len(w.vocab) == s.V == w.V
+    assert w.eos_id == s.V - 1 and w.vocab[w.eos_id] == b""
+    assert len(set(w.vocab)) == s.V                          # unique strings
+    assert SINGLES <= set(w.vocab)                           # every prefix is tokenizable
+    assert max(len(t) for t in w.vocab) <= s.vocab_max_len
+    assert all(len(t) >= 1 for t in w.vocab[:-1])
+    assert len(w.prefixes) == len(w.prefix_ids) == w.B == (batch or s.B)
+    o = None
+    for p, ids in zip(w.prefixes, w.prefix_ids):
+        assert 1 <= len(p) <= s.prefix_max
+        if len(p) < s.prefix_min:   # the drawn length is a target: a sentence that ends first is kept whole
+            if o is None:
+                from oracle import Oracle
+                o = Oracle(w.grammar_text)
+            c = o.initial()
+            o.advance(c, p)
+            assert o.allowed(c, None), p
+        assert b"".join(w.vocab[i] for i in ids) == p        # greedy tokenization is exact
+        assert w.eos_id not in ids
+    m = w.token_matrix()
+    assert m.shape[0] == w.B and m.dtype == np.int32
+
+
+def test_inputs_are_deterministic():
+    a, b = configs.load(2, batch=8), configs.load(2, batch=8)
+    assert a.vocab == b.vocab and a.prefixes == b.prefixes and a.prefix_ids == b.prefix_ids
+    x, y = a.logits(3), b.logits(3)
+    assert torch.equal(x.view(torch.int16), y.view(torch.int16))
+    assert not torch.equal(a.logits(3).float(), a.logits(4).float())   # fresh logits per step
+
+
+@pytest.mark.parametrize("cfg_id", [1, 2])
+def test_logits_distribution(cfg_id):
+    """fp32 N(0,1) for config 1; bf16 N(0,2) (variance 2) for the others."""
+    w = configs.load(cfg_id, batch=8)
+    x = w.logits(0)
+    assert tuple(x.shape) == (w.B, w.V)
+    assert x.dtype == (torch.float32 if cfg_id == 1 else torch.bfloat16)
+    v = x.float().var().item()
+    want = 1.0 if cfg_id == 1 else 2.0
+    assert abs(v - want) < 0.1 * want
+    assert abs(x.float().mean().item()) < 0.05 * want ** 0.5
