@@ -287,6 +287,27 @@ def test_host_tables_on_sentences_and_mutations(psc, cfg_id):
     assert n == 60 and stopped > 10
 
 
+def test_host_tables_terminal_rank(psc):
+    """The compiled lexer resolves colliding terminals like the hand-derived
+    oracle pin: priority first, then name (basic), or the first one the parser
+    can take (contextual)."""
+    from workloads.sample import TrieTokenizer
+    from .test_oracle_pins import PRIO, TIE
+    toks = [b"12", b"12 ", b"x", b"+", b" ", b"1", b"2", b""]
+    cases = [(PRIO, b"", {4}, {0, 1, 4, 5, 6}), (TIE, b"", {0, 1, 4, 5, 6}, {0, 1, 4, 5, 6}),
+             (TIE, b"1+", {4}, {0, 1, 4, 5, 6}), (TIE, b"1+2", None, {0, 1, 4, 5, 6, 7})]
+    tok = TrieTokenizer(toks)
+    for text, prefix, want_basic, want_ctx in cases:
+        for mode, want in (("basic", want_basic), ("contextual", want_ctx)):
+            if want is None:
+                continue
+            h = psc.psc_compile(text.replace("%lexer basic", "%lexer " + mode), toks, 7, host_only=True)
+            c = _host_cfg(h, tok.encode(prefix) if prefix else [])
+            assert c["status"] == psc.ROW_OK
+            bits = np.unpackbits(_host_mask(h, c).view(np.uint8), bitorder="little")[:len(toks)]
+            assert set(np.nonzero(bits)[0].tolist()) == want, (prefix, mode)
+
+
 def test_host_tables_deep_parentheses(psc):
     """Balanced parentheses to depth 200: the classifier walk reads deep stacks."""
     g = 'start: s\ns: | s "(" s ")"\n'

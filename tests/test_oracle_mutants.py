@@ -23,6 +23,7 @@ BATTERY = [
     "test_closed_form_balanced_parentheses_deep", "test_closed_form_single_literal",
     "test_closed_form_any_bytes", "test_eq1_completion_search_arithmetic",
     "test_contextual_keyword_resolution", "test_contextual_uses_lalr_action_set",
+    "test_terminal_rank_priority_then_name",
     "test_eos_only_after_complete_sentence", "test_sampled_sentences_are_sentences",
     ("test_earley_cross_check_workload", 1), ("test_invariants_on_workloads", 1),
     ("test_tokenwise_equals_bytewise", 1), ("test_tokenwise_equals_bytewise", 2),

@@ -267,6 +267,50 @@ def test_contextual_keyword_resolution():
             assert orc.mask_set(cf, voc) == want, (prefix, orc.grammar.lexer_mode)
 
 
+PRIO = '''
+start: A "+" B
+A: /[0-9]+/
+B.2: /[0-9a-z]+/
+WS: /[ ]+/
+%ignore WS
+%lexer basic
+'''
+
+TIE = '''
+start: AA "+" BB
+AA: /[0-9]+/
+BB: /[0-9]+/
+WS: /[ ]+/
+%ignore WS
+%lexer basic
+'''
+
+
+def test_terminal_rank_priority_then_name():
+    """Hand-derived: with the basic lexer a lexeme matching several terminals is
+    the highest-ranked one, by priority first (B.2 over A, so no digit string
+    can be the A the grammar starts with), then by name (AA over BB, so after
+    "1+" no digit string can be the BB the grammar wants); the contextual lexer
+    picks, among them, one the parser can take."""
+    toks = [b"12", b"12 ", b"x", b"+", b" ", b"1", b"2"]
+    voc = Vocab.from_list(toks + [b""], eos_id=len(toks))
+    cases = [   # (grammar, prefix, basic mask, contextual mask); None: the prefix is not reachable
+        (PRIO, b"", {4}, {0, 1, 4, 5, 6}),
+        (TIE, b"", {0, 1, 4, 5, 6}, {0, 1, 4, 5, 6}),
+        (TIE, b"1+", {4}, {0, 1, 4, 5, 6}),
+        (TIE, b"1+2", None, {0, 1, 4, 5, 6, 7}),
+    ]
+    for text, prefix, want_basic, want_ctx in cases:
+        for mode, want in (("basic", want_basic), ("contextual", want_ctx)):
+            if want is None:
+                continue
+            o = Oracle(text.replace("%lexer basic", "%lexer " + mode))
+            cf = o.initial()
+            for ch in prefix:
+                assert o.advance(cf, bytes([ch])) == ST_OK
+            assert o.mask_set(cf, voc) == want, (text.split()[1], prefix, mode, sorted(o.mask_set(cf, voc)))
+
+
 LALR_MERGE = '''
 start: "a" e "x" | "a" e NAME "z" | "b" e "y"
 e: "e"
