@@ -177,6 +177,39 @@ def test_eq1_completion_search_arithmetic():
             assert (v in got) == brute, (prefix, t)
 
 
+def test_eq1_completion_search_json():
+    """Eq. (1) by search on the JSON grammar with the JSON micro vocabulary:
+    completions y over 9 single bytes up to length 4 (memoised; a branch stops
+    once its terminals are no prefix of a sentence), on prefixes inside numbers,
+    strings, escapes, objects and arrays."""
+    text = grammars.json_grammar().text()
+    o = Oracle(text)
+    voc = Vocab.from_list(JSON_MICRO, eos_id=18)
+    py = PyCheck(parse_grammar(text))
+    alphabet = [b'"', b"a", b"1", b"}", b"]", b":", b",", b"u", b"e"]
+    memo = {}
+
+    def witness(s: bytes, budget: int) -> bool:
+        if (s, budget) not in memo:
+            r = py.lex(s)
+            if r is None or not py.earley.viable(r[0]):
+                memo[s, budget] = False
+            elif py.sentence(s):
+                memo[s, budget] = True
+            else:
+                memo[s, budget] = budget > 0 and any(witness(s + c, budget - 1) for c in alphabet)
+        return memo[s, budget]
+
+    for prefix in [b"", b"{", b'{"a":', b"[1", b"[1e", b"[1,", b'"', b'"\\', b"0", b"-", b"[", b'{"a"']:
+        cf = o.initial()
+        for ch in prefix:
+            assert o.advance(cf, bytes([ch])) == ST_OK
+        got = o.mask_set(cf, voc)
+        for v, t in enumerate(JSON_MICRO):
+            brute = py.sentence(prefix) if v == voc.eos_id else witness(prefix + t, 4)
+            assert (v in got) == brute, (prefix, t)
+
+
 # ------------------------------------------------------ independent parser
 @pytest.mark.parametrize("cfg_id", [1, 2])
 def test_earley_cross_check_workload(cfg_id):
