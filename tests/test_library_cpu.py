@@ -157,6 +157,38 @@ def test_bottom_up_classifier_c_like_random_walks(psc):
     assert n > 1000 and deepest > 16
 
 
+@pytest.mark.parametrize("name", ["literal", "any_bytes", "parentheses"])
+def test_bottom_up_classifier_small_grammars(psc, name):
+    """Degenerate classifiers (a single literal, every byte string, balanced
+    parentheses): the bottom-up classifier is built and agrees with the walk
+    along random decodes."""
+    grammar, toks = {
+        "literal": ('start: "hello world"\n', [b"h", b"he", b"hello", b" ", b"world", b"o w", b"d", b"x", b""]),
+        "any_bytes": ("start: | start ANY\nANY: /[\\x00-\\xff]/\n", [bytes([b]) for b in range(256)] + [b"ab", b""]),
+        "parentheses": ('start: s\ns: | s "(" s ")"\n', [b"(", b")", b"((", b"))", b""]),
+    }[name]
+    eos = len(toks) - 1
+    h = psc.psc_compile(grammar, toks, eos, host_only=True)
+    assert h.info().bottom_up_states > 0
+    rng = np.random.default_rng(0)
+    n = 0
+    for _ in range(20):
+        c = h.host_initial()
+        for _ in range(40):
+            mid = h.host_classify(c["q"], c["stack"])
+            assert h.host_classify_bottom_up(c["q"], c["stack"]) == mid, c
+            n += 1
+            bits = np.unpackbits(h.host_mask_row(mid).view(np.uint8), bitorder="little")[:len(toks)].astype(bool)
+            bits[eos] = False
+            allowed = np.nonzero(bits)[0]
+            if len(allowed) == 0:
+                break
+            c = h.host_advance(c, int(rng.choice(allowed)), cap=512)
+            if c["status"] != psc.ROW_OK:
+                break
+    assert n >= 20
+
+
 def test_bottom_up_classifier_limits(psc):
     """Not built on request or over its memory limit (compilation still succeeds;
     the device then walks stacks from the top)."""
