@@ -114,9 +114,13 @@ def _stream(stream) -> int | None:
     return stream.cuda_stream or None
 
 
-def _ptr(t, dtype=None, name="tensor"):
+def _ptr(t, dtype=None, name="tensor", n=None):
+    """Device address of a tensor argument; n = the elements the call reads or
+    writes (a smaller or non-contiguous tensor is refused before any launch)."""
     if t is None:
         return None
+    if n is not None and (t.numel() < n or not t.is_contiguous()):
+        raise ValueError(f"{name} must be a contiguous tensor of at least {n} elements")
     if not t.is_cuda:
         raise ValueError(f"{name} must be a CUDA tensor")
     if dtype is not None and t.dtype != dtype:
@@ -273,7 +277,7 @@ def psc_state_init(h: Handle, B: int, cap: int = 256, stream=None) -> States:
 def psc_state_reset(st: States, rows=None, stream=None):
     import torch
     n = st.B if rows is None else rows.numel()
-    _check(load().psc_state_reset(st.ptr, _ptr(rows, torch.int32, "rows"), n, _stream(stream)))
+    _check(load().psc_state_reset(st.ptr, _ptr(rows, torch.int32, "rows", n), n, _stream(stream)))
 
 
 def psc_state_copy(dst: States, src: States, stream=None):
@@ -283,8 +287,8 @@ def psc_state_copy(dst: States, src: States, stream=None):
 
 def psc_advance(h: Handle, st: States, tokens, row_status=None, stream=None):
     import torch
-    _check(load().psc_advance(h.ptr, st.ptr, _ptr(tokens, torch.int32, "tokens"), st.B,
-                              _ptr(row_status, torch.int32, "row_status"), _stream(stream)))
+    _check(load().psc_advance(h.ptr, st.ptr, _ptr(tokens, torch.int32, "tokens", st.B), st.B,
+                              _ptr(row_status, torch.int32, "row_status", st.B), _stream(stream)))
 
 
 def psc_fill_mask(h: Handle, st: States, bitmask, stream=None):
@@ -322,7 +326,7 @@ def psc_argmax_masked(h: Handle, st: States, logits, tokens, stream=None):
     if tokens.numel() != st.B:
         raise ValueError("tokens must hold B int32 values")
     _check(load().psc_argmax_masked(h.ptr, st.ptr, st.B, _ptr(logits, None, "logits"), _dtype_code(logits),
-                                    _row_stride(logits), h.V, _ptr(tokens, torch.int32, "tokens"),
+                                    _row_stride(logits), h.V, _ptr(tokens, torch.int32, "tokens", st.B),
                                     _stream(stream)))
 
 
@@ -336,7 +340,7 @@ def psc_fill_apply_argmax(h: Handle, st: States, logits, tokens, bitmask_out=Non
         raise ValueError("bitmask_out must be a contiguous [B, W] tensor")
     _check(load().psc_fill_apply_argmax(h.ptr, st.ptr, st.B, _ptr(logits, None, "logits"), _dtype_code(logits),
                                         _row_stride(logits), h.V, _ptr(bitmask_out, torch.int32, "bitmask_out"),
-                                        _ptr(tokens, torch.int32, "tokens"), _stream(stream)))
+                                        _ptr(tokens, torch.int32, "tokens", st.B), _stream(stream)))
 
 
 def psc_decode_step(h: Handle, st: States, logits, tokens, bitmask_out=None, row_status=None, stream=None):
@@ -349,8 +353,8 @@ def psc_decode_step(h: Handle, st: States, logits, tokens, bitmask_out=None, row
         raise ValueError("bitmask_out must be a contiguous [B, W] tensor")
     _check(load().psc_decode_step(h.ptr, st.ptr, st.B, _ptr(logits, None, "logits"), _dtype_code(logits),
                                   _row_stride(logits), h.V, _ptr(bitmask_out, torch.int32, "bitmask_out"),
-                                  _ptr(tokens, torch.int32, "tokens"), _ptr(row_status, torch.int32, "row_status"),
-                                  _stream(stream)))
+                                  _ptr(tokens, torch.int32, "tokens", st.B),
+                                  _ptr(row_status, torch.int32, "row_status", st.B), _stream(stream)))
 
 
 def psc_decode_step_mask(h: Handle, st: States, logits, bitmask_out=None, stream=None):
@@ -370,8 +374,8 @@ def psc_decode_step_advance(h: Handle, st: States, tokens, row_status=None, stre
     import torch
     if tokens.numel() != st.B:
         raise ValueError("tokens must hold B int32 values")
-    _check(load().psc_decode_step_advance(h.ptr, st.ptr, st.B, _ptr(tokens, torch.int32, "tokens"),
-                                          _ptr(row_status, torch.int32, "row_status"), _stream(stream)))
+    _check(load().psc_decode_step_advance(h.ptr, st.ptr, st.B, _ptr(tokens, torch.int32, "tokens", st.B),
+                                          _ptr(row_status, torch.int32, "row_status", st.B), _stream(stream)))
 
 
 def psc_states_download(st: States, stream=None) -> dict:
@@ -395,8 +399,8 @@ def psc_fill_apply_noalloc(h: Handle, q, depth, status, stack, logits, bitmask_o
         raise ValueError("stack must be a contiguous [B, cap] 16-bit tensor")
     if logits.shape[0] != B or logits.shape[1] < V:
         raise ValueError("logits must be [B, >=V]")
-    _check(load().psc_fill_apply_noalloc(h.ptr, _ptr(q, torch.int32, "q"), _ptr(depth, torch.int32, "depth"),
-                                         _ptr(status, torch.int32, "status"), _ptr(stack, None, "stack"),
+    _check(load().psc_fill_apply_noalloc(h.ptr, _ptr(q, torch.int32, "q", B), _ptr(depth, torch.int32, "depth", B),
+                                         _ptr(status, torch.int32, "status", B), _ptr(stack, None, "stack"),
                                          stack.shape[1], B, _ptr(logits, None, "logits"), _dtype_code(logits),
                                          _row_stride(logits), V, _ptr(bitmask_out, torch.int32, "bitmask_out"),
                                          _stream(stream)))

@@ -428,6 +428,22 @@ def test_host_calls_check_their_arguments(psc):
     assert c == h.host_initial()
 
 
+def test_binding_refuses_short_or_host_arrays(psc):
+    """The binding checks per-row arrays before any launch: fewer elements than
+    rows, a non-contiguous view, or host memory are refused with ValueError."""
+    torch = pytest.importorskip("torch")
+    _, h = _handle(psc, 1, 8)
+    st = psc.States(0, h, 4, 16)   # never reaches the library: every call below fails first
+    for tokens in (torch.zeros(2, dtype=torch.int32), torch.zeros(8, dtype=torch.int32)[::2],
+                   torch.zeros(4, dtype=torch.int32)):
+        with pytest.raises(ValueError):
+            psc.psc_advance(h, st, tokens)
+        with pytest.raises(ValueError):
+            psc.psc_decode_step_advance(h, st, tokens)
+    with pytest.raises(ValueError):
+        psc.psc_state_reset(st, torch.zeros(3, dtype=torch.int64))
+
+
 def test_device_calls_refuse_host_only_handle(psc):
     h = psc.psc_compile(grammars.arithmetic().text(), [b"1", b""], 1, host_only=True)
     with pytest.raises(psc.PscError) as e:
