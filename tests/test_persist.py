@@ -77,6 +77,23 @@ def test_tables_without_bottom_up_round_trip(psc, tmp_path):
         assert h2.host_classify_bottom_up(c["q"], c["stack"]) == -2
 
 
+def test_compiled_tables_do_not_depend_on_the_thread_count(psc, tmp_path):
+    """Files compiled with 1 and with 8 host threads are byte-identical except
+    for the recorded compile time (and so the checksum): table ids are numbered
+    in an order that does not depend on which thread finishes first."""
+    w = configs.load(2, batch=2)
+    data = []
+    for th in (1, 8):
+        h = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id, host_only=True, threads=th)
+        path = str(tmp_path / f"t{th}.psc")
+        psc.psc_save(h, path)
+        data.append(open(path, "rb").read())
+    a, b = data
+    t0 = 8 + 15 * 4 + 3 * 8   # magic, 15 int32 and 3 int64 scalars, then the compile time (double)
+    assert len(a) == len(b)
+    assert a[:t0] == b[:t0] and a[t0 + 8:-8] == b[t0 + 8:-8]
+
+
 def _fnv1a64(data: bytes) -> int:
     h = 1469598103934665603
     for b in data:
