@@ -13,7 +13,7 @@
  * pending lexeme p can still become) takes the parser from the current stack to
  * a stable stack.  It does this the slow way: for every row and every token it
  * lexes the token's bytes and simulates the LR(1) parser on a copy-on-write view
- * of the row's stack.  This is the "call the parser for every token" scheme the
+ * of the row's stack: the scheme that runs the parser once per token, which the
  * paper sets against PSC (Fig. 1b).
  *
  * Lexer reading (the paper defers its lexer to prior work): bytes, maximal munch
