@@ -27,6 +27,7 @@ BATTERY = [
     "test_eos_only_after_complete_sentence", "test_sampled_sentences_are_sentences",
     ("test_earley_cross_check_workload", 1), ("test_invariants_on_workloads", 1),
     ("test_tokenwise_equals_bytewise", 1), ("test_tokenwise_equals_bytewise", 2),
+    ("test_earley_cross_check_random_grammars", 40),
 ]
 
 # name: (text in brute.c, replacement)
