@@ -2,7 +2,8 @@
 grammars: the library's compiled tables (its own grammar reader, lexer DFA,
 LALR(1) tables, classifier and bottom-up classifier) against the oracle (its
 own reader, Thompson-NFA lexer, canonical LR(1) parser and per-token brute
-force), on every configuration a random vocabulary reaches in up to 5 tokens.
+force), on the configurations a random vocabulary reaches in up to 5 tokens
+(small grammars) or 6 tokens (the larger variant), at most 200 / 400 of them.
 
 Grammars mix literals with two regex terminals that collide with them (so
 lexemes form classes), ignored whitespace, empty alternatives and recursion,
@@ -27,12 +28,13 @@ def psc():
     return mod
 
 
-def test_random_grammars_compiled_tables_match_the_oracle(psc):
-    rng = np.random.default_rng(20261202)
+@pytest.mark.parametrize("large,draws,depth,keep", [(False, 600, 5, 200), (True, 1500, 6, 400)])
+def test_random_grammars_compiled_tables_match_the_oracle(psc, large, draws, depth, keep):
+    rng = np.random.default_rng(20261202 + large)
     compared = configs_checked = 0
-    for _ in range(600):
-        text = random_grammar(rng)
-        vocab = random_vocab(rng)
+    for _ in range(draws):
+        text = random_grammar(rng, large)
+        vocab = random_vocab(rng, large)
         if text is None:
             continue
         eos = len(vocab) - 1
@@ -45,18 +47,18 @@ def test_random_grammars_compiled_tables_match_the_oracle(psc):
         voc = Vocab.from_list(vocab, eos)
         seen = {}
         frontier = [((), h.host_initial())]
-        for _ in range(5):
+        for _ in range(depth):
             nxt = []
             for seq, c in frontier:
                 for v in range(eos):
                     c2 = h.host_advance(c, v, cap=256)
                     key = (c2["q"], tuple(c2["stack"]))
-                    if c2["status"] == psc.ROW_OK and key not in seen:
+                    if c2["status"] == psc.ROW_OK and key not in seen and len(seen) < keep:
                         seen[key] = seq + (v,)
                         nxt.append((seq + (v,), c2))
             frontier = nxt
         cfgs, ocs = [h.host_initial()], [o.initial()]
-        for (q, stack), seq in list(seen.items())[:200]:
+        for (q, stack), seq in seen.items():
             oc = o.initial()
             assert o.advance_tokens(oc, voc, seq) == ST_OK, (text, seq)   # same reachable prefixes
             cfgs.append({"q": q, "stack": list(stack), "status": psc.ROW_OK})
