@@ -3,6 +3,7 @@ with nvcc (static CUDA runtime).  Translation units compile in parallel."""
 from __future__ import annotations
 
 import concurrent.futures as cf
+import fcntl
 import os
 import shutil
 import subprocess
@@ -33,7 +34,15 @@ def _stale(target: str, deps: list[str]) -> bool:
 
 
 def build(force: bool = False, verbose: bool = False) -> str:
+    """Compiles what is stale and links the library.  Processes that build at
+    the same time (one per rank) take turns on a lock file."""
     os.makedirs(BUILD, exist_ok=True)
+    with open(os.path.join(BUILD, ".lock"), "w") as lock:
+        fcntl.flock(lock, fcntl.LOCK_EX)
+        return _build_locked(force, verbose)
+
+
+def _build_locked(force: bool, verbose: bool) -> str:
     headers = [os.path.join(CSRC, "psc_internal.h"), os.path.join(INCLUDE, "psc.h")]
     nvcc = _nvcc()
     jobs = []
