@@ -38,6 +38,34 @@ def test_library_exports_every_declared_symbol(psc):
     assert set(syms) == set(psc.EXPORTED)
 
 
+def _c_type(decl: str):
+    """ctypes type the binding must use for one C parameter or return declaration."""
+    import ctypes
+    d = " ".join(decl.replace("const ", "").split())
+    if "*" in d:
+        return (ctypes.c_void_p, ctypes.c_char_p)
+    base = d.split()[0]
+    return {"int32_t": (ctypes.c_int32,), "psc_dtype": (ctypes.c_int32,), "psc_status": (ctypes.c_int32,),
+            "int64_t": (ctypes.c_int64,), "size_t": (ctypes.c_size_t,), "void": (None,)}[base]
+
+
+def test_binding_signatures_match_the_header(psc):
+    """Every prototype of include/psc.h has the same number and kinds of
+    parameters (pointer, int32, int64, size_t) and return type in the binding."""
+    lib = psc.load()
+    text = re.sub(r"/\*.*?\*/", "", open(os.path.join(ROOT, "include", "psc.h")).read(), flags=re.S)
+    protos = re.findall(r"([A-Za-z_][\w ]*?\**)\s*\b(psc_[a-z_]+)\s*\(([^)]*)\)\s*;", text)
+    assert len(protos) == len(psc.EXPORTED)
+    for ret, name, params in protos:
+        f = getattr(lib, name)
+        args = [] if params.strip() in ("", "void") else [p.strip() for p in params.split(",")]
+        assert len(f.argtypes) == len(args), name
+        for decl, t in zip(args, f.argtypes):
+            want = _c_type(decl.rsplit(" ", 1)[0] if "*" not in decl.split()[-1] else decl)
+            assert t in want, (name, decl, t)
+        assert f.restype in _c_type(ret), (name, ret, f.restype)
+
+
 def _host_cfg(h, ids):
     c = h.host_initial()
     for v in ids:
