@@ -66,6 +66,23 @@ def test_binding_signatures_match_the_header(psc):
         assert f.restype in _c_type(ret), (name, ret, f.restype)
 
 
+def test_binding_structs_match_the_header(psc):
+    """psc_options and psc_info_t: same fields, order and types in the binding."""
+    import ctypes
+    text = re.sub(r"/\*.*?\*/", "", open(os.path.join(ROOT, "include", "psc.h")).read(), flags=re.S)
+    ctype = {"int32_t": ctypes.c_int32, "int64_t": ctypes.c_int64, "double": ctypes.c_double}
+    for cname, py in (("psc_options", psc.Options), ("psc_info_t", psc.InfoT)):
+        body = re.search(r"typedef struct \{([^}]*)\}\s*" + cname + r"\s*;", text).group(1)
+        fields = []
+        for decl in body.split(";"):
+            decl = decl.strip()
+            if not decl:
+                continue
+            typ, names = decl.split(None, 1)
+            fields += [(n.strip(), ctype[typ]) for n in names.split(",")]
+        assert [(n, t) for n, t in py._fields_] == fields, cname   # ctypes then lays them out as C does
+
+
 def _host_cfg(h, ids):
     c = h.host_initial()
     for v in ids:
