@@ -489,6 +489,35 @@ def test_binding_refuses_short_or_host_arrays(psc):
         psc.psc_state_reset(st, torch.zeros(3, dtype=torch.int64))
 
 
+def test_c_abi_argument_errors(psc):
+    """Calls straight through the C ABI with bad arguments return PSC_ERR_ARG
+    (1) and leave a message; nothing is dereferenced."""
+    import ctypes
+    lib = psc.load()
+    g = b'start: "x"\n'
+    blob = (ctypes.c_uint8 * 1)(120)
+    offs = (ctypes.c_int64 * 3)(0, 1, 1)
+    bad_offs = (ctypes.c_int64 * 3)(0, 1, 0)
+    out = ctypes.c_void_p()
+    cases = [
+        lib.psc_compile(g, len(g), blob, offs, 2, 1, None, None),                 # out is NULL
+        lib.psc_compile(g, len(g), blob, offs, 0, -1, None, ctypes.byref(out)),   # V = 0
+        lib.psc_compile(g, len(g), blob, offs, 2, 2, None, ctypes.byref(out)),    # eos_id >= V
+        lib.psc_compile(g, len(g), blob, bad_offs, 2, 1, None, ctypes.byref(out)),  # offsets decrease
+        lib.psc_compile(None, 0, blob, offs, 2, 1, None, ctypes.byref(out)),      # no grammar
+        lib.psc_info(None, None),
+        lib.psc_save(None, b"/nonexistent/x"),
+        lib.psc_load(None, None, ctypes.byref(out)),
+        lib.psc_host_mask_row(None, 0, None),
+        lib.psc_host_advance(None, None, None, None, 2, None, 0),
+        lib.psc_state_init(None, 4, 16, None, ctypes.byref(out)),
+    ]
+    assert cases == [1] * len(cases), cases
+    assert lib.psc_last_error()
+    assert lib.psc_host_classify(None, 0, None, 0, 0) == -1
+    assert lib.psc_host_classify_bottom_up(None, 0, None, 0, 0) == -1
+
+
 def test_device_calls_refuse_host_only_handle(psc):
     h = psc.psc_compile(grammars.arithmetic().text(), [b"1", b""], 1, host_only=True)
     with pytest.raises(psc.PscError) as e:
