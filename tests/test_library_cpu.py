@@ -5,6 +5,7 @@ from __future__ import annotations
 
 import os
 import re
+import sys
 
 import numpy as np
 import pytest
@@ -487,6 +488,21 @@ def test_binding_refuses_short_or_host_arrays(psc):
             psc.psc_decode_step_advance(h, st, tokens)
     with pytest.raises(ValueError):
         psc.psc_state_reset(st, torch.zeros(3, dtype=torch.int64))
+
+
+def test_binding_fails_loudly_without_the_library(tmp_path):
+    """No fallback: a binding that cannot find the compiled library raises."""
+    import importlib.util
+    spec = importlib.util.spec_from_file_location(
+        "psc_fresh", os.path.join(ROOT, "paper_2608_03065_gb300", "psc.py"))
+    fresh = importlib.util.module_from_spec(spec)
+    sys.modules["psc_fresh"] = fresh   # dataclasses look their module up there
+    try:
+        spec.loader.exec_module(fresh)
+        with pytest.raises(RuntimeError, match="missing"):
+            fresh.load(str(tmp_path / "libpsc_gb300.so"))
+    finally:
+        del sys.modules["psc_fresh"]
 
 
 def test_c_abi_argument_errors(psc):
