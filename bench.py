@@ -7,9 +7,11 @@ that the masking kernel can be timed on its own):
                    place, write the packed bitmask [B][V/32] and pick the greedy
                    token among the allowed ones, in one TMA-pipelined pass
   k_advance_warp   lex + parse the chosen tokens on the device-resident stacks
-                   and classify the new configurations (classifier DFA walk)
+                   and classify the new configurations (bottom-up classifier:
+                   only the stack entries the step changed are re-read)
 
 Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+                       [--mode teacher | sweep]
 For N > 1 launch with torch.distributed.run: every rank runs an independent
 replica (the rows of different sequences are independent; no collective on the
 data path) and the step rate is summed over ranks (weak scaling).
