@@ -97,15 +97,36 @@ bool lex_token(const Lexer& L, int q, const uint8_t* b, int64_t len, std::vector
 }
 
 struct LocalTrie {
-    std::unordered_map<uint64_t, int32_t> edge;
+    // edges (node, class) -> child in an open-addressing table (keys ~0 = empty)
+    std::vector<uint64_t> keys = std::vector<uint64_t>(1024, ~0ull);
+    std::vector<int32_t> vals = std::vector<int32_t>(1024, 0);
+    size_t used = 0;
     std::vector<std::pair<int32_t, int32_t>> toks;  // (node, token)
     int32_t n = 1;
+    static uint64_t key_of(int32_t node, int cls) { return ((uint64_t)(uint32_t)node << 24) | (uint32_t)(cls + 1); }
     int32_t child(int32_t node, int cls) {
-        uint64_t key = ((uint64_t)(uint32_t)node << 24) | (uint32_t)(cls + 1);
-        auto it = edge.find(key);
-        if (it != edge.end()) return it->second;
-        edge.emplace(key, n);
+        uint64_t key = key_of(node, cls);
+        size_t m = keys.size() - 1, i = mix64(key) & m;
+        for (; keys[i] != ~0ull; i = (i + 1) & m)
+            if (keys[i] == key) return vals[i];
+        keys[i] = key;
+        vals[i] = n;
+        if (++used * 2 > keys.size()) grow();
         return n++;
+    }
+    void grow() {
+        std::vector<uint64_t> k2(keys.size() * 2, ~0ull);
+        std::vector<int32_t> v2(keys.size() * 2, 0);
+        size_t m = k2.size() - 1;
+        for (size_t j = 0; j < keys.size(); j++) {
+            if (keys[j] == ~0ull) continue;
+            size_t i = mix64(keys[j]) & m;
+            while (k2[i] != ~0ull) i = (i + 1) & m;
+            k2[i] = keys[j];
+            v2[i] = vals[j];
+        }
+        keys.swap(k2);
+        vals.swap(v2);
     }
 };
 
@@ -153,8 +174,10 @@ Trie build_tries(const Lexer& L, const uint8_t* vb, const int64_t* vo, int V, in
         LocalTrie& T = local[q];
         tr.root.push_back(base);
         std::vector<std::tuple<int32_t, int32_t, int32_t>> edges;  // parent, cls, child
-        edges.reserve(T.edge.size());
-        for (auto& [key, ch] : T.edge) edges.emplace_back((int32_t)(key >> 24), (int32_t)(key & 0xFFFFFF) - 1, ch);
+        edges.reserve(T.used);
+        for (size_t j = 0; j < T.keys.size(); j++)
+            if (T.keys[j] != ~0ull)
+                edges.emplace_back((int32_t)(T.keys[j] >> 24), (int32_t)(T.keys[j] & 0xFFFFFF) - 1, T.vals[j]);
         std::sort(edges.begin(), edges.end());
         std::sort(T.toks.begin(), T.toks.end());
         T.toks.erase(std::unique(T.toks.begin(), T.toks.end()), T.toks.end());
@@ -170,7 +193,8 @@ Trie build_tries(const Lexer& L, const uint8_t* vb, const int64_t* vo, int V, in
             tr.tok_off.push_back((int32_t)tr.toks.size());
         }
         base += T.n;
-        LocalTrie().edge.swap(T.edge);
+        std::vector<uint64_t>().swap(T.keys);
+        std::vector<int32_t>().swap(T.vals);
         std::vector<std::pair<int32_t, int32_t>>().swap(T.toks);
     }
     return tr;
