@@ -500,28 +500,56 @@ void Builder::expand(int32_t n, const int32_t* g, int glen) {
 
 }  // namespace
 
-void set_mask_rows(Tables& t, const uint32_t* rows, int n, int W) {
+namespace {
+
+// The chunk table of mask rows given by pointer (row m = rows[m], W words):
+// chunk hashes are computed in parallel, then chunk ids are given serially in
+// the order chunks are first met (row by row), so the result does not depend on
+// the thread count.
+void set_mask_rows_from(Tables& t, const std::vector<const uint32_t*>& rows, int W, int threads) {
+    int n = (int)rows.size();
     int nch = (W + 31) / 32;
     t.W = W;
     t.n_masks = n;
     t.nch = nch;
     t.mask_rows.assign((size_t)n * nch, 0);
     t.mask_chunks.clear();
-    // open addressing over chunk contents (64-bit FNV-1a of the 32 words)
+    auto load_chunk = [&](int m, int c, uint32_t* chunk) {
+        int w0 = c * 32, nw = std::min(32, W - w0);
+        std::memcpy(chunk, rows[m] + w0, sizeof(uint32_t) * nw);
+        for (int k = nw; k < 32; k++) chunk[k] = 0;
+    };
+    auto fnv = [](const uint32_t* chunk) {
+        uint64_t h = 1469598103934665603ull;
+        for (int k = 0; k < 32; k++) h = (h ^ chunk[k]) * 1099511628211ull;
+        return h;
+    };
+    std::vector<uint64_t> hs((size_t)n * nch);
+    {
+        std::atomic<int> next{0};
+        auto work = [&]() {
+            uint32_t chunk[32];
+            for (int m; (m = next.fetch_add(1)) < n;)
+                for (int c = 0; c < nch; c++) {
+                    load_chunk(m, c, chunk);
+                    hs[(size_t)m * nch + c] = fnv(chunk);
+                }
+        };
+        std::vector<std::thread> pool;
+        for (int i = 0; i < std::max(1, threads); i++) pool.emplace_back(work);
+        for (auto& th : pool) th.join();
+    }
+    // open addressing over chunk contents (load factor below 1/2)
     size_t cap = 1024;
     while (cap < (size_t)n * nch / 4 + 1024) cap <<= 1;
     std::vector<int64_t> slot(cap, -1);
     std::vector<uint64_t> slot_hash(cap, 0);
     uint32_t chunk[32];
     for (int m = 0; m < n; m++) {
-        const uint32_t* row = rows + (size_t)m * W;
         for (int c = 0; c < nch; c++) {
-            int w0 = c * 32, nw = std::min(32, W - w0);
-            std::memcpy(chunk, row + w0, sizeof(uint32_t) * nw);
-            for (int k = nw; k < 32; k++) chunk[k] = 0;
-            uint64_t h = 1469598103934665603ull;
-            for (int k = 0; k < 32; k++) h = (h ^ chunk[k]) * 1099511628211ull;
-            if ((size_t)t.mask_chunks.size() / 32 * 2 >= cap) {   // keep the load factor below 1/2
+            uint64_t h = hs[(size_t)m * nch + c];
+            load_chunk(m, c, chunk);
+            if ((size_t)t.mask_chunks.size() / 32 * 2 >= cap) {
                 size_t ncap = cap << 1;
                 std::vector<int64_t> ns(ncap, -1);
                 std::vector<uint64_t> nh(ncap, 0);
@@ -556,6 +584,14 @@ void set_mask_rows(Tables& t, const uint32_t* rows, int n, int W) {
         }
     }
     t.n_chunks = (int)(t.mask_chunks.size() / 32);
+}
+
+}  // namespace
+
+void set_mask_rows(Tables& t, const uint32_t* rows, int n, int W) {
+    std::vector<const uint32_t*> ptr(n);
+    for (int m = 0; m < n; m++) ptr[m] = rows + (size_t)m * W;
+    set_mask_rows_from(t, ptr, W, (int)std::max(1u, std::thread::hardware_concurrency()));
 }
 
 Tables compile_tables(const std::string& text, const uint8_t* vb, const int64_t* vo, int V, int eos_id,
@@ -835,13 +871,14 @@ Tables compile_tables(const std::string& text, const uint8_t* vb, const int64_t*
     T.dfa_start.resize(L.nq);
     for (int q = 0; q < L.nq; q++) T.dfa_start[q] = enc(cls[start_state[q]]);
     T.V = V;
+    double t5 = now();
     {
-        std::vector<uint32_t> dense((size_t)n_masks * W, 0);
+        std::vector<const uint32_t*> rows_by_id(n_masks, nullptr);   // final mask id -> its pool row
         for (size_t m = 0; m < mask_new.size(); m++)
-            if (mask_new[m] >= 0)
-                std::memcpy(dense.data() + (size_t)mask_new[m] * W, grows.data() + m * W, sizeof(uint32_t) * W);
-        set_mask_rows(T, dense.data(), n_masks, W);
+            if (mask_new[m] >= 0) rows_by_id[mask_new[m]] = grows.data() + m * W;
+        set_mask_rows_from(T, rows_by_id, W, threads);
     }
+    double t6 = now();
 
     // lexer and parser tables for the device
     T.nq = L.nq;
@@ -880,8 +917,8 @@ Tables compile_tables(const std::string& text, const uint8_t* vb, const int64_t*
     T.seconds_total = now() - t0;
     if (getenv("PSC_LOG"))
         fprintf(stderr, "psc: compile %.2f s: grammar+lexer+LALR %.2f s, token tries %.2f s, classifier %.2f s, "
-                        "minimisation %.2f s, flatten+bottom-up %.2f s\n",
-                T.seconds_total, t1 - t0, t2 - t1, t3 - t2, t4 - t3, T.seconds_total - (t4 - t0));
+                        "minimisation %.2f s, flatten+bottom-up %.2f s (mask rows %.2f s)\n",
+                T.seconds_total, t1 - t0, t2 - t1, t3 - t2, t4 - t3, T.seconds_total - (t4 - t0), t6 - t5);
     return T;
 }
 
