@@ -165,38 +165,71 @@ Trie build_tries(const Lexer& L, const uint8_t* vb, const int64_t* vo, int V, in
             }
         }
     };
+    double t0 = now();
     std::vector<std::thread> pool;
     for (int i = 0; i < threads; i++) pool.emplace_back(work);
     for (auto& t : pool) t.join();
-    Trie tr;
-    int32_t base = 0;
-    for (int q = 0; q < nq; q++) {
-        LocalTrie& T = local[q];
-        tr.root.push_back(base);
-        std::vector<std::tuple<int32_t, int32_t, int32_t>> edges;  // parent, cls, child
-        edges.reserve(T.used);
-        for (size_t j = 0; j < T.keys.size(); j++)
-            if (T.keys[j] != ~0ull)
-                edges.emplace_back((int32_t)(T.keys[j] >> 24), (int32_t)(T.keys[j] & 0xFFFFFF) - 1, T.vals[j]);
-        std::sort(edges.begin(), edges.end());
-        std::sort(T.toks.begin(), T.toks.end());
-        T.toks.erase(std::unique(T.toks.begin(), T.toks.end()), T.toks.end());
-        size_t e = 0, k = 0;
-        for (int32_t nd = 0; nd < T.n; nd++) {
-            while (e < edges.size() && std::get<0>(edges[e]) == nd) {
-                tr.child_cls.push_back(std::get<1>(edges[e]));
-                tr.child_node.push_back(base + std::get<2>(edges[e]));
-                e++;
+    double t1 = now();
+    // each lexer state's part laid out on its own (in parallel), then concatenated
+    struct Part {
+        std::vector<int32_t> child_cls, child_node, child_cnt, toks, tok_cnt;
+    };
+    std::vector<Part> parts(nq);
+    std::vector<int32_t> base(nq + 1, 0);
+    for (int q = 0; q < nq; q++) base[q + 1] = base[q] + local[q].n;
+    {
+        std::atomic<int> next_q{0};
+        auto lay_out = [&]() {
+            for (int q; (q = next_q.fetch_add(1)) < nq;) {
+                LocalTrie& T = local[q];
+                Part& P = parts[q];
+                std::vector<std::tuple<int32_t, int32_t, int32_t>> edges;  // parent, cls, child
+                edges.reserve(T.used);
+                for (size_t j = 0; j < T.keys.size(); j++)
+                    if (T.keys[j] != ~0ull)
+                        edges.emplace_back((int32_t)(T.keys[j] >> 24), (int32_t)(T.keys[j] & 0xFFFFFF) - 1, T.vals[j]);
+                std::sort(edges.begin(), edges.end());
+                std::sort(T.toks.begin(), T.toks.end());
+                T.toks.erase(std::unique(T.toks.begin(), T.toks.end()), T.toks.end());
+                P.child_cnt.assign(T.n, 0);
+                P.tok_cnt.assign(T.n, 0);
+                for (auto& [parent, cls, ch] : edges) {
+                    P.child_cls.push_back(cls);
+                    P.child_node.push_back(base[q] + ch);
+                    P.child_cnt[parent]++;
+                }
+                for (auto& [node, tok] : T.toks) {
+                    P.toks.push_back(tok);
+                    P.tok_cnt[node]++;
+                }
+                std::vector<uint64_t>().swap(T.keys);
+                std::vector<int32_t>().swap(T.vals);
+                std::vector<std::pair<int32_t, int32_t>>().swap(T.toks);
             }
-            tr.child_off.push_back((int32_t)tr.child_cls.size());
-            while (k < T.toks.size() && T.toks[k].first == nd) tr.toks.push_back(T.toks[k++].second);
-            tr.tok_off.push_back((int32_t)tr.toks.size());
-        }
-        base += T.n;
-        std::vector<uint64_t>().swap(T.keys);
-        std::vector<int32_t>().swap(T.vals);
-        std::vector<std::pair<int32_t, int32_t>>().swap(T.toks);
+        };
+        std::vector<std::thread> workers;
+        for (int i = 0; i < threads; i++) workers.emplace_back(lay_out);
+        for (auto& t : workers) t.join();
     }
+    Trie tr;
+    for (int q = 0; q < nq; q++) {
+        Part& P = parts[q];
+        tr.root.push_back(base[q]);
+        tr.child_cls.insert(tr.child_cls.end(), P.child_cls.begin(), P.child_cls.end());
+        tr.child_node.insert(tr.child_node.end(), P.child_node.begin(), P.child_node.end());
+        tr.toks.insert(tr.toks.end(), P.toks.begin(), P.toks.end());
+        int32_t co = tr.child_off.back(), to = tr.tok_off.back();
+        for (int32_t nd = 0; nd < (int32_t)P.child_cnt.size(); nd++) {
+            co += P.child_cnt[nd];
+            to += P.tok_cnt[nd];
+            tr.child_off.push_back(co);
+            tr.tok_off.push_back(to);
+        }
+        Part().child_cls.swap(P.child_cls);
+        P = Part();
+    }
+    if (getenv("PSC_LOG"))
+        fprintf(stderr, "psc: token tries: %d nodes, lexing %.2f s, merging %.2f s\n", tr.n(), t1 - t0, now() - t1);
     return tr;
 }
 
