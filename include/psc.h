@@ -278,7 +278,7 @@ int32_t psc_host_classify(const psc_handle* h, int32_t q, const uint16_t* h_stac
  * bad arguments, or -2 when the handle has no bottom-up classifier or the
  * stack is not a path of the LR automaton (no parser builds such a stack).
  * States objects keep this automaton's state after every stack prefix of
- * every row, so a decode step re-reads only the entries it pushed. */
+ * every row, so a decode step re-reads only the stack entries it changed. */
 int32_t psc_host_classify_bottom_up(const psc_handle* h, int32_t q, const uint16_t* h_stack, int32_t depth,
                                     int32_t status);
 psc_status psc_host_mask_row(const psc_handle* h, int32_t mask_id, uint32_t* h_row);
