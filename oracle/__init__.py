@@ -3,4 +3,4 @@
 Only ``tests/``, ``__graft_entry__.smoke()`` and the CPU-baseline leg of
 ``bench.py`` may import it.  It shares no code with the CUDA path.
 """
-from .psc_oracle import Config, Oracle, Vocab, ST_OK, ST_DONE, ST_ERROR  # noqa: F401
+from .psc_oracle import Config, Oracle, OracleLimitError, Vocab, ST_OK, ST_DONE, ST_ERROR  # noqa: F401

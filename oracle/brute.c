@@ -33,7 +33,36 @@
 
 enum { K_ERR = 0, K_SHIFT = 1, K_REDUCE = 2, K_ACCEPT = 3 };
 enum { ST_OK = 0, ST_DONE = 1, ST_ERROR = 2 };
-enum { MAX_CLASS = 32, MAX_EMIT = 256, LOC_MAX = 8192 };
+
+/* Capacities of the checker.  None of them is part of the method: reaching one
+ * is a failure of the checker, never a "token not allowed".  Each sets a bit of
+ * the worker's error word, the call that hit it returns that word (negated or
+ * as its result) and the Python wrapper raises.  They can be set at build time
+ * so that a test can reach each of them on a small grammar. */
+#ifndef ORACLE_MAX_CLASS
+#define ORACLE_MAX_CLASS 32      /* terminals in one lexeme class */
+#endif
+#ifndef ORACLE_MAX_EMIT
+#define ORACLE_MAX_EMIT 256      /* classes emitted while lexing one token */
+#endif
+#ifndef ORACLE_LOC_MAX
+#define ORACLE_LOC_MAX 8192      /* entries pushed above the row's stack while checking one token */
+#endif
+#ifndef ORACLE_TP_SLOTS
+#define ORACLE_TP_SLOTS 1024     /* pending lexemes whose T_p a worker keeps */
+#endif
+#ifndef ORACLE_MAX_STEPS
+#define ORACLE_MAX_STEPS 10000000L  /* parser actions while feeding one terminal */
+#endif
+enum { MAX_CLASS = ORACLE_MAX_CLASS, MAX_EMIT = ORACLE_MAX_EMIT, LOC_MAX = ORACLE_LOC_MAX };
+enum {
+    ERR_CLASS = 1,     /* a class with more than MAX_CLASS terminals */
+    ERR_MIXED = 2,     /* a lexeme matched by an ignored and a kept terminal (a grammar error) */
+    ERR_EMIT = 4,      /* more than MAX_EMIT classes from one token */
+    ERR_LOC = 8,       /* more than LOC_MAX pushed entries */
+    ERR_TP_CACHE = 16, /* the T_p cache is full */
+    ERR_STEPS = 32     /* more than ORACLE_MAX_STEPS parser actions for one terminal */
+};
 
 typedef struct {
     int n_nfa, words, nfa_start;
@@ -64,6 +93,7 @@ typedef struct {
 typedef struct {
     const OTables *T;
     int32_t *dfs;
+    int *err;   /* the worker's error word */
 } Lex;
 
 static int set_empty(const uint64_t *a, int w) {
@@ -118,8 +148,9 @@ static void set_step(Lex *L, const uint64_t *cur, int byte, uint64_t *out) {
 }
 
 /* The class of a set: all terminals accepted in it, sorted by rank.  Returns
- * the count (0 = not complete), or -1 if ignored and kept terminals mix. */
-static int set_class(const OTables *T, const uint64_t *set, int32_t *cls) {
+ * the count (0 = not complete), or -1 (with a bit of *err set) if the class
+ * overflows or ignored and kept terminals mix. */
+static int set_class(const OTables *T, const uint64_t *set, int32_t *cls, int *err) {
     int n = 0;
     for (int i = 0; i < T->words; i++) {
         uint64_t m = set[i];
@@ -131,7 +162,10 @@ static int set_class(const OTables *T, const uint64_t *set, int32_t *cls) {
             int dup = 0;
             for (int k = 0; k < n; k++) dup |= cls[k] == t;
             if (!dup) {
-                if (n == MAX_CLASS) return -1;
+                if (n == MAX_CLASS) {
+                    *err |= ERR_CLASS;
+                    return -1;
+                }
                 cls[n++] = t;
             }
         }
@@ -147,7 +181,10 @@ static int set_class(const OTables *T, const uint64_t *set, int32_t *cls) {
     }
     int ign = 0;
     for (int k = 0; k < n; k++) ign += T->term_ignored[cls[k]];
-    if (ign && ign != n) return -1;
+    if (ign && ign != n) {
+        *err |= ERR_MIXED;
+        return -1;
+    }
     return n;
 }
 
@@ -173,11 +210,14 @@ static int lex_bytes(Lex *L, uint64_t *pend, int *plen, const uint8_t *bytes, in
         }
         if (*plen == 0) return -1;
         Class cl;
-        cl.n = set_class(T, pend, cl.t);
+        cl.n = set_class(T, pend, cl.t, L->err);
         if (cl.n <= 0) return -1;
         cl.ignored = T->term_ignored[cl.t[0]];
         if (!cl.ignored) {
-            if (n_out == MAX_EMIT) return -1;
+            if (n_out == MAX_EMIT) {
+                *L->err |= ERR_EMIT;
+                return -1;
+            }
             out[n_out++] = cl;
         }
         set_start(L, pend);
@@ -227,7 +267,7 @@ static int tp_explore(Lex *L, const uint64_t *p, TpSet *res) {
     int rc = 0;
     for (int i = 0; i < n; i++) {
         Class cl;
-        cl.n = set_class(T, seen + (size_t)i * w, cl.t);
+        cl.n = set_class(T, seen + (size_t)i * w, cl.t, L->err);
         if (cl.n < 0) { rc = -1; break; }
         if (cl.n > 0) {
             cl.ignored = T->term_ignored[cl.t[0]];
@@ -279,7 +319,8 @@ static const TpSet *tp_lookup(Lex *L, TpCache *C, const uint64_t *p) {
         }
         if (!memcmp(C->keys + (size_t)s * w, p, sizeof(uint64_t) * w)) return &C->vals[s];
     }
-    return NULL; /* cache full: caller treats as an error */
+    *L->err |= ERR_TP_CACHE;
+    return NULL;
 }
 
 /* ------------------------------------------------------- parser simulation */
@@ -288,6 +329,7 @@ typedef struct {
     const int32_t *base;
     int base_top;           /* entries base[0..base_top) are still on the stack */
     int nloc;
+    int *err;               /* the worker's error word */
     int32_t loc[LOC_MAX];   /* pushed on top of base[0..base_top) */
 } Ov;
 
@@ -304,14 +346,17 @@ static int ov_pop(Ov *o, int k) {
 }
 
 static int ov_push(Ov *o, int s) {
-    if (o->nloc == LOC_MAX) return -1;
+    if (o->nloc == LOC_MAX) {
+        *o->err |= ERR_LOC;
+        return -1;
+    }
     o->loc[o->nloc++] = s;
     return 0;
 }
 
 /* Feed terminal t: reductions until t is shifted (1), accepted (2) or rejected (0). */
 static int feed_terminal(const OTables *T, Ov *o, int t) {
-    for (long guard = 0; guard < 10000000L; guard++) {
+    for (long guard = 0; guard < ORACLE_MAX_STEPS; guard++) {
         int s = ov_top(o);
         int k = T->act_kind[(size_t)s * T->n_terms + t];
         int v = T->act_val[(size_t)s * T->n_terms + t];
@@ -322,6 +367,7 @@ static int feed_terminal(const OTables *T, Ov *o, int t) {
         int g = T->go[(size_t)ov_top(o) * T->n_nt + T->rule_lhs[v]];
         if (g < 0 || ov_push(o, g) < 0) return 0;
     }
+    *o->err |= ERR_STEPS;
     return 0;
 }
 
@@ -347,13 +393,17 @@ typedef struct {
     uint64_t *pend, *tmp;
     Class *emit;
     Ov ov, ov2;
+    int err;   /* capacity failures (ERR_* bits) since the worker was made */
 } Worker;
 
 static void worker_init(Worker *W, const OTables *T) {
     memset(W, 0, sizeof(*W));
     W->L.T = T;
+    W->L.err = &W->err;
+    W->ov.err = &W->err;
+    W->ov2.err = &W->err;
     W->L.dfs = malloc(sizeof(int32_t) * (T->n_nfa + 1) * 2);
-    W->cache.slots = 1024;
+    W->cache.slots = ORACLE_TP_SLOTS;
     W->cache.keys = malloc(sizeof(uint64_t) * T->words * W->cache.slots);
     W->cache.used = calloc(W->cache.slots, sizeof(int));
     W->cache.vals = malloc(sizeof(TpSet) * W->cache.slots);
@@ -381,6 +431,7 @@ static void ov_init(Ov *o, const OConfig *c) {
 }
 
 static void ov_copy(Ov *dst, const Ov *src) {
+    dst->err = src->err;
     dst->base = src->base;
     dst->base_top = src->base_top;
     dst->nloc = src->nloc;
@@ -395,7 +446,7 @@ static int check_eos(Worker *W, const OConfig *c) {
     ov_init(&W->ov, c);
     if (c->pend_len > 0) {
         Class cl;
-        cl.n = set_class(T, c->pend, cl.t);
+        cl.n = set_class(T, c->pend, cl.t, &W->err);
         if (cl.n <= 0) return 0;
         if (!T->term_ignored[cl.t[0]] && !feed_class(T, &W->ov, &cl)) return 0;
     }
@@ -428,7 +479,8 @@ static int check_token(Worker *W, const OConfig *c, const uint8_t *bytes, int le
 
 OConfig *oracle_config_new(const OTables *T, int cap) {
     OConfig *c = calloc(1, sizeof(OConfig));
-    Lex L = {T, malloc(sizeof(int32_t) * (T->n_nfa + 1) * 2)};
+    int err = 0;
+    Lex L = {T, malloc(sizeof(int32_t) * (T->n_nfa + 1) * 2), &err};
     c->pend = malloc(sizeof(uint64_t) * T->words);
     set_start(&L, c->pend);
     free(L.dfs);
@@ -471,12 +523,19 @@ int oracle_config_pending(const OTables *T, const OConfig *c, uint64_t *out_word
 }
 
 /* Commit one token (is_eos: the end-of-sequence token).  A token the mask does
- * not allow moves the row to the error status.  Returns the new status. */
+ * not allow moves the row to the error status.  Returns the new status, or
+ * -(ERR_* bits) with the row unchanged if a capacity of the checker ran out. */
 int oracle_advance(const OTables *T, OConfig *c, const uint8_t *bytes, int len, int is_eos) {
     if (c->status == ST_ERROR) return c->status;
     Worker *W = malloc(sizeof(Worker));
     worker_init(W, T);
     int allowed = is_eos ? check_eos(W, c) : check_token(W, c, bytes, len);
+    if (W->err) {
+        int e = W->err;
+        worker_free(W);
+        free(W);
+        return -e;
+    }
     if (!allowed) {
         c->status = ST_ERROR;
     } else if (is_eos) {
@@ -511,6 +570,7 @@ typedef struct {
     const int64_t *vo;
     uint32_t *out;
     int tid, nthreads;
+    int err;   /* the worker's error word when it finished */
 } Job;
 
 static void *mask_worker(void *arg) {
@@ -527,15 +587,18 @@ static void *mask_worker(void *arg) {
         if (c->status == ST_DONE) ok = v == J->eos_id;
         else if (v == J->eos_id) ok = check_eos(W, c);
         else ok = check_token(W, c, J->vb + J->vo[v], (int)(J->vo[v + 1] - J->vo[v]));
+        if (W->err) break;
         if (ok) __atomic_fetch_or(&J->out[(size_t)b * J->W + (v >> 5)], 1u << (v & 31), __ATOMIC_RELAXED);
     }
+    J->err = W->err;
     worker_free(W);
     free(W);
     return NULL;
 }
 
 /* Masks of B rows over a vocabulary of V tokens (token v = vb[vo[v]..vo[v+1])),
- * packed LSB-first into out[B][ceil(V/32)] (bits v >= V stay zero). */
+ * packed LSB-first into out[B][ceil(V/32)] (bits v >= V stay zero).  Returns 0,
+ * or the ERR_* bits of the capacities that ran out (the masks are then void). */
 int oracle_masks(const OTables *T, OConfig *const *rows, int B, const uint8_t *vb,
                  const int64_t *vo, int V, int eos_id, uint32_t *out, int nthreads) {
     int W = (V + 31) / 32;
@@ -544,16 +607,21 @@ int oracle_masks(const OTables *T, OConfig *const *rows, int B, const uint8_t *v
     pthread_t *th = malloc(sizeof(pthread_t) * nthreads);
     Job *jobs = malloc(sizeof(Job) * nthreads);
     for (int t = 0; t < nthreads; t++) {
-        jobs[t] = (Job){T, rows, B, V, W, eos_id, vb, vo, out, t, nthreads};
+        jobs[t] = (Job){T, rows, B, V, W, eos_id, vb, vo, out, t, nthreads, 0};
         pthread_create(&th[t], NULL, mask_worker, &jobs[t]);
     }
-    for (int t = 0; t < nthreads; t++) pthread_join(th[t], NULL);
+    int err = 0;
+    for (int t = 0; t < nthreads; t++) {
+        pthread_join(th[t], NULL);
+        err |= jobs[t].err;
+    }
     free(th);
     free(jobs);
-    return 0;
+    return err;
 }
 
-/* One (row, token) decision; used to sample outputs of large workloads. */
+/* One (row, token) decision; used to sample outputs of large workloads.
+ * Returns 1 / 0, or -(ERR_* bits) if a capacity of the checker ran out. */
 int oracle_allowed(const OTables *T, const OConfig *c, const uint8_t *bytes, int len,
                    int is_eos) {
     Worker *W = malloc(sizeof(Worker));
@@ -562,6 +630,7 @@ int oracle_allowed(const OTables *T, const OConfig *c, const uint8_t *bytes, int
     if (c->status == ST_DONE) ok = is_eos;
     else if (is_eos) ok = check_eos(W, c);
     else ok = check_token(W, c, bytes, len);
+    if (W->err) ok = -W->err;
     worker_free(W);
     free(W);
     return ok;

@@ -44,18 +44,36 @@ _lib = None
 
 ST_OK, ST_DONE, ST_ERROR = 0, 1, 2
 
+# bits of the checker's error word (brute.c): a capacity of the checker ran out
+# (or the grammar mixes ignored and kept terminals in one lexeme); never a mask bit
+ERRORS = {1: "a lexeme class has too many terminals", 2: "a lexeme matches an ignored and a kept terminal",
+          4: "a token emits too many lexemes", 8: "too many stack entries pushed while checking a token",
+          16: "the T_p cache is full", 32: "too many parser actions for one terminal"}
 
-def build_library(force: bool = False) -> str:
-    """Compile brute.c (plain C, pthreads) next to this file."""
+
+class OracleLimitError(RuntimeError):
+    """The oracle could not decide: one of its checker's capacities ran out."""
+
+    def __init__(self, bits: int):
+        super().__init__("oracle capacity exceeded: " +
+                         "; ".join(m for b, m in ERRORS.items() if bits & b))
+        self.bits = bits
+
+
+def build_library(force: bool = False, defines: dict | None = None, path: str | None = None) -> str:
+    """Compile brute.c (plain C, pthreads) next to this file.  ``defines``
+    overrides the checker's capacities (ORACLE_* macros) in a build at ``path``."""
     src = os.path.join(_HERE, "brute.c")
-    if not force and os.path.exists(_LIB_PATH) and os.path.getmtime(_LIB_PATH) >= os.path.getmtime(src):
-        return _LIB_PATH
-    os.makedirs(_BUILD, exist_ok=True)
-    tmp = _LIB_PATH + f".{os.getpid()}.tmp"
-    subprocess.check_call(["gcc", "-O2", "-std=c11", "-shared", "-fPIC", "-pthread",
+    out = path or _LIB_PATH
+    if not force and os.path.exists(out) and os.path.getmtime(out) >= os.path.getmtime(src):
+        return out
+    os.makedirs(os.path.dirname(out), exist_ok=True)
+    tmp = out + f".{os.getpid()}.tmp"
+    flags = [f"-D{k}={v}" for k, v in (defines or {}).items()]
+    subprocess.check_call(["gcc", "-O2", "-std=c11", "-shared", "-fPIC", "-pthread", *flags,
                            "-o", tmp, src])
-    os.replace(tmp, _LIB_PATH)
-    return _LIB_PATH
+    os.replace(tmp, out)
+    return out
 
 
 def _load():
@@ -202,8 +220,12 @@ class Oracle:
     def advance(self, cfg: Config, token: bytes | None) -> int:
         """Commit one token in place (``None`` = end of sequence); returns the status."""
         if token is None:
-            return _load().oracle_advance(ctypes.byref(self._t), cfg._p, b"", 0, 1)
-        return _load().oracle_advance(ctypes.byref(self._t), cfg._p, token, len(token), 0)
+            r = _load().oracle_advance(ctypes.byref(self._t), cfg._p, b"", 0, 1)
+        else:
+            r = _load().oracle_advance(ctypes.byref(self._t), cfg._p, token, len(token), 0)
+        if r < 0:
+            raise OracleLimitError(-r)
+        return r
 
     def advance_tokens(self, cfg: Config, vocab: Vocab, ids) -> int:
         st = ST_OK
@@ -214,8 +236,12 @@ class Oracle:
 
     def allowed(self, cfg: Config, token: bytes | None) -> bool:
         if token is None:
-            return bool(_load().oracle_allowed(ctypes.byref(self._t), cfg._p, b"", 0, 1))
-        return bool(_load().oracle_allowed(ctypes.byref(self._t), cfg._p, token, len(token), 0))
+            r = _load().oracle_allowed(ctypes.byref(self._t), cfg._p, b"", 0, 1)
+        else:
+            r = _load().oracle_allowed(ctypes.byref(self._t), cfg._p, token, len(token), 0)
+        if r < 0:
+            raise OracleLimitError(-r)
+        return bool(r)
 
     # ------------------------------------------------------------------ masks
     def masks(self, cfgs: list[Config], vocab: Vocab, threads: int | None = None) -> np.ndarray:
@@ -225,8 +251,10 @@ class Oracle:
         out = np.zeros((B, W), dtype=np.uint32)
         arr = (ctypes.c_void_p * max(B, 1))(*[c._p for c in cfgs])
         threads = threads or os.cpu_count() or 1
-        _load().oracle_masks(ctypes.byref(self._t), arr, B, vocab.blob.ctypes.data,
-                             vocab.offsets.ctypes.data, V, vocab.eos_id, out.ctypes.data, threads)
+        err = _load().oracle_masks(ctypes.byref(self._t), arr, B, vocab.blob.ctypes.data,
+                                   vocab.offsets.ctypes.data, V, vocab.eos_id, out.ctypes.data, threads)
+        if err:
+            raise OracleLimitError(err)
         return out
 
     def mask_set(self, cfg: Config, vocab: Vocab) -> set[int]:
