@@ -24,20 +24,25 @@ def test_vocabulary_and_prefixes(cfg_id, batch):
     assert max(len(t) for t in w.vocab) <= s.vocab_max_len
     assert all(len(t) >= 1 for t in w.vocab[:-1])
     assert len(w.prefixes) == len(w.prefix_ids) == w.B == (batch or s.B)
-    o = None
     for p, ids in zip(w.prefixes, w.prefix_ids):
-        assert 1 <= len(p) <= s.prefix_max
-        if len(p) < s.prefix_min:   # the drawn length is a target: a sentence that ends first is kept whole
-            if o is None:
-                from oracle import Oracle
-                o = Oracle(w.grammar_text)
-            c = o.initial()
-            o.advance(c, p)
-            assert o.allowed(c, None), p
+        assert s.prefix_min <= len(p) <= s.prefix_max        # the drawn length, never a shorter sentence
         assert b"".join(w.vocab[i] for i in ids) == p        # greedy tokenization is exact
         assert w.eos_id not in ids
     m = w.token_matrix()
     assert m.shape[0] == w.B and m.dtype == np.int32
+
+
+@pytest.mark.parametrize("cfg_id", [1, 2])
+def test_prefix_lengths_are_uniform_over_the_range(cfg_id):
+    """Prefix lengths are drawn uniformly in [prefix_min, prefix_max] (a sentence
+    that ends before its drawn length is drawn again): the lengths spread over the
+    whole range instead of piling up at the short sentences."""
+    w = configs.load(cfg_id)
+    s = configs.SPECS[cfg_id]
+    L = np.array([len(p) for p in w.prefixes])
+    lo, hi = s.prefix_min, s.prefix_max
+    assert np.quantile(L, 0.75) > lo + 0.5 * (hi - lo)
+    assert np.quantile(L, 0.25) < lo + 0.5 * (hi - lo)
 
 
 def test_inputs_are_deterministic():

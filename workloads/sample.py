@@ -209,14 +209,20 @@ class TrieTokenizer:
 
 # ---------------------------------------------------------------------- prefixes
 def build_prefixes(spec: GrammarSpec, n: int, min_len: int, max_len: int, seed_key,
-                   max_depth: int = 40, nest_bias: float = 1.0) -> list[bytes]:
-    """``n`` prefixes of sampled sentences, each cut at a uniform length in
-    [min_len, max_len] bytes (or the whole sentence when it ends first)."""
+                   max_depth: int = 40, nest_bias: float = 1.0, max_draws: int = 100000) -> list[bytes]:
+    """``n`` prefixes of sampled sentences, each exactly a uniform length in
+    [min_len, max_len] bytes: a sentence is drawn again until it reaches the
+    drawn length, then cut there (so short sentences do not skew the lengths)."""
     rng = np.random.default_rng(seed_key)
     sampler = SentenceSampler(spec, max_depth=max_depth, nest_bias=nest_bias)
     out = []
     for _ in range(n):
         target = int(rng.integers(min_len, max_len + 1))
-        txt, finished = sampler.text(rng, target)
+        for _ in range(max_draws):
+            txt, _ = sampler.text(rng, target)
+            if len(txt) >= target:
+                break
+        else:
+            raise RuntimeError(f"no sentence of {spec.name} reached {target} bytes in {max_draws} draws")
         out.append(txt[:target])
     return out
