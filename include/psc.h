@@ -304,12 +304,16 @@ psc_status psc_host_advance(const psc_handle* h, int32_t* q, uint16_t* h_stack, 
  * every GPU that loads the library until the process exits).  Nothing is
  * allocated or freed by the call.
  *   d_q, d_depth, d_status : device int32 [B] (lexer state, stack depth, row status)
- *   d_stack                : device uint16 [B][cap], bottom first (the layout psc_states_download returns)
+ *   d_stack                : device uint16 [B][cap], bottom first (the layout psc_states_download returns);
+ *                            a row whose lexer state, depth or stack symbols are out of range gets
+ *                            the empty mask (its logits all -inf)
  *   other arguments        : as for psc_fill_apply
  * Errors: PSC_ERR_LIMIT when B > PSC_NOALLOC_MAX_ROWS; PSC_ERR_ARG for bad arguments.
  * The first call on a device looks up the scratch array's device address
  * (cudaGetSymbolAddress) with that device current; make that first call
- * before any stream capture.  Every call shares the same scratch array, which
+ * before any stream capture.  The address is kept for the life of the
+ * process: it does not survive cudaDeviceReset (which unloads the module), so
+ * do not call this entry point after resetting the device.  Every call shares the same scratch array, which
  * keeps the last call's contents (each call writes every entry it reads, so
  * nothing needs clearing); calls that overlap on the GPU (different streams,
  * or host threads racing on one device) race on it and must be serialised by

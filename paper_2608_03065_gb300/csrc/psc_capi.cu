@@ -150,7 +150,9 @@ __device__ __forceinline__ int memo_classify(const DevTables& T, const DevStates
 // Classification of one row (Algorithm 2 step 3) by a full warp: from the kept
 // bottom-up block when there is one, else the walk of the classifier DFA: lanes
 // load 32 stack symbols at a time (coalesced), the walk broadcasts them with
-// shuffles and follows the DFA; every lane ends with the same mask id.
+// shuffles and follows the DFA; every lane ends with the same mask id.  A stack
+// symbol outside the LR states (only a caller-owned stack can hold one) gives
+// the row the empty mask instead of a read outside the table.
 __device__ int warp_classify(const DevTables& T, const DevStates& S, int b, int lane) {
     int status = S.status[b];
     if (status == ROW_DONE) return 1;
@@ -168,7 +170,8 @@ __device__ int warp_classify(const DevTables& T, const DevStates& S, int b, int 
         int x = i >= 0 ? st[i] : 0;
         int n = top + 1 < 32 ? top + 1 : 32;
         for (int j = 0; j < n; j++) {
-            int X = __shfl_sync(FULL, x, j);
+            int X = __shfl_sync(FULL, x, j);   // the same in every lane: the warp returns together
+            if ((unsigned)X >= (unsigned)T.n_lr) return 0;
             int nx = __ldg(T.dfa + (size_t)s * T.n_lr + X);
             if (nx < 0) return -nx - 1;
             s = nx;
@@ -177,7 +180,7 @@ __device__ int warp_classify(const DevTables& T, const DevStates& S, int b, int 
     return __ldg(T.dfa_mask + s);
 }
 
-// the same classification by one thread
+// the same classification by one thread (same guard on stack symbols)
 __device__ int thread_classify(const DevTables& T, const DevStates& S, int b) {
     int status = S.status[b];
     if (status == ROW_DONE) return 1;
@@ -191,7 +194,9 @@ __device__ int thread_classify(const DevTables& T, const DevStates& S, int b) {
     if (s < 0) return -s - 1;
     const uint16_t* st = S.stack + (size_t)b * S.cap;
     for (int i = depth - 1; i >= 0; i--) {
-        int nx = __ldg(T.dfa + (size_t)s * T.n_lr + st[i]);
+        int X = st[i];
+        if (X >= T.n_lr) return 0;
+        int nx = __ldg(T.dfa + (size_t)s * T.n_lr + X);
         if (nx < 0) return -nx - 1;
         s = nx;
     }
@@ -932,6 +937,11 @@ int adv_smem(const DevTables& d) { return d.adv_bytes + ADV_WARPS * ADV_WIN * 2;
 __device__ __forceinline__ uint32_t smem_addr(const void* p) {
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
+// Global-window address of a device pointer, for the source operand of bulk copies
+// (the same value for cudaMalloc memory; the conversion makes the state space explicit).
+__device__ __forceinline__ uint64_t gmem_addr(const void* p) {
+    return static_cast<uint64_t>(__cvta_generic_to_global(p));
+}
 
 // Programmatic dependent launch: the next kernel of the stream may be scheduled
 // now (it waits for this grid's results with grid_dep_wait); and the wait for
@@ -1034,6 +1044,7 @@ __device__ __forceinline__ int warp_walk(const DevTables& T, const StackView& sv
         int n = top + 1 < 32 ? top + 1 : 32;
         for (int j = 0; j < n; j++) {
             int X = __shfl_sync(FULL, x, j);
+            if ((unsigned)X >= (unsigned)T.n_lr) return 0;
             int nx = ld_keep(T.dfa + (size_t)s * T.n_lr + X, pol);
             if (nx < 0) return -nx - 1;
             s = nx;
@@ -1093,7 +1104,7 @@ __global__ void __launch_bounds__(ADV_WARPS * 32) k_advance_warp(DevTables T, De
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
         asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar_a), "r"(T.adv_bytes) : "memory");
         asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
-                     ::"r"(smem_addr(sm)), "l"(T.adv), "r"(T.adv_bytes), "r"(bar_a)
+                     ::"r"(smem_addr(sm)), "l"(gmem_addr(T.adv)), "r"(T.adv_bytes), "r"(bar_a)
                      : "memory");
     }
     grid_dep_launch();
@@ -1289,7 +1300,7 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
 // 1-D bulk copy global -> shared, completing on the mbarrier (16-byte aligned, size a multiple of 16).
 __device__ __forceinline__ void tma_load_1d(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
     asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
-                 ::"r"(dst), "l"(src), "r"(bytes), "r"(bar)
+                 ::"r"(dst), "l"(gmem_addr(src)), "r"(bytes), "r"(bar)
                  : "memory");
 }
 // The same with an L2 cache policy (the streamed logits go first when L2 evicts,
@@ -1298,7 +1309,7 @@ __device__ __forceinline__ void tma_load_1d_hint(uint32_t dst, const void* src, 
                                                  uint64_t policy) {
     asm volatile(
         "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], %4;"
-        ::"r"(dst), "l"(src), "r"(bytes), "r"(bar), "l"(policy)
+        ::"r"(dst), "l"(gmem_addr(src)), "r"(bytes), "r"(bar), "l"(policy)
         : "memory");
 }
 __device__ __forceinline__ uint64_t l2_evict_first_policy() {

@@ -397,8 +397,10 @@ def psc_fill_apply_noalloc(h: Handle, q, depth, status, stack, logits, bitmask_o
     V = h.V if V is None else V
     if stack.dim() != 2 or stack.shape[0] != B or not stack.is_contiguous() or stack.element_size() != 2:
         raise ValueError("stack must be a contiguous [B, cap] 16-bit tensor")
-    if logits.shape[0] != B or logits.shape[1] < V:
+    if logits.dim() != 2 or logits.shape[0] != B or logits.shape[1] < V:
         raise ValueError("logits must be [B, >=V]")
+    if bitmask_out is not None and (bitmask_out.shape != (B, h.W) or not bitmask_out.is_contiguous()):
+        raise ValueError(f"bitmask_out must be a contiguous [{B}, {h.W}] tensor")
     _check(load().psc_fill_apply_noalloc(h.ptr, _ptr(q, torch.int32, "q", B), _ptr(depth, torch.int32, "depth", B),
                                          _ptr(status, torch.int32, "status", B), _ptr(stack, None, "stack"),
                                          stack.shape[1], B, _ptr(logits, None, "logits"), _dtype_code(logits),

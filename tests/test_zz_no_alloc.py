@@ -43,8 +43,15 @@ def _bits(t):
     return t.view(torch.int16 if t.dtype == torch.bfloat16 else torch.int32).numpy()
 
 
-def test_noalloc_matches_fill_apply_on_two_calls(psc):
-    w = configs.load(2)
+@pytest.mark.parametrize("cfg_id,pad,with_bitmask", [(2, 0, True), (1, 0, True), (2, 40, False), (1, 7, True)])
+def test_noalloc_matches_fill_apply_on_two_calls(psc, cfg_id, pad, with_bitmask):
+    """Two calls in a row, each against psc_fill_apply on the same states: bf16
+    (config 2) and f32 (config 1) logits, rows padded past V (row stride > V,
+    columns >= V untouched), with and without the bitmask copy.  psc_fill_apply
+    classifies through the states object's kept bottom-up blocks; the no-alloc
+    call has none and walks the classifier DFA from the stack top, so the
+    comparison also checks those two classifications against each other."""
+    w = configs.load(cfg_id)
     h = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id)
     st = psc.psc_state_init(h, w.B, 64)
     tm = torch.from_numpy(w.token_matrix()).cuda()
@@ -52,18 +59,23 @@ def test_noalloc_matches_fill_apply_on_two_calls(psc):
         psc.psc_advance(h, st, tm[:, j].contiguous())
     tok = torch.empty(w.B, dtype=torch.int32, device="cuda")
     for call in range(2):
-        logits = w.logits(call + 20).cuda()
+        base = w.logits(call + 20)
+        padded = torch.cat([base, base[:, :pad]], dim=1) if pad else base
+        logits = padded.cuda()
         a, b = logits.clone(), logits.clone()
+        av, bv = a[:, :w.V], b[:, :w.V]          # row stride V + pad
         bm_a = torch.zeros(w.B, h.W, dtype=torch.int32, device="cuda")
-        bm_b = torch.full((w.B, h.W), -1, dtype=torch.int32, device="cuda")
+        bm_b = torch.full((w.B, h.W), -1, dtype=torch.int32, device="cuda") if with_bitmask else None
         q, depth, status, stack = _device_copy_of_states(psc, st)
-        psc.psc_fill_apply(h, st, a, bm_a)
-        psc.psc_fill_apply_noalloc(h, q, depth, status, stack, b, bm_b)
+        psc.psc_fill_apply(h, st, av, bm_a)
+        psc.psc_fill_apply_noalloc(h, q, depth, status, stack, bv, bm_b)
         torch.cuda.synchronize()
         np.testing.assert_array_equal(_bits(b), _bits(a))
-        np.testing.assert_array_equal(bm_b.cpu().numpy(), bm_a.cpu().numpy())
+        np.testing.assert_array_equal(_bits(b)[:, w.V:], _bits(logits)[:, w.V:])
+        if with_bitmask:
+            np.testing.assert_array_equal(bm_b.cpu().numpy(), bm_a.cpu().numpy())
         # move the batch on by one greedy step before the second call
-        psc.psc_argmax_masked(h, st, a, tok)
+        psc.psc_argmax_masked(h, st, av, tok)
         psc.psc_advance(h, st, tok)
     torch.cuda.synchronize()
 
@@ -74,7 +86,7 @@ def test_noalloc_rejects_batches_above_the_scratch_size(psc):
     B = psc.NOALLOC_MAX_ROWS + 1
     q = torch.zeros(B, dtype=torch.int32, device="cuda")
     stack = torch.zeros(B, 4, dtype=torch.int16, device="cuda")
-    x = torch.zeros(B, w.V, device="cuda")
+    x = torch.zeros(1, w.V, device="cuda").expand(B, w.V)   # row stride 0: nothing is read
     with pytest.raises(psc.PscError) as e:
         psc.psc_fill_apply_noalloc(h, q, q, q, stack, x)
     assert e.value.code == 5 and "PSC_NOALLOC_MAX_ROWS" in str(e.value)
