@@ -963,56 +963,118 @@ __device__ __forceinline__ bool mbar_wait0(uint32_t bar, int limit) {
     return false;
 }
 
+// Shared-memory loads and stores by 32-bit shared-window address.  The parser's
+// table reads are chains of dependent loads, one lane at a time: naming the state
+// space keeps each one a plain shared-memory access.
+__device__ __forceinline__ int lds_s16(uint32_t a) {
+    short v;
+    asm volatile("ld.shared.s16 %0, [%1];" : "=h"(v) : "r"(a));
+    return v;
+}
+__device__ __forceinline__ int lds_u16(uint32_t a) {
+    unsigned short v;
+    asm volatile("ld.shared.u16 %0, [%1];" : "=h"(v) : "r"(a));
+    return v;
+}
+__device__ __forceinline__ int lds_u8(uint32_t a) {
+    unsigned short v;
+    asm volatile("ld.shared.u8 %0, [%1];" : "=h"(v) : "r"(a));
+    return v;
+}
+__device__ __forceinline__ void sts_u16(uint32_t a, int v) {
+    asm volatile("st.shared.u16 [%0], %1;" ::"r"(a), "h"((unsigned short)v) : "memory");
+}
+
 // A row's stack seen through its window: indices in [base, base + ADV_WIN) live
-// in shared memory, the others in global memory.  `lo` tracks the lowest index
-// written (for the write-back and the bottom-up classifier).
+// in shared memory (at shared address wa), the others in global memory.  `lo`
+// tracks the lowest index written (for the write-back and the bottom-up classifier).
 struct StackView {
     uint16_t* win;
     uint16_t* st;
     int base;
     int lo;
-    __device__ __forceinline__ bool in_win(int i) const { return i >= base && i < base + ADV_WIN; }
-    __device__ __forceinline__ int get(int i) const { return in_win(i) ? win[i - base] : st[i]; }
+    uint32_t wa;   // shared-window address of win
+    __device__ __forceinline__ bool in_win(int i) const { return (unsigned)(i - base) < (unsigned)ADV_WIN; }
+    __device__ __forceinline__ int get(int i) const { return in_win(i) ? lds_u16(wa + 2u * (i - base)) : st[i]; }
     __device__ __forceinline__ void set(int i, int v) {
-        if (in_win(i)) win[i - base] = (uint16_t)v;
+        if (in_win(i)) sts_u16(wa + 2u * (i - base), v);
         else st[i] = (uint16_t)v;
         lo = i < lo ? i : lo;
     }
+};
+
+// Shared-window addresses of the compact lexer/parser tables staged by
+// k_advance_warp, and their row strides in bytes.
+struct AdvTabs {
+    uint32_t bc, trans, acc, ign, res, act, go, rlen, rlhs;
+    uint32_t trans_row, res_row, act_row, go_row;   // bytes per row: nbc, n_lr, n_terms, n_nts int16 entries
+    int q0;
+    __device__ __forceinline__ AdvTabs(uint32_t sb, const DevTables& T)
+        : bc(sb + T.o_bc), trans(sb + T.o_trans), acc(sb + T.o_accept), ign(sb + T.o_ign), res(sb + T.o_resolve),
+          act(sb + T.o_action), go(sb + T.o_go), rlen(sb + T.o_rlen), rlhs(sb + T.o_rlhs),
+          trans_row(2u * T.nbc), res_row(2u * T.n_lr), act_row(2u * T.n_terms), go_row(2u * T.n_nts), q0(T.q0) {}
 };
 
 // Feed one lexeme class to the parser: resolve it to a terminal with the
 // current top (contextual lexing), reduce until it is shifted.  Returns a row
 // status.  `top` and `below` hold the two topmost entries in registers: a
 // reduction of one symbol (the chains of unit rules) uncovers `below`, so it
-// reads no stack entry.
-__device__ __forceinline__ int feed_class_win(const uint8_t* sm, const DevTables& T, StackView& sv, int& depth,
-                                              int& top, int& below, int cap, int cls) {
-    const int16_t* resolve = reinterpret_cast<const int16_t*>(sm + T.o_resolve);
-    const int16_t* action = reinterpret_cast<const int16_t*>(sm + T.o_action);
-    const int16_t* go = reinterpret_cast<const int16_t*>(sm + T.o_go);
-    const uint8_t* rlen = sm + T.o_rlen;
-    const int16_t* rlhs = reinterpret_cast<const int16_t*>(sm + T.o_rlhs);
-    int t = resolve[cls * T.n_lr + top];
+// reads no stack entry; only a reduction of two or more symbols reads one.
+// PACKED: reduce entries carry (rule length << 10 | left-hand side); then a run
+// of one-symbol reductions takes a short loop (one action and one goto lookup
+// each, the goto row of `below` fixed for the run) and the new top is written
+// to the stack once, when the run ends (not at all when a longer reduction then
+// pops it).
+template <bool PACKED>
+__device__ __forceinline__ int feed_class_win(const AdvTabs& A, StackView& sv, int& depth, int& top, int& below,
+                                              int cap, int cls) {
+    int t = lds_s16(A.res + cls * A.res_row + 2u * top);
     if (t < 0) return ROW_REJECTED;
+    const uint32_t col = A.act + 2u * t;   // ACTION[.][t]
+    bool dirty = false;                     // top changed by one-symbol reductions, not yet on the stack
     for (int guard = 0; guard < 4 * cap + 64; guard++) {
-        int a = action[top * T.n_terms + t];
+        int a = lds_s16(col + top * A.act_row);
+        if (PACKED) {
+            // packed unit reduction: kind REDUCE, rule length 1 (bits 12-15), lhs in bits 2-11
+            const uint32_t go_below = A.go + below * A.go_row;
+            while ((a & 0xF003) == 0x1002 && depth >= 2) {
+                int g = lds_s16(go_below + ((a >> 1) & 0x7FE));   // GOTO[below][lhs], 2 * lhs = (a >> 1) & 0x7FE
+                if (g < 0) return ROW_REJECTED;
+                if (++guard >= 4 * cap + 64) return ROW_LIMIT;
+                top = g;
+                dirty = true;
+                a = lds_s16(col + top * A.act_row);
+            }
+        }
         int kind = a & 3, val = (a >> 2) & 0x3FFF;
         if (kind == psc::ACT_SHIFT) {
             if (depth >= cap) return ROW_OVERFLOW;
+            if (dirty) sv.set(depth - 1, top);
             sv.set(depth++, val);
             below = top;
             top = val;
             return ROW_OK;
         }
         if (kind != psc::ACT_REDUCE) return ROW_REJECTED;
-        int k = T.adv_packed ? val >> 10 : rlen[val];
-        int lhs = T.adv_packed ? val & 1023 : rlhs[val];
+        int k, lhs;
+        if (PACKED) {
+            k = val >> 10;
+            lhs = val & 1023;
+        } else {
+            k = lds_u8(A.rlen + val);
+            lhs = lds_s16(A.rlhs + 2u * val);
+        }
         if (depth - k < 1) return ROW_REJECTED;
+        if (k == 0 && dirty) sv.set(depth - 1, top);   // an empty rule pushes above the current top
+        dirty = false;
         depth -= k;
-        // the entry the reduction uncovers: the top itself (k = 0), the one below it
-        // (k = 1), else read from the stack
-        int under = k == 0 ? top : k == 1 ? below : sv.get(depth - 1);
-        int g = go[under * T.n_nts + lhs];
+        // the entry the reduction uncovers: the one below the top (k = 1), the top
+        // itself (k = 0), else read from the stack
+        int under;
+        if (k == 1) under = below;
+        else if (k == 0) under = top;
+        else under = sv.get(depth - 1);
+        int g = lds_s16(A.go + under * A.go_row + 2u * lhs);
         if (g < 0) return ROW_REJECTED;
         if (depth >= cap) return ROW_OVERFLOW;
         sv.set(depth++, g);
@@ -1091,11 +1153,13 @@ __device__ __forceinline__ int warp_memo_extend(const DevTables& T, const StackV
 // then classify the new configuration into S.mid.  Everything that needs only
 // global memory (the row's state, its mask word, the token's bytes, the stack
 // window) is loaded while the tables are still being staged.
+template <bool PACKED>
 __global__ void __launch_bounds__(ADV_WARPS * 32) k_advance_warp(DevTables T, DevStates S, const int32_t* tokens,
                                                                  int B, int use_mid, int32_t* status_out,
                                                                  int from_keys, int32_t* tokens_out) {
     extern __shared__ uint4 smem4[];
     __shared__ __align__(8) uint64_t bar;
+    __shared__ uint8_t tokc[ADV_WARPS][32];   // the lexer byte classes of each row's token (first 32 bytes)
     uint8_t* sm = reinterpret_cast<uint8_t*>(smem4);
     // one TMA bulk copy stages the compact tables (16-byte aligned, multiple of 16 bytes)
     uint32_t bar_a = smem_addr(&bar);
@@ -1113,13 +1177,14 @@ __global__ void __launch_bounds__(ADV_WARPS * 32) k_advance_warp(DevTables T, De
     int b = blockIdx.x * ADV_WARPS + warp;
     bool active = b < B;   // warp-uniform
     StackView sv{reinterpret_cast<uint16_t*>(sm + T.adv_bytes) + warp * ADV_WIN,
-                 S.stack + (size_t)(active ? b : 0) * S.cap, 0x40000000, 0x7FFFFFFF};
+                 S.stack + (size_t)(active ? b : 0) * S.cap, 0x40000000, 0x7FFFFFFF, 0u};
+    sv.wa = smem_addr(sv.win);
     int tok = -1, status = ROW_OK, q = 0, depth = 0;
     bool parse = false;
     int32_t* memo = active && S.rmemo && T.bu ? S.rmemo + (size_t)b * S.cap : nullptr;
     int memo_top = -1, depth0 = 0;
     uint32_t mword = 0;
-    uint32_t tw[8] = {0, 0, 0, 0, 0, 0, 0, 0};   // the token's bytes (tokens up to 32 bytes)
+    int tbyte = 0;   // lane i: byte i of the token (first 32 bytes)
     int len = 0;
     int64_t vlo = 0;
     if (active) {
@@ -1158,7 +1223,7 @@ __global__ void __launch_bounds__(ADV_WARPS * 32) k_advance_warp(DevTables T, De
                     if (!use_mid) {   // the kept bottom-up block, else a walk of the stack in global memory
                         int e = __shfl_sync(FULL, memo_top, 0);
                         mid = memo && live && q >= 0 && q < T.nq ? memo_mask(T, e, q) : -1;
-                        StackView g{sv.win, sv.st, 0x40000000, 0x7FFFFFFF};
+                        StackView g{sv.win, sv.st, 0x40000000, 0x7FFFFFFF, sv.wa};
                         if (mid < 0) mid = depth >= 1 && depth <= S.cap ? warp_walk(T, g, q, depth, lane) : 0;
                     }
                     // the token's mask bit (in flight while the token is parsed); the row is
@@ -1170,16 +1235,17 @@ __global__ void __launch_bounds__(ADV_WARPS * 32) k_advance_warp(DevTables T, De
                 }
             }
         }
-        if (parse && lane == 0) {   // the token's bytes
+        if (parse) {   // the token's bytes: lane i holds byte i
             vlo = T.vocab_off[tok];
             len = (int)(T.vocab_off[tok + 1] - vlo);
-#pragma unroll
-            for (int i = 0; i < 32; i++)
-                if (i < len) tw[i >> 2] |= (uint32_t)T.vocab[vlo + i] << (8 * (i & 3));
+            if (lane < len) tbyte = T.vocab[vlo + lane];
         }
     }
     __syncthreads();
     bool staged = __all_sync(FULL, mbar_wait0(bar_a, 1 << 24));
+    // the tables are in: each lane turns its byte into a lexer byte class
+    if (staged && active && parse && lane < len) tokc[warp][lane] = sm[T.o_bc + tbyte];
+    __syncwarp();
     if (!staged) {
         // the copy did not land: give the rows a LIMIT status, wait (bounded) for the copy, return
         if (threadIdx.x == 0) atomicAdd(&g_pipeline_timeouts, 1);
@@ -1194,34 +1260,34 @@ __global__ void __launch_bounds__(ADV_WARPS * 32) k_advance_warp(DevTables T, De
     }
     if (!active) return;
     if (parse) {
-        const uint8_t* bc = sm + T.o_bc;
-        const int16_t* trans = reinterpret_cast<const int16_t*>(sm + T.o_trans);
-        const int16_t* acc = reinterpret_cast<const int16_t*>(sm + T.o_accept);
-        const uint8_t* ign = sm + T.o_ign;
+        const AdvTabs A(smem_addr(sm), T);
         int nq = q, nd = depth;
         if (lane == 0) {
-            int top = sv.win[depth - 1 - sv.base];
+            int top = sv.get(depth - 1);
             int below = depth >= 2 ? sv.get(depth - 2) : 0;
-            for (int i = 0; i < len && status == ROW_OK; i++) {
-                uint32_t wsel = tw[0];   // tw[i >> 2] by selects (registers, not local memory)
-#pragma unroll
-                for (int k = 1; k < 8; k++) wsel = (i >> 2) == k ? tw[k] : wsel;
-                int byte = i < 32 ? (int)((wsel >> (8 * (i & 3))) & 0xFFu) : (int)T.vocab[vlo + i];
-                int c = bc[byte];
-                int nx = trans[nq * T.nbc + c];
+            // one byte (as its byte class) through the lexer DFA; a completed lexeme
+            // goes to the parser
+            auto lex = [&](int c) {
+                int nx = lds_s16(A.trans + nq * A.trans_row + 2u * c);
                 if (nx >= 0) {
                     nq = nx;
-                    continue;
+                    return;
                 }
-                int cls = nq == T.q0 ? -1 : acc[nq];
+                int cls = nq == A.q0 ? -1 : lds_s16(A.acc + 2u * nq);
                 if (cls < 0) {
                     status = ROW_REJECTED;
-                    break;
+                    return;
                 }
-                if (!ign[cls]) status = feed_class_win(sm, T, sv, nd, top, below, S.cap, cls);
-                nq = trans[T.q0 * T.nbc + c];
+                if (!lds_u8(A.ign + cls)) status = feed_class_win<PACKED>(A, sv, nd, top, below, S.cap, cls);
+                nq = lds_s16(A.trans + A.q0 * A.trans_row + 2u * c);
                 if (nq < 0) status = ROW_REJECTED;
-            }
+            };
+            // the classes of the first 32 bytes were staged by the lanes; longer tokens
+            // read the rest from the vocabulary
+            int n0 = len < 32 ? len : 32;
+            const uint32_t ca = smem_addr(&tokc[warp][0]);
+            for (int i = 0; i < n0 && status == ROW_OK; i++) lex(lds_u8(ca + i));
+            for (int i = 32; i < len && status == ROW_OK; i++) lex(lds_u8(A.bc + T.vocab[vlo + i]));
             if (!((mword >> (tok & 31)) & 1)) status = ROW_REJECTED;
             if (status == ROW_OK) {
                 S.q[b] = nq;
@@ -1672,7 +1738,8 @@ psc_status launch_advance(const psc_handle* h, psc_states* st, const int32_t* d_
     int from_keys = d_tokens_out ? 1 : 0;
     psc_status s;
     if (h->d.adv_bytes > 0) {
-        s = launch_pdl(k_advance_warp, dim3((B + ADV_WARPS - 1) / ADV_WARPS), dim3(ADV_WARPS * 32), adv_smem(h->d), cs,
+        s = launch_pdl(h->d.adv_packed ? k_advance_warp<true> : k_advance_warp<false>,
+                       dim3((B + ADV_WARPS - 1) / ADV_WARPS), dim3(ADV_WARPS * 32), adv_smem(h->d), cs,
                        "k_advance_warp", h->d, st->d, d_tokens, B, use_mid, d_row_status, from_keys, d_tokens_out);
     } else {
         k_advance<<<(B + 127) / 128, 128, 0, cs>>>(h->d, st->d, d_tokens, B, use_mid, d_row_status, from_keys,
@@ -1905,12 +1972,12 @@ psc_status upload_tables(std::unique_ptr<psc_handle>& h, bool global_tables) {
         int optin = 0;
         cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, h->device);
         cudaFuncAttributes fa{};
-        cudaFuncGetAttributes(&fa, k_advance_warp);
+        auto kadv = d.adv_packed ? k_advance_warp<true> : k_advance_warp<false>;
+        cudaFuncGetAttributes(&fa, kadv);
         optin -= (int)fa.sharedSizeBytes;   // the limit covers dynamic memory only
         if (optin < adv_smem(d)) {
             d.adv_bytes = 0;   // cannot stage: fall back to global tables
-        } else if ((s = cuda_check(cudaFuncSetAttribute(k_advance_warp, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                        optin),
+        } else if ((s = cuda_check(cudaFuncSetAttribute(kadv, cudaFuncAttributeMaxDynamicSharedMemorySize, optin),
                                    "cudaFuncSetAttribute(k_advance_warp)")) != PSC_OK) {
             for (int i = 0; i < h->n_blocks; i++) cudaFree(h->blocks[i]);
             return s;
