@@ -104,6 +104,8 @@ struct psc_states {
     int device = -1;
     uint64_t gen = 1;        // bumped by every call that changes the rows
     uint64_t mid_gen = 0;    // generation the mask ids in d.mid were computed for
+    bool after_mask = false; // the last work enqueued on these states is the TMA masking pass with
+                             // the mask ids as they were (the advance may read the rows early)
 };
 
 namespace {
@@ -1153,13 +1155,20 @@ __device__ __forceinline__ int warp_memo_extend(const DevTables& T, const StackV
 // then classify the new configuration into S.mid.  Everything that needs only
 // global memory (the row's state, its mask word, the token's bytes, the stack
 // window) is loaded while the tables are still being staged.
+// early: the row's state (lexer state, depth, status, mask id, stack window, kept
+// bottom-up blocks) is read before waiting for the previous kernel.  Only the greedy
+// keys come from that kernel (the masking pass), and the masking pass lets this
+// kernel start only after its own wait for the advance before it, which wrote the
+// rows; the host sets `early` only when the masking pass is the last work on
+// these states and took the mask ids as they were.
 template <bool PACKED>
 __global__ void __launch_bounds__(ADV_WARPS * 32) k_advance_warp(DevTables T, DevStates S, const int32_t* tokens,
                                                                  int B, int use_mid, int32_t* status_out,
-                                                                 int from_keys, int32_t* tokens_out) {
+                                                                 int from_keys, int32_t* tokens_out, int early) {
     extern __shared__ uint4 smem4[];
     __shared__ __align__(8) uint64_t bar;
-    __shared__ uint8_t tokc[ADV_WARPS][32];   // the lexer byte classes of each row's token (first 32 bytes)
+    __shared__ uint8_t tokc[ADV_WARPS][32];     // the lexer byte classes of each row's token (first 32 bytes)
+    __shared__ uint16_t lexcls[ADV_WARPS][32];  // the lexeme classes the token emits (tokens up to 32 bytes)
     uint8_t* sm = reinterpret_cast<uint8_t*>(smem4);
     // one TMA bulk copy stages the compact tables (16-byte aligned, multiple of 16 bytes)
     uint32_t bar_a = smem_addr(&bar);
@@ -1172,7 +1181,6 @@ __global__ void __launch_bounds__(ADV_WARPS * 32) k_advance_warp(DevTables T, De
                      : "memory");
     }
     grid_dep_launch();
-    grid_dep_wait();   // the greedy keys and rows come from the previous kernel
     int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     int b = blockIdx.x * ADV_WARPS + warp;
     bool active = b < B;   // warp-uniform
@@ -1187,13 +1195,29 @@ __global__ void __launch_bounds__(ADV_WARPS * 32) k_advance_warp(DevTables T, De
     int tbyte = 0;   // lane i: byte i of the token (first 32 bytes)
     int len = 0;
     int64_t vlo = 0;
-    if (active) {
-        // the loads that need nothing but the row index go first, together
-        q = S.q[b];
-        depth = S.depth[b];
+    int cur_mid = 0;   // the mask the row's token is checked against
+    bool live = false;
+    // the row's state and the window of its stack top (for the parse and for the
+    // classifier walk after it); read from L2 (an SM's L1 may still hold these lines
+    // from an earlier kernel)
+    auto load_row = [&]() {
+        q = __ldcg(S.q + b);
+        depth = __ldcg(S.depth + b);
         depth0 = depth;
-        status = S.status[b];
-        int mid = use_mid ? S.mid[b] : 0;
+        status = __ldcg(S.status + b);
+        cur_mid = use_mid ? __ldcg(S.mid + b) : 0;
+        live = status == ROW_OK && depth >= 1 && depth <= S.cap;
+        if (live) {
+            sv.base = depth > ADV_KEEP ? depth - ADV_KEEP : 0;
+            for (int i = lane; i < depth - sv.base; i += 32) sv.win[i] = __ldcg(sv.st + sv.base + i);
+            // the kept bottom-up blocks of the top 32 prefixes (lane l: stack [0, depth-1-l])
+            if (memo && depth - 1 - lane >= 0) memo_top = __ldcg(memo + depth - 1 - lane);
+        }
+    };
+    if (active && early) load_row();
+    grid_dep_wait();   // the greedy keys (and, unless early, the rows) come from the previous kernel
+    if (active) {
+        if (!early) load_row();
         if (from_keys) {   // the greedy choice of the fused masking pass
             unsigned long long k = S.best[b];
             tok = k ? (int32_t)(~(uint32_t)(k & 0xFFFFFFFFu)) : -1;
@@ -1205,14 +1229,6 @@ __global__ void __launch_bounds__(ADV_WARPS * 32) k_advance_warp(DevTables T, De
         } else {
             tok = tokens[b];
         }
-        // the window of the stack top: for the parse and for the classifier walk after it
-        bool live = status == ROW_OK && depth >= 1 && depth <= S.cap;
-        if (live) {
-            sv.base = depth > ADV_KEEP ? depth - ADV_KEEP : 0;
-            for (int i = lane; i < depth - sv.base; i += 32) sv.win[i] = sv.st[sv.base + i];
-            // the kept bottom-up blocks of the top 32 prefixes (lane l: stack [0, depth-1-l])
-            if (memo && depth - 1 - lane >= 0) memo_top = memo[depth - 1 - lane];
-        }
         if (tok >= 0) {
             if (status == ROW_DONE) {
                 status = tok == T.eos_id ? ROW_DONE : ROW_REJECTED;
@@ -1222,13 +1238,14 @@ __global__ void __launch_bounds__(ADV_WARPS * 32) k_advance_warp(DevTables T, De
                 } else {
                     if (!use_mid) {   // the kept bottom-up block, else a walk of the stack in global memory
                         int e = __shfl_sync(FULL, memo_top, 0);
-                        mid = memo && live && q >= 0 && q < T.nq ? memo_mask(T, e, q) : -1;
+                        cur_mid = memo && live && q >= 0 && q < T.nq ? memo_mask(T, e, q) : -1;
                         StackView g{sv.win, sv.st, 0x40000000, 0x7FFFFFFF, sv.wa};
-                        if (mid < 0) mid = depth >= 1 && depth <= S.cap ? warp_walk(T, g, q, depth, lane) : 0;
+                        if (cur_mid < 0)
+                            cur_mid = depth >= 1 && depth <= S.cap ? warp_walk(T, g, q, depth, lane) : 0;
                     }
                     // the token's mask bit (in flight while the token is parsed); the row is
                     // only committed (q, depth) when it is set
-                    mword = mask_word(T, mid, tok >> 5);
+                    mword = mask_word(T, cur_mid, tok >> 5);
                     if (tok == T.eos_id) status = ((mword >> (tok & 31)) & 1) ? ROW_DONE : ROW_REJECTED;
                     else if (!live) status = ROW_REJECTED;
                     else parse = true;
@@ -1262,32 +1279,95 @@ __global__ void __launch_bounds__(ADV_WARPS * 32) k_advance_warp(DevTables T, De
     if (parse) {
         const AdvTabs A(smem_addr(sm), T);
         int nq = q, nd = depth;
+        const uint32_t ca = smem_addr(&tokc[warp][0]);
+        const uint32_t la = smem_addr(&lexcls[warp][0]);
+        int ncls = -1;   // classes in lexcls; -1: the token is lexed by lane 0 (longer than 32 bytes)
+        if (len <= 32) {
+            // Lexing in parallel (the lexer does not depend on the parser): lane j runs the
+            // lexer DFA over the lexeme that starts afresh at byte j, lane 0 over the
+            // continuation of the row's pending lexeme; each records where its lexeme
+            // ends (the byte it cannot take, or the end of the token) and the DFA state
+            // there.  Then the lexemes are followed from one end to the next.
+            int ls = lane == 0 ? q : A.q0;
+            int le = lane;
+            int pre = -2;   // class of the pending lexeme when the token's first byte ends it
+            auto run = [&]() {
+                while (le < len) {
+                    int nx = lds_s16(A.trans + ls * A.trans_row + 2u * lds_u8(ca + le));
+                    if (nx < 0) break;
+                    ls = nx;
+                    le++;
+                }
+            };
+            if (lane < len) {
+                run();
+                if (lane == 0 && le == 0 && q != A.q0) {
+                    pre = lds_s16(A.acc + 2u * q);
+                    ls = A.q0;
+                    run();
+                }
+            }
+            pre = __shfl_sync(FULL, pre, 0);
+            ncls = 0;
+            if (pre != -2) {
+                if (pre < 0) {
+                    status = ROW_REJECTED;
+                } else if (!lds_u8(A.ign + pre)) {
+                    if (lane == 0) sts_u16(la, pre);
+                    ncls = 1;
+                }
+            }
+            int pos = 0;
+            while (status == ROW_OK) {   // warp-uniform: pos and the lexeme ends come by shuffles
+                int ep = __shfl_sync(FULL, le, pos), sp = __shfl_sync(FULL, ls, pos);
+                if (ep == len) {   // the last lexeme stays pending
+                    nq = sp;
+                    break;
+                }
+                if (ep == pos) {   // the byte at pos starts no lexeme
+                    status = ROW_REJECTED;
+                    break;
+                }
+                int cls = sp == A.q0 ? -1 : lds_s16(A.acc + 2u * sp);
+                if (cls < 0) {
+                    status = ROW_REJECTED;
+                    break;
+                }
+                if (!lds_u8(A.ign + cls)) {
+                    if (lane == 0) sts_u16(la + 2u * ncls, cls);
+                    ncls++;
+                }
+                pos = ep;
+            }
+        }
+        __syncwarp();
         if (lane == 0) {
             int top = sv.get(depth - 1);
             int below = depth >= 2 ? sv.get(depth - 2) : 0;
-            // one byte (as its byte class) through the lexer DFA; a completed lexeme
-            // goes to the parser
-            auto lex = [&](int c) {
-                int nx = lds_s16(A.trans + nq * A.trans_row + 2u * c);
-                if (nx >= 0) {
-                    nq = nx;
-                    return;
-                }
-                int cls = nq == A.q0 ? -1 : lds_s16(A.acc + 2u * nq);
-                if (cls < 0) {
-                    status = ROW_REJECTED;
-                    return;
-                }
-                if (!lds_u8(A.ign + cls)) status = feed_class_win<PACKED>(A, sv, nd, top, below, S.cap, cls);
-                nq = lds_s16(A.trans + A.q0 * A.trans_row + 2u * c);
-                if (nq < 0) status = ROW_REJECTED;
-            };
-            // the classes of the first 32 bytes were staged by the lanes; longer tokens
-            // read the rest from the vocabulary
-            int n0 = len < 32 ? len : 32;
-            const uint32_t ca = smem_addr(&tokc[warp][0]);
-            for (int i = 0; i < n0 && status == ROW_OK; i++) lex(lds_u8(ca + i));
-            for (int i = 32; i < len && status == ROW_OK; i++) lex(lds_u8(A.bc + T.vocab[vlo + i]));
+            if (ncls >= 0) {
+                for (int k = 0; k < ncls && status == ROW_OK; k++)
+                    status = feed_class_win<PACKED>(A, sv, nd, top, below, S.cap, lds_u16(la + 2u * k));
+            } else {
+                // one byte (as its byte class) through the lexer DFA; a completed lexeme
+                // goes to the parser
+                auto lex = [&](int c) {
+                    int nx = lds_s16(A.trans + nq * A.trans_row + 2u * c);
+                    if (nx >= 0) {
+                        nq = nx;
+                        return;
+                    }
+                    int cls = nq == A.q0 ? -1 : lds_s16(A.acc + 2u * nq);
+                    if (cls < 0) {
+                        status = ROW_REJECTED;
+                        return;
+                    }
+                    if (!lds_u8(A.ign + cls)) status = feed_class_win<PACKED>(A, sv, nd, top, below, S.cap, cls);
+                    nq = lds_s16(A.trans + A.q0 * A.trans_row + 2u * c);
+                    if (nq < 0) status = ROW_REJECTED;
+                };
+                for (int i = 0; i < 32 && status == ROW_OK; i++) lex(lds_u8(ca + i));
+                for (int i = 32; i < len && status == ROW_OK; i++) lex(lds_u8(A.bc + T.vocab[vlo + i]));
+            }
             if (!((mword >> (tok & 31)) & 1)) status = ROW_REJECTED;
             if (status == ROW_OK) {
                 S.q[b] = nq;
@@ -1449,9 +1529,11 @@ __global__ void __launch_bounds__(TMA_WARPS * 32, 3) k_step_tma(T* logits, int64
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     }
-    grid_dep_launch();
     __syncthreads();
     grid_dep_wait();   // mask ids, greedy keys and rows come from the previous kernel
+    // the next kernel (the advance) may start now: the rows' writer before this pass
+    // has completed, so the advance can read the rows before its own wait
+    grid_dep_launch();
     bool failed = false;
     if (warp == 0) {
         // ---------------------------------------------------------- producer
@@ -1681,6 +1763,7 @@ psc_status check_device(const psc_handle* h, const char* what) {
 }
 
 psc_status ensure_mid(const psc_handle* h, const psc_states* st, cudaStream_t s) {
+    const_cast<psc_states*>(st)->after_mask = false;
     if (st->mid_gen == st->gen) return PSC_OK;
     int B = st->d.B;
     int threads = 256;
@@ -1736,11 +1819,14 @@ psc_status launch_advance(const psc_handle* h, psc_states* st, const int32_t* d_
                           int32_t* d_row_status, int32_t* d_tokens_out, cudaStream_t cs) {
     int B = st->d.B;
     int from_keys = d_tokens_out ? 1 : 0;
+    int early = from_keys && st->after_mask ? 1 : 0;
+    st->after_mask = false;
     psc_status s;
     if (h->d.adv_bytes > 0) {
         s = launch_pdl(h->d.adv_packed ? k_advance_warp<true> : k_advance_warp<false>,
                        dim3((B + ADV_WARPS - 1) / ADV_WARPS), dim3(ADV_WARPS * 32), adv_smem(h->d), cs,
-                       "k_advance_warp", h->d, st->d, d_tokens, B, use_mid, d_row_status, from_keys, d_tokens_out);
+                       "k_advance_warp", h->d, st->d, d_tokens, B, use_mid, d_row_status, from_keys, d_tokens_out,
+                       early);
     } else {
         k_advance<<<(B + 127) / 128, 128, 0, cs>>>(h->d, st->d, d_tokens, B, use_mid, d_row_status, from_keys,
                                                     d_tokens_out);
@@ -1798,6 +1884,7 @@ psc_status launch_fused(const psc_handle* h, const psc_states* st, void* d_logit
         s = launch_check("k_apply_argmax");
     }
     if (s == PSC_OK) const_cast<psc_states*>(st)->mid_gen = st->gen;
+    const_cast<psc_states*>(st)->after_mask = s == PSC_OK && vec && have_mid;
     return s;
 }
 
@@ -2164,6 +2251,7 @@ psc_status psc_state_copy(psc_states* dst, const psc_states* src, void* stream) 
         return s;
     dst->gen++;
     dst->mid_gen = src->mid_gen == src->gen ? dst->gen : 0;   // the mask ids are as current as src's
+    dst->after_mask = false;
     return PSC_OK;
 }
 
@@ -2172,6 +2260,7 @@ psc_status psc_state_reset(psc_states* st, const int32_t* d_rows, int32_t n, voi
     int cnt = d_rows ? n : st->d.B;
     if (cnt < 0) return fail_with(PSC_ERR_ARG, "psc_state_reset: negative count");
     st->gen++;
+    st->after_mask = false;
     if (cnt == 0) return PSC_OK;
     k_state_init<<<(cnt + 255) / 256, 256, 0, (cudaStream_t)stream>>>(st->d, st->h->d.q0, d_rows, cnt);
     return launch_check("k_state_init");
@@ -2266,6 +2355,7 @@ psc_status psc_fill_apply_argmax(const psc_handle* h, const psc_states* st, int3
         return fail_with(PSC_ERR_ARG, "psc_fill_apply_argmax: bad arguments");
     cudaStream_t cs = (cudaStream_t)stream;
     if ((s = launch_fused(h, st, d_logits, dtype, row_stride, V, d_bitmask_out, cs)) != PSC_OK) return s;
+    const_cast<psc_states*>(st)->after_mask = false;
     k_finalize_tokens<<<(B + 255) / 256, 256, 0, cs>>>(st->d.best, B, d_tokens);
     return launch_check("k_finalize_tokens");
 }
