@@ -407,35 +407,31 @@ def run_teacher(args):
 
 
 # --------------------------------------------------------------- sweep mode
-def run_sweep(args):
-    """psc_decode_step on config 5's tables at several batch sizes (rows of the
-    workload's prefix states, repeated) and both logit types: µs per step (median
-    of 16 steps, each on fresh logits, from the same prefix states) and the rate of
-    the formula's bytes."""
+def batch_points(psc, h, w, dev, batches, dtypes, n=16):
+    """psc_decode_step on the workload's tables at the given batch sizes (rows
+    0..B-1 of the prefix states) and logit types: µs per step (median of n steps,
+    each on fresh logits from the same prefix states restored with psc_state_copy,
+    CUDA events around the step) and the rate of the formula's bytes."""
     import torch
-    from paper_2608_03065_gb300 import build, psc
-    from workloads import configs
-    build.build()
-    dev = torch.device("cuda", 0)
-    w = configs.load(WORKLOAD)
-    h = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id)
     V = w.V
     tm = torch.from_numpy(w.token_matrix()).to(dev)
     peak, _ = measured_peaks()
-    out = {"metric": "decode step over batch size and logit type", "mode": "sweep", "vocab": V, "points": []}
     stream = torch.cuda.current_stream()
     snaps = {}
-    for B in (1, 16, 128, 1024):   # rows 0..B-1 of the prefix states
+    for B in batches:
         snaps[B] = psc.psc_state_init(h, B, 256)
         for j in range(tm.shape[1]):
             psc.psc_advance(h, snaps[B], tm[:B, j].contiguous())
-    for dt, esz in ((torch.bfloat16, 2), (torch.float32, 4)):
-        for B in (1, 16, 128, 1024):
+    points = []
+    for dt, esz in dtypes:
+        for B in batches:
             st = psc.psc_state_init(h, B, 256)
             tok = torch.empty(B, dtype=torch.int32, device=dev)
-            n = 16
             gen = torch.Generator(device=dev).manual_seed(B)
             xs = [(torch.randn(B, V, generator=gen, device=dev) * w.spec.sigma).to(dt) for _ in range(n)]
+            for i in range(3):   # warm-up
+                psc.psc_state_copy(st, snaps[B], stream=stream)
+                psc.psc_decode_step(h, st, xs[i].clone(), tok, stream=stream)
             times = []
             for i in range(n):
                 psc.psc_state_copy(st, snaps[B], stream=stream)
@@ -448,12 +444,56 @@ def run_sweep(args):
             times.sort()
             us = times[n // 2]
             alg = B * V // 8 + 2 * B * V * esz
-            out["points"].append({"dtype": "bf16" if esz == 2 else "f32", "batch": B, "us_per_step": round(us, 1),
-                                  "algorithmic_GBps": round(alg / (us * 1e-6) / 1e9, 1),
-                                  "frac": round(alg / (us * 1e-6) / 1e9 / peak, 3)})
+            points.append({"dtype": "bf16" if esz == 2 else "f32", "batch": B, "us_per_step": round(us, 2),
+                           "algorithmic_GBps": round(alg / (us * 1e-6) / 1e9, 1),
+                           "frac": round(alg / (us * 1e-6) / 1e9 / peak, 3)})
             del xs
             torch.cuda.empty_cache()
-    print(json.dumps(out))
+    return points
+
+
+def run_sweep(args):
+    """psc_decode_step on config 5's tables at batch 1, 16, 128 and 1024 with bf16
+    and f32 logits (see batch_points)."""
+    import torch
+    from paper_2608_03065_gb300 import build, psc
+    from workloads import configs
+    build.build()
+    dev = torch.device("cuda", 0)
+    w = configs.load(WORKLOAD)
+    h = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id)
+    pts = batch_points(psc, h, w, dev, (1, 16, 128, 1024), ((torch.bfloat16, 2), (torch.float32, 4)))
+    print(json.dumps({"metric": "decode step over batch size and logit type", "mode": "sweep", "vocab": w.V,
+                      "points": pts}))
+
+
+# ------------------------------------------------------------- profile mode
+def run_profile(args):
+    """A small case for profiler captures: the workload's tables and prefix states,
+    then three decode steps (psc_decode_step_mask + psc_decode_step_advance) on
+    fresh logits, each inside an NVTX range named "decode" (about 2 GB on the device)."""
+    import torch
+    from paper_2608_03065_gb300 import build, psc
+    from workloads import configs
+    build.build()
+    w = configs.load(WORKLOAD)
+    h = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id)
+    st = psc.psc_state_init(h, w.B, 256)
+    tm = torch.from_numpy(w.token_matrix()).cuda()
+    for j in range(tm.shape[1]):
+        psc.psc_advance(h, st, tm[:, j].contiguous())
+    g = torch.Generator(device="cuda").manual_seed(3)
+    xs = [(torch.randn(w.B, w.V, generator=g, device="cuda") * w.spec.sigma).to(torch.bfloat16) for _ in range(3)]
+    bm = torch.empty(w.B, h.W, dtype=torch.int32, device="cuda")
+    tok = torch.empty(w.B, dtype=torch.int32, device="cuda")
+    torch.cuda.synchronize()
+    for i in range(3):
+        torch.cuda.nvtx.range_push("decode")
+        psc.psc_decode_step_mask(h, st, xs[i], bm)
+        psc.psc_decode_step_advance(h, st, tok)
+        torch.cuda.synchronize()
+        torch.cuda.nvtx.range_pop()
+    print(json.dumps({"mode": "profile", "steps": 3, "rows_with_a_token": int((tok >= 0).sum())}))
 
 
 # ------------------------------------------------------------------ main arm
@@ -464,10 +504,11 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="gb300")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--mode", default="decode", choices=["decode", "teacher", "sweep"],
+    ap.add_argument("--mode", default="decode", choices=["decode", "teacher", "sweep", "profile"],
                     help="decode: the benchmark line; teacher: teacher-forcing pass rates and "
                          "batch-1 step latency (the paper's RQ1/RQ2 measurements on these workloads); "
-                         "sweep: decode-step time over batch sizes and logit types on config 5's tables")
+                         "sweep: decode-step time over batch sizes and logit types on config 5's tables; "
+                         "profile: three decode steps in NVTX ranges, a small case for profiler captures")
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)
@@ -475,6 +516,8 @@ def main():
         return run_teacher(args)
     if args.mode == "sweep":
         return run_sweep(args)
+    if args.mode == "profile":
+        return run_profile(args)
 
     import torch
     import torch.distributed as dist
@@ -623,6 +666,9 @@ def main():
         "classify_us": median_us(lambda x: psc.psc_advance(h, st, no_tokens, stream=stream)),
     }
 
+    # small batches (decode latency): psc_decode_step at batch 1, 16 and 128 on the same tables
+    small = batch_points(psc, h, w, dev, (1, 16, 128), ((torch.bfloat16, 2),))
+
     if rank != 0:
         if world > 1:
             dist.destroy_process_group()
@@ -668,6 +714,8 @@ def main():
         "clocks": clocks.summary(),
         "cpu_baseline": cpu,
         "mask_paths": paths,
+        "small_batch": {"points": small, "note": "psc_decode_step (masking pass + greedy choice + advance) at "
+                        "batch 1/16/128 on the same tables, bf16; median of 16 steps, CUDA events around each"},
         "device_timeouts": h.info().device_timeouts,
         "tables": {"classifier_states": info.n_classifier_states, "masks": info.n_masks,
                    "classifier_bytes": info.classifier_bytes, "mask_bytes": info.mask_bytes,

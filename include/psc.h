@@ -26,7 +26,8 @@
  *    synchronise.  Their return value reports argument and launch errors only.
  *  - Errors in the data (a token the mask does not allow, a stack that
  *    overflows its capacity) are per-row statuses written by the kernels;
- *    kernels never trap and never spin.
+ *    kernels never trap and never spin.  Every in-kernel wait is bounded; one
+ *    that gives up is counted on the states object (psc_state_faults).
  *  - psc_last_error() returns a thread-local message for the last failing call.
  *  - Bit v of a packed mask row is bit (v & 31) of 32-bit word (v >> 5)
  *    (least significant bit first); bits v >= V are zero.
@@ -258,6 +259,23 @@ psc_status psc_decode_step_mask(const psc_handle* h, psc_states* st, int32_t B, 
                                 int64_t row_stride, int32_t V, uint32_t* d_bitmask_out, void* stream);
 psc_status psc_decode_step_advance(const psc_handle* h, psc_states* st, int32_t B, int32_t* d_tokens,
                                    int32_t* d_row_status, void* stream);
+
+/* Faults of the bounded in-kernel waits on this states object: every wait of
+ * the masking pass and of the advance is bounded, and one that gives up (a
+ * pipeline fault; the step's logits or rows may then be incomplete, rows whose
+ * advance could not run get PSC_ROW_LIMIT) adds 1 to a counter kept in the
+ * states object (zero after psc_state_init).  Copies the counter to *h_faults
+ * and synchronises the stream; reset != 0 then zeroes it (enqueued on stream).
+ * The paper has no counterpart: this is the per-batch error word a serving
+ * loop checks between steps.  Errors: PSC_ERR_ARG, PSC_ERR_CUDA. */
+psc_status psc_state_faults(psc_states* st, int32_t* h_faults, int32_t reset, void* stream);
+
+/* Self-test of fault reporting: launches one CTA whose bounded wait, on an
+ * mbarrier phase that no thread completes, gives up after `limit` polls
+ * (1..2^24) and adds 1 to the states object's fault counter, the path a
+ * pipeline wait that gives up takes.  Nothing faults and the device stays
+ * usable.  Errors: PSC_ERR_ARG, PSC_ERR_CUDA. */
+psc_status psc_check_wait(psc_states* st, int32_t limit, void* stream);
 
 /* Copies the batch to host memory and synchronises the stream (tests and
  * debugging).  Any output pointer may be NULL.

@@ -84,6 +84,7 @@ struct DevStates {
     int B, cap;
     unsigned long long* best;   // per-row greedy-choice key (nullable)
     int32_t* rmemo;             // [B][cap] bottom-up classifier block after each stack prefix (nullable)
+    int32_t* fault;             // bounded in-kernel waits on these states that gave up (nullable)
 };
 
 }  // namespace
@@ -656,41 +657,47 @@ __device__ __forceinline__ void apply_argmax_chunk_bf16(const uint16_t* src, uin
     }
 }
 
-// One 1024-column chunk of f32 (4 elements per 16-byte piece).
+// One 1024-column chunk of f32 (4 elements per 16-byte piece), in two halves of
+// four pieces per lane (eight pieces and their bits at once exceed the register
+// budget of three resident CTAs).
 __device__ __forceinline__ void apply_argmax_chunk_f32(const uint32_t* src, uint32_t* row, int col0, uint32_t word, int lane,
                                                        Best& best, const uint4* lut) {
     const uint4 ninf = make_uint4(0xFF800000u, 0xFF800000u, 0xFF800000u, 0xFF800000u);
-    uint32_t bits[8];
-    uint4 v[8];
+#pragma unroll 1
+    for (int h = 0; h < 8; h += 4) {
+        uint32_t bits[4];
+        uint4 v[4];
 #pragma unroll
-    for (int k = 0; k < 8; k++) bits[k] = (__shfl_sync(FULL, word, k * 4 + (lane >> 3)) >> ((lane & 7) * 4)) & 0xFu;
+        for (int k = 0; k < 4; k++)
+            bits[k] = (__shfl_sync(FULL, word, (h + k) * 4 + (lane >> 3)) >> ((lane & 7) * 4)) & 0xFu;
 #pragma unroll
-    for (int k = 0; k < 8; k++)
-        if (bits[k]) v[k] = *reinterpret_cast<const uint4*>(src + (k * 32 + lane) * 4);
+        for (int k = 0; k < 4; k++)
+            if (bits[k]) v[k] = *reinterpret_cast<const uint4*>(src + ((h + k) * 32 + lane) * 4);
 #pragma unroll
-    for (int k = 0; k < 8; k++) {
-        uint32_t* p = row + col0 + (k * 32 + lane) * 4;
-        uint32_t bk = bits[k];
-        if (bk == 0) {
-            st_cs_v4(p, ninf);
-            continue;
-        }
-        uint4 am = lut[bk];
-        uint32_t x0 = sel_ninf(v[k].x, am.x, 0xFF800000u), x1 = sel_ninf(v[k].y, am.y, 0xFF800000u);
-        uint32_t x2 = sel_ninf(v[k].z, am.z, 0xFF800000u), x3 = sel_ninf(v[k].w, am.w, 0xFF800000u);
-        float mf = fmaxf(fmaxf(__uint_as_float(x0), __uint_as_float(x1)), fmaxf(__uint_as_float(x2), __uint_as_float(x3)));
-        if (best.col < 0 || mf >= best.val) {
-            uint32_t w[4] = {v[k].x, v[k].y, v[k].z, v[k].w};
+        for (int k = 0; k < 4; k++) {
+            uint32_t* p = row + col0 + ((h + k) * 32 + lane) * 4;
+            uint32_t bk = bits[k];
+            if (bk == 0) {
+                st_cs_v4(p, ninf);
+                continue;
+            }
+            uint4 am = lut[bk];
+            uint32_t x0 = sel_ninf(v[k].x, am.x, 0xFF800000u), x1 = sel_ninf(v[k].y, am.y, 0xFF800000u);
+            uint32_t x2 = sel_ninf(v[k].z, am.z, 0xFF800000u), x3 = sel_ninf(v[k].w, am.w, 0xFF800000u);
+            float mf = fmaxf(fmaxf(__uint_as_float(x0), __uint_as_float(x1)), fmaxf(__uint_as_float(x2), __uint_as_float(x3)));
+            if (best.col < 0 || mf >= best.val) {
+                uint32_t w[4] = {v[k].x, v[k].y, v[k].z, v[k].w};
 #pragma unroll
-            for (int e = 0; e < 4; e++) {
-                float f = __uint_as_float(w[e]);
-                if (((bk >> e) & 1) && f == mf) {
-                    note_best(best, f, col0 + (k * 32 + lane) * 4 + e);
-                    break;
+                for (int e = 0; e < 4; e++) {
+                    float f = __uint_as_float(w[e]);
+                    if (((bk >> e) & 1) && f == mf) {
+                        note_best(best, f, col0 + ((h + k) * 32 + lane) * 4 + e);
+                        break;
+                    }
                 }
             }
+            st_cs_v4(p, make_uint4(x0, x1, x2, x3));
         }
-        st_cs_v4(p, make_uint4(x0, x1, x2, x3));
     }
 }
 
@@ -1265,7 +1272,10 @@ __global__ void __launch_bounds__(ADV_WARPS * 32) k_advance_warp(DevTables T, De
     __syncwarp();
     if (!staged) {
         // the copy did not land: give the rows a LIMIT status, wait (bounded) for the copy, return
-        if (threadIdx.x == 0) atomicAdd(&g_pipeline_timeouts, 1);
+        if (threadIdx.x == 0) {
+            atomicAdd(&g_pipeline_timeouts, 1);
+            if (S.fault) atomicAdd(S.fault, 1);
+        }
         if (active && lane == 0) {
             if (status == ROW_OK) status = ROW_LIMIT;
             S.status[b] = status;
@@ -1714,7 +1724,25 @@ __global__ void __launch_bounds__(TMA_WARPS * 32, 3) k_step_tma(T* logits, int64
             }
         }
     }
-    if (failed && lane == 0) atomicAdd(&g_pipeline_timeouts, 1);
+    if (failed && lane == 0) {
+        atomicAdd(&g_pipeline_timeouts, 1);
+        if (S.fault) atomicAdd(S.fault, 1);
+    }
+}
+
+// A bounded wait on an mbarrier phase that nothing completes: gives up after
+// `limit` polls and records it on the states object, as the pipeline's waits do
+// (lets tests see fault reporting without any fault).
+__global__ void k_wait_gives_up(DevStates S, int limit) {
+    __shared__ __align__(8) uint64_t bar;
+    uint32_t a = smem_addr(&bar);
+    if (threadIdx.x == 0) {
+        mbar_init(a, 1);
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    __syncthreads();
+    bool ok = mbar_wait0(a, limit);   // no thread arrives
+    if (!ok && threadIdx.x == 0 && S.fault) atomicAdd(S.fault, 1);
 }
 
 // ----------------------------------------------------------------- host glue
@@ -1853,11 +1881,14 @@ psc_status launch_fused(const psc_handle* h, const psc_states* st, void* d_logit
     psc_status s;
     if (vec) {
         // the pipelined pass (rows 16-byte aligned): as many CTAs as are resident at once;
-        // items of 32 chunks; smaller (multiples of a stage) when the batch has too few
-        // chunks to give every resident CTA work
+        // items of 32 chunks; smaller when the batch has too few chunks to give every
+        // resident CTA work (multiples of a stage, down to one chunk per item: a
+        // batch-1 step spreads its 256 chunks over 256 CTAs)
         long resident = (long)sm_count(h->device) * h->tma_ctas[dtype == PSC_BF16 ? 0 : 1];
         long want = ((long)B * cpr + resident - 1) / resident;
-        int seg = (int)std::min<long>(TMA_SEG, std::max<long>(TMA_NCONS, (want + TMA_NCONS - 1) / TMA_NCONS * TMA_NCONS));
+        int seg = want >= TMA_NCONS
+                      ? (int)std::min<long>(TMA_SEG, (want + TMA_NCONS - 1) / TMA_NCONS * TMA_NCONS)
+                      : (int)std::max<long>(1, want);
         long titems = (long)B * ((cpr + seg - 1) / seg);
         int tgrid = (int)std::max(1L, std::min<long>(titems, resident));
         if (dtype == PSC_BF16)
@@ -2190,11 +2221,13 @@ psc_status psc_state_init(const psc_handle* h, int32_t B, int32_t cap, void* str
     DevStates& d = st->d;
     d.B = B;
     d.cap = cap;
-    // the bottom-up classifier's kept blocks only when the handle has that classifier
-    const int n_arr = h->d.bu ? 7 : 6;
-    void* p[7] = {};
-    size_t sz[7] = {sizeof(int32_t) * B, sizeof(int32_t) * B, sizeof(int32_t) * B, sizeof(uint16_t) * (size_t)B * cap,
-                    sizeof(int32_t) * B, sizeof(unsigned long long) * B, sizeof(int32_t) * (size_t)B * cap};
+    // the fault word, then the bottom-up classifier's kept blocks only when the handle has
+    // that classifier
+    const int n_arr = h->d.bu ? 8 : 7;
+    void* p[8] = {};
+    size_t sz[8] = {sizeof(int32_t) * B, sizeof(int32_t) * B, sizeof(int32_t) * B, sizeof(uint16_t) * (size_t)B * cap,
+                    sizeof(int32_t) * B, sizeof(unsigned long long) * B, sizeof(int32_t),
+                    sizeof(int32_t) * (size_t)B * cap};
     for (int i = 0; i < n_arr; i++) {
         s = cuda_check(cudaMalloc(&p[i], sz[i]), "cudaMalloc(states)");
         if (s != PSC_OK) {
@@ -2208,10 +2241,14 @@ psc_status psc_state_init(const psc_handle* h, int32_t B, int32_t cap, void* str
     d.stack = (uint16_t*)p[3];
     d.mid = (int32_t*)p[4];
     d.best = (unsigned long long*)p[5];
-    d.rmemo = (int32_t*)p[6];
+    d.fault = (int32_t*)p[6];
+    d.rmemo = (int32_t*)p[7];
     cudaStream_t cs = (cudaStream_t)stream;
-    k_state_init<<<(B + 255) / 256, 256, 0, cs>>>(d, h->d.q0, nullptr, B);
-    s = launch_check("k_state_init");
+    s = cuda_check(cudaMemsetAsync(d.fault, 0, sizeof(int32_t), cs), "cudaMemsetAsync(fault)");
+    if (s == PSC_OK) {
+        k_state_init<<<(B + 255) / 256, 256, 0, cs>>>(d, h->d.q0, nullptr, B);
+        s = launch_check("k_state_init");
+    }
     if (s != PSC_OK) {
         for (int j = 0; j < n_arr; j++) cudaFree(p[j]);
         return s;
@@ -2274,6 +2311,7 @@ void psc_state_destroy(psc_states* st) {
     cudaFree(st->d.stack);
     cudaFree(st->d.mid);
     cudaFree(st->d.best);
+    cudaFree(st->d.fault);
     cudaFree(st->d.rmemo);
     delete st;
 }
@@ -2413,6 +2451,26 @@ psc_status psc_states_download(const psc_states* st, int32_t* h_q, int32_t* h_de
                                     "download status")))
         return s;
     return cuda_check(cudaStreamSynchronize(cs), "cudaStreamSynchronize");
+}
+
+psc_status psc_state_faults(psc_states* st, int32_t* h_faults, int32_t reset, void* stream) {
+    if (!st || !h_faults) return fail_with(PSC_ERR_ARG, "psc_state_faults: NULL argument");
+    cudaStream_t cs = (cudaStream_t)stream;
+    psc_status s = cuda_check(cudaMemcpyAsync(h_faults, st->d.fault, sizeof(int32_t), cudaMemcpyDeviceToHost, cs),
+                              "psc_state_faults");
+    if (s == PSC_OK) s = cuda_check(cudaStreamSynchronize(cs), "cudaStreamSynchronize");
+    if (s == PSC_OK && reset)
+        s = cuda_check(cudaMemsetAsync(st->d.fault, 0, sizeof(int32_t), cs), "cudaMemsetAsync(fault)");
+    return s;
+}
+
+psc_status psc_check_wait(psc_states* st, int32_t limit, void* stream) {
+    if (!st || limit < 1 || limit > (1 << 24)) return fail_with(PSC_ERR_ARG, "psc_check_wait: bad arguments");
+    int dev = -1;
+    cudaGetDevice(&dev);
+    if (dev != st->device) return fail_with(PSC_ERR_ARG, "psc_check_wait: current device differs from the states'");
+    k_wait_gives_up<<<1, 32, 0, (cudaStream_t)stream>>>(st->d, limit);
+    return launch_check("k_wait_gives_up");
 }
 
 int32_t psc_host_classify(const psc_handle* h, int32_t q, const uint16_t* h_stack, int32_t depth, int32_t status) {

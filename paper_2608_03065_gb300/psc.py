@@ -27,7 +27,7 @@ EXPORTED = ["psc_compile", "psc_destroy", "psc_last_error", "psc_info", "psc_sta
             "psc_argmax_masked", "psc_states_download", "psc_host_classify", "psc_host_mask_row",
             "psc_host_advance", "psc_fill_apply_noalloc", "psc_fill_apply_argmax", "psc_save", "psc_load",
             "psc_decode_step", "psc_decode_step_mask", "psc_decode_step_advance", "psc_state_copy",
-            "psc_host_classify_bottom_up"]
+            "psc_host_classify_bottom_up", "psc_state_faults", "psc_check_wait"]
 NOALLOC_MAX_ROWS = 16384
 
 
@@ -91,6 +91,8 @@ def load(path: str = LIB_PATH):
         "psc_state_copy": (i32, [vp, vp, vp]),
         "psc_decode_step_advance": (i32, [vp, vp, i32, vp, vp, vp]),
         "psc_load": (i32, [ctypes.c_char_p, vp, vp]),
+        "psc_state_faults": (i32, [vp, vp, i32, vp]),
+        "psc_check_wait": (i32, [vp, i32, vp]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -376,6 +378,19 @@ def psc_decode_step_advance(h: Handle, st: States, tokens, row_status=None, stre
         raise ValueError("tokens must hold B int32 values")
     _check(load().psc_decode_step_advance(h.ptr, st.ptr, st.B, _ptr(tokens, torch.int32, "tokens", st.B),
                                           _ptr(row_status, torch.int32, "row_status", st.B), _stream(stream)))
+
+
+def psc_state_faults(st: States, reset: bool = False, stream=None) -> int:
+    """Bounded in-kernel waits on these states that gave up (synchronises the stream)."""
+    out = ctypes.c_int32(0)
+    _check(load().psc_state_faults(st.ptr, ctypes.byref(out), 1 if reset else 0, _stream(stream)))
+    return out.value
+
+
+def psc_check_wait(st: States, limit: int = 4096, stream=None):
+    """Self-test of fault reporting: a bounded wait that nothing completes gives up
+    after `limit` polls and is counted on the states object."""
+    _check(load().psc_check_wait(st.ptr, limit, _stream(stream)))
 
 
 def psc_states_download(st: States, stream=None) -> dict:

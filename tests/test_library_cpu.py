@@ -527,6 +527,8 @@ def test_c_abi_argument_errors(psc):
         lib.psc_host_mask_row(None, 0, None),
         lib.psc_host_advance(None, None, None, None, 2, None, 0),
         lib.psc_state_init(None, 4, 16, None, ctypes.byref(out)),
+        lib.psc_state_faults(None, None, 0, None),
+        lib.psc_check_wait(None, 1, None),
     ]
     assert cases == [1] * len(cases), cases
     assert lib.psc_last_error()
