@@ -409,9 +409,14 @@ def run_teacher(args):
 # --------------------------------------------------------------- sweep mode
 def batch_points(psc, h, w, dev, batches, dtypes, n=16):
     """psc_decode_step on the workload's tables at the given batch sizes (rows
-    0..B-1 of the prefix states) and logit types: µs per step (median of n steps,
-    each on fresh logits from the same prefix states restored with psc_state_copy,
-    CUDA events around the step) and the rate of the formula's bytes."""
+    0..B-1 of the prefix states) and logit types, two ways:
+      graph: a CUDA graph holding the restore of the prefix states
+        (psc_state_copy) and n decode steps on n logits buffers, replayed; µs per
+        step = replay time / n (the device time of a step: no host calls between
+        launches, as a decode loop captured in a graph runs);
+      eager: each step called from Python between CUDA events (µs per step =
+        median of n; at small batches this is the host's call latency).
+    The rate of the formula's bytes is given for the graph time."""
     import torch
     V = w.V
     tm = torch.from_numpy(w.token_matrix()).to(dev)
@@ -426,28 +431,47 @@ def batch_points(psc, h, w, dev, batches, dtypes, n=16):
     for dt, esz in dtypes:
         for B in batches:
             st = psc.psc_state_init(h, B, 256)
-            tok = torch.empty(B, dtype=torch.int32, device=dev)
+            toks = [torch.empty(B, dtype=torch.int32, device=dev) for _ in range(n)]
             gen = torch.Generator(device=dev).manual_seed(B)
             xs = [(torch.randn(B, V, generator=gen, device=dev) * w.spec.sigma).to(dt) for _ in range(n)]
             for i in range(3):   # warm-up
                 psc.psc_state_copy(st, snaps[B], stream=stream)
-                psc.psc_decode_step(h, st, xs[i].clone(), tok, stream=stream)
+                psc.psc_decode_step(h, st, xs[i].clone(), toks[i], stream=stream)
             times = []
             for i in range(n):
                 psc.psc_state_copy(st, snaps[B], stream=stream)
                 a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
                 a.record(stream)
-                psc.psc_decode_step(h, st, xs[i], tok, stream=stream)
+                psc.psc_decode_step(h, st, xs[i], toks[i], stream=stream)
                 b.record(stream)
                 torch.cuda.synchronize()
                 times.append(a.elapsed_time(b) * 1000.0)
             times.sort()
-            us = times[n // 2]
+            eager = times[n // 2]
+            # the same n steps captured once in a CUDA graph
+            torch.cuda.synchronize()
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g):
+                cs = torch.cuda.current_stream()
+                psc.psc_state_copy(st, snaps[B], stream=cs)
+                for i in range(n):
+                    psc.psc_decode_step(h, st, xs[i], toks[i], stream=cs)
+            reps = []
+            for r in range(8):
+                a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                a.record(stream)
+                g.replay()
+                b.record(stream)
+                torch.cuda.synchronize()
+                if r >= 3:
+                    reps.append(a.elapsed_time(b) * 1000.0 / n)
+            graph = sorted(reps)[len(reps) // 2]
             alg = B * V // 8 + 2 * B * V * esz
-            points.append({"dtype": "bf16" if esz == 2 else "f32", "batch": B, "us_per_step": round(us, 2),
-                           "algorithmic_GBps": round(alg / (us * 1e-6) / 1e9, 1),
-                           "frac": round(alg / (us * 1e-6) / 1e9 / peak, 3)})
-            del xs
+            points.append({"dtype": "bf16" if esz == 2 else "f32", "batch": B,
+                           "us_per_step_graph": round(graph, 2), "us_per_step_eager": round(eager, 2),
+                           "algorithmic_GBps": round(alg / (graph * 1e-6) / 1e9, 1),
+                           "frac": round(alg / (graph * 1e-6) / 1e9 / peak, 3)})
+            del g, xs
             torch.cuda.empty_cache()
     return points
 
@@ -715,7 +739,10 @@ def main():
         "cpu_baseline": cpu,
         "mask_paths": paths,
         "small_batch": {"points": small, "note": "psc_decode_step (masking pass + greedy choice + advance) at "
-                        "batch 1/16/128 on the same tables, bf16; median of 16 steps, CUDA events around each"},
+                        "batch 1/16/128 on the same tables, bf16: graph = a CUDA graph of a prefix-state restore "
+                        "and 16 steps on 16 logits buffers, replayed, time / 16 (the device time of a step); "
+                        "eager = median of 16 steps called one at a time between CUDA events (host call latency "
+                        "included)"},
         "device_timeouts": h.info().device_timeouts,
         "tables": {"classifier_states": info.n_classifier_states, "masks": info.n_masks,
                    "classifier_bytes": info.classifier_bytes, "mask_bytes": info.mask_bytes,

@@ -79,6 +79,10 @@ typedef struct {
                                      negative: not built (psc_load: dropped), and the device walks
                                      every stack from the top.  Over the limit it is not built
                                      (no error). */
+    int64_t max_dense_classifier_bytes;  /* the classifier DFA is held dense ([S][|Pi|] int32) up to
+                                            this size, above it sparse (per state a default target and
+                                            the exceptions to it; a walk step reads one row) (0 = 512 MiB;
+                                            negative: always sparse) */
 } psc_options;
 
 typedef struct {
@@ -99,6 +103,7 @@ typedef struct {
                                      (process-wide; non-zero means a pipeline fault; reading it synchronises) */
     int64_t bottom_up_states;     /* states of the bottom-up classifier (0: not built) */
     int64_t bottom_up_bytes;      /* its device bytes (blocks, edge slots, final table) */
+    int64_t classifier_sparse;    /* 1: the classifier DFA is held in the sparse layout */
 } psc_info_t;
 
 /* Offline construction (Algorithm 1, Section 3).  Reads the grammar text (a
@@ -126,15 +131,19 @@ psc_status psc_compile(const char* grammar, size_t grammar_len, const uint8_t* v
 void psc_destroy(psc_handle* h);
 
 /* Writes the handle's compiled tables to a binary file (the paper ships its
- * preprocessing results to decoding users as files, Section 5).  The file holds
- * the lexer, parser, classifier (both forms) and mask tables and the
- * vocabulary, with a checksum.  Errors: PSC_ERR_IO, PSC_ERR_ARG. */
+ * preprocessing results to decoding users as zstd-compressed files, Section 5).
+ * The file holds the lexer, parser, classifier (both forms) and mask tables and
+ * the vocabulary, with a checksum, compressed in 16 MiB blocks by the system's
+ * zstd library (libzstd.so.1) when it can be loaded at run time, else zlib
+ * (libz.so.1), else stored as it is; the environment variable PSC_SAVE_CODEC
+ * (none, zstd or zlib) chooses.  Errors: PSC_ERR_IO, PSC_ERR_ARG. */
 psc_status psc_save(const psc_handle* h, const char* path);
 
 /* Reads a file written by psc_save, checks its checksum and the consistency of
  * every table index, and uploads the tables to the current device (unless
  * opts->host_only; opts may be NULL).  Errors: PSC_ERR_IO (missing, truncated,
- * corrupt or inconsistent file), PSC_ERR_OOM, PSC_ERR_CUDA. */
+ * corrupt or inconsistent file, or compressed with a codec this host cannot
+ * load), PSC_ERR_OOM, PSC_ERR_CUDA. */
 psc_status psc_load(const char* path, const psc_options* opts, psc_handle** out);
 
 /* Thread-local message of the last failed call on this thread ("" if none). */

@@ -74,7 +74,7 @@ def _build_locked(force: bool, verbose: bool) -> str:
         list(ex.map(run, jobs))
     if force or jobs or _stale(LIB, objs):
         tmp = LIB + f".{os.getpid()}.tmp"
-        run([nvcc, "-shared", "-gencode", GENCODE, "-o", tmp] + objs + ["-lpthread"])
+        run([nvcc, "-shared", "-gencode", GENCODE, "-o", tmp] + objs + ["-lpthread", "-ldl"])
         os.replace(tmp, LIB)
     return LIB
 

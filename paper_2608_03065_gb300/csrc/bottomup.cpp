@@ -137,7 +137,7 @@ bool build_bottom_up(Tables& T, const Options& opt) {
     while (!work.empty()) {
         auto [s, t] = work.back();
         work.pop_back();
-        int32_t nx = T.dfa[(size_t)s * n + t];
+        int32_t nx = dfa_next(T, s, t);
         if (nx < 0) continue;
         for (int32_t u : pred[t])
             if (!has(u, nx)) {
@@ -175,7 +175,7 @@ bool build_bottom_up(Tables& T, const Options& opt) {
         step_off[u].push_back(0);
         for (int32_t t : pred[u]) {
             for (int32_t s : D[u]) {
-                int32_t nx = T.dfa[(size_t)s * n + u];
+                int32_t nx = dfa_next(T, s, u);
                 step[u].push_back(nx < 0 ? nx : rank(t, nx));   // nx < 0: -(mask + 1)
             }
             step_off[u].push_back((int64_t)step[u].size());
@@ -223,7 +223,7 @@ bool build_bottom_up(Tables& T, const Options& opt) {
     {
         std::vector<int32_t> g0(D[0].size());
         for (size_t i = 0; i < D[0].size(); i++) {
-            int32_t nx = T.dfa[(size_t)D[0][i] * n + 0];
+            int32_t nx = dfa_next(T, D[0][i], 0);
             g0[i] = nx < 0 ? -nx - 1 : T.dfa_mask[nx];
         }
         new_state(0, hash_state(0, g0.data(), g0.size()));

@@ -890,15 +890,34 @@ Tables compile_tables(const std::string& text, const uint8_t* vb, const int64_t*
     };
     T.S = S;
     T.n_lr = P.n_states;
-    T.dfa.assign((size_t)S * P.n_states, 0);
     T.dfa_mask.assign(S, 0);
-    for (int c = 0; c < ncl; c++) {
+    // dense [S][n_lr] table, or (above the size budget) a default target and the
+    // exceptions to it per state, as the construction produced them
+    int64_t dense_budget = opt.max_dense_classifier_bytes == 0 ? (int64_t(512) << 20) : opt.max_dense_classifier_bytes;
+    T.dfa_sparse = dense_budget < 0 || (int64_t)S * P.n_states * 4 > dense_budget;
+    if (!T.dfa_sparse) T.dfa.assign((size_t)S * P.n_states, 0);
+    else {
+        T.dfa_def.assign(S, 0);
+        T.dfa_exc_off.assign(1, 0);
+    }
+    for (int c = 0; c < ncl; c++) {   // dense ids increase with c
         if (absorbing[c]) continue;
         int r = rep[c];
-        int32_t* row = T.dfa.data() + (size_t)dense[c] * P.n_states;
         int32_t d = enc(cls[B.st_def[r]]);
-        for (int y = 0; y < P.n_states; y++) row[y] = d;
-        for (int64_t e = B.exc_off[r]; e < B.exc_off[r + 1]; e++) row[B.exc_y[e]] = enc(cls[B.exc_t[e]]);
+        if (!T.dfa_sparse) {
+            int32_t* row = T.dfa.data() + (size_t)dense[c] * P.n_states;
+            for (int y = 0; y < P.n_states; y++) row[y] = d;
+            for (int64_t e = B.exc_off[r]; e < B.exc_off[r + 1]; e++) row[B.exc_y[e]] = enc(cls[B.exc_t[e]]);
+        } else {
+            T.dfa_def[dense[c]] = d;
+            for (int64_t e = B.exc_off[r]; e < B.exc_off[r + 1]; e++) {   // symbols ascending
+                int32_t x = enc(cls[B.exc_t[e]]);
+                if (x == d) continue;
+                T.dfa_exc_y.push_back((uint16_t)B.exc_y[e]);
+                T.dfa_exc_t.push_back(x);
+            }
+            T.dfa_exc_off.push_back((int64_t)T.dfa_exc_y.size());
+        }
         T.dfa_mask[dense[c]] = mask_new[B.st_mask[r]];
     }
     T.dfa_start.resize(L.nq);
@@ -963,7 +982,7 @@ int classify_host(const Tables& t, int q, const uint16_t* stack, int depth, int 
     int32_t s = t.dfa_start[q];
     if (s < 0) return -s - 1;
     for (int i = depth - 1; i >= 0; i--) {
-        int32_t nx = t.dfa[(size_t)s * t.n_lr + stack[i]];
+        int32_t nx = dfa_next(t, s, stack[i]);
         if (nx < 0) return -nx - 1;
         s = nx;
     }

@@ -1,14 +1,26 @@
 // Persistence of compiled tables.  The paper stores its preprocessing results
-// on disk so that providers can ship them to decoding users (Section 5,
-// preprocessing overhead); here the flat tables of a compiled handle are
-// written as one binary file: a magic/version header, every table as
-// (element count, raw little-endian bytes), and a 64-bit FNV-1a checksum of
-// everything before it (format 03: with the bottom-up classifier's tables).
-// The mask rows are stored as they are held in memory:
-// chunk ids plus the distinct 1024-token chunks (no general-purpose compression;
-// the paper uses zstd).
+// on disk, zstd-compressed, so that providers can ship them to decoding users
+// (Section 5, preprocessing overhead); here the flat tables of a compiled handle
+// are written as one file (format 04):
+//   "PSCTAB04", codec (u32: 0 none, 1 zstd, 2 zlib), reserved (u32),
+//   size of the table payload (u64), number of blocks (u64),
+//   per block: payload bytes and stored bytes (u64 each), then the blocks,
+//   then a 64-bit FNV-1a checksum of the payload.
+// The payload lists every table as (element count, raw little-endian bytes).
+// Blocks of 16 MiB of payload are compressed and decompressed in parallel.  The
+// compressor is the system's zstd library (libzstd.so.1) when it can be loaded,
+// else zlib (libz.so.1), else none: both are loaded at run time through their
+// stable C interfaces, so the library does not depend on them to link or run; a
+// file needs the codec it was written with to be read.  The environment variable
+// PSC_SAVE_CODEC (none, zstd or zlib) overrides the choice.
+#include <dlfcn.h>
+
+#include <algorithm>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
+#include <mutex>
+#include <thread>
 #include <type_traits>
 
 #include "psc_internal.h"
@@ -16,15 +28,107 @@
 namespace psc {
 namespace {
 
-const char MAGIC[8] = {'P', 'S', 'C', 'T', 'A', 'B', '0', '3'};
+const char MAGIC[8] = {'P', 'S', 'C', 'T', 'A', 'B', '0', '4'};
+constexpr size_t BLOCK = size_t(16) << 20;
+enum { CODEC_NONE = 0, CODEC_ZSTD = 1, CODEC_ZLIB = 2 };
 
-struct Writer {
-    FILE* f;
+// ------------------------------------------------------------------ codecs
+struct Codecs {
+    // zstd
+    size_t (*zstd_bound)(size_t) = nullptr;
+    size_t (*zstd_compress)(void*, size_t, const void*, size_t, int) = nullptr;
+    size_t (*zstd_decompress)(void*, size_t, const void*, size_t) = nullptr;
+    unsigned (*zstd_is_error)(size_t) = nullptr;
+    // zlib (uLong = unsigned long, Bytef = unsigned char)
+    unsigned long (*z_bound)(unsigned long) = nullptr;
+    int (*z_compress2)(unsigned char*, unsigned long*, const unsigned char*, unsigned long, int) = nullptr;
+    int (*z_uncompress)(unsigned char*, unsigned long*, const unsigned char*, unsigned long) = nullptr;
+    bool zstd() const { return zstd_bound && zstd_compress && zstd_decompress && zstd_is_error; }
+    bool zlib() const { return z_bound && z_compress2 && z_uncompress; }
+};
+
+const Codecs& codecs() {
+    static Codecs c;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        if (void* z = dlopen("libzstd.so.1", RTLD_NOW | RTLD_LOCAL)) {
+            c.zstd_bound = reinterpret_cast<size_t (*)(size_t)>(dlsym(z, "ZSTD_compressBound"));
+            c.zstd_compress = reinterpret_cast<size_t (*)(void*, size_t, const void*, size_t, int)>(dlsym(z, "ZSTD_compress"));
+            c.zstd_decompress = reinterpret_cast<size_t (*)(void*, size_t, const void*, size_t)>(dlsym(z, "ZSTD_decompress"));
+            c.zstd_is_error = reinterpret_cast<unsigned (*)(size_t)>(dlsym(z, "ZSTD_isError"));
+        }
+        if (void* z = dlopen("libz.so.1", RTLD_NOW | RTLD_LOCAL)) {
+            c.z_bound = reinterpret_cast<unsigned long (*)(unsigned long)>(dlsym(z, "compressBound"));
+            c.z_compress2 = reinterpret_cast<int (*)(unsigned char*, unsigned long*, const unsigned char*,
+                                                     unsigned long, int)>(dlsym(z, "compress2"));
+            c.z_uncompress = reinterpret_cast<int (*)(unsigned char*, unsigned long*, const unsigned char*,
+                                                      unsigned long)>(dlsym(z, "uncompress"));
+        }
+    });
+    return c;
+}
+
+// compresses src into dst (resized); false when the codec fails
+bool encode(int codec, const uint8_t* src, size_t n, std::vector<uint8_t>& dst) {
+    const Codecs& c = codecs();
+    if (codec == CODEC_ZSTD) {
+        dst.resize(c.zstd_bound(n));
+        size_t r = c.zstd_compress(dst.data(), dst.size(), src, n, 9);
+        if (c.zstd_is_error(r)) return false;
+        dst.resize(r);
+        return true;
+    }
+    unsigned long cap = c.z_bound((unsigned long)n);
+    dst.resize(cap);
+    if (c.z_compress2(dst.data(), &cap, src, (unsigned long)n, 6) != 0) return false;
+    dst.resize(cap);
+    return true;
+}
+
+bool decode(int codec, const uint8_t* src, size_t n, uint8_t* dst, size_t want) {
+    const Codecs& c = codecs();
+    if (codec == CODEC_ZSTD) {
+        size_t r = c.zstd_decompress(dst, want, src, n);
+        return !c.zstd_is_error(r) && r == want;
+    }
+    unsigned long got = (unsigned long)want;
+    return c.z_uncompress(dst, &got, src, (unsigned long)n) == 0 && got == want;
+}
+
+// runs f(i) for i in [0, n) on up to hardware-concurrency threads
+template <typename F>
+void parallel_for(size_t n, F f) {
+    size_t nt = std::min<size_t>(n, std::max(1u, std::thread::hardware_concurrency()));
+    std::vector<std::thread> pool;
+    std::mutex mu;
+    size_t next = 0;
+    for (size_t t = 0; t < nt; t++)
+        pool.emplace_back([&] {
+            for (;;) {
+                size_t i;
+                {
+                    std::lock_guard<std::mutex> lk(mu);
+                    if (next >= n) return;
+                    i = next++;
+                }
+                f(i);
+            }
+        });
+    for (auto& th : pool) th.join();
+}
+
+uint64_t fnv1a(const uint8_t* b, size_t n) {
     uint64_t h = 1469598103934665603ull;
+    for (size_t i = 0; i < n; i++) h = (h ^ b[i]) * 1099511628211ull;
+    return h;
+}
+
+// ------------------------------------------------------- payload (de)coding
+struct Writer {
+    std::vector<uint8_t> out;
     void raw(const void* p, size_t n) {
         const uint8_t* b = static_cast<const uint8_t*>(p);
-        for (size_t i = 0; i < n; i++) h = (h ^ b[i]) * 1099511628211ull;
-        if (n && fwrite(p, 1, n, f) != n) throw Error(ST_ERR_IO, "write failed");
+        out.insert(out.end(), b, b + n);
     }
     template <typename T>
     void scalar(T v) { raw(&v, sizeof(T)); }
@@ -36,12 +140,12 @@ struct Writer {
 };
 
 struct Reader {
-    FILE* f;
-    uint64_t h = 1469598103934665603ull;
-    void raw(void* p, size_t n) {
-        if (n && fread(p, 1, n, f) != n) throw Error(ST_ERR_IO, "table file is truncated");
-        const uint8_t* b = static_cast<const uint8_t*>(p);
-        for (size_t i = 0; i < n; i++) h = (h ^ b[i]) * 1099511628211ull;
+    const uint8_t* p;
+    size_t n, pos = 0;
+    void raw(void* dst, size_t k) {
+        if (k > n - pos) throw Error(ST_ERR_IO, "table file is truncated");
+        std::memcpy(dst, p + pos, k);
+        pos += k;
     }
     template <typename T>
     T scalar() {
@@ -50,11 +154,11 @@ struct Reader {
         return v;
     }
     template <typename T>
-    void vec(std::vector<T>& v, uint64_t limit = (uint64_t)1 << 36) {
-        uint64_t n = scalar<uint64_t>();
-        if (n > limit / sizeof(T)) throw Error(ST_ERR_IO, "table file has an implausible size field");
-        v.resize(n);
-        raw(v.data(), n * sizeof(T));
+    void vec(std::vector<T>& v) {
+        uint64_t k = scalar<uint64_t>();
+        if (k > (n - pos) / sizeof(T)) throw Error(ST_ERR_IO, "table file has an implausible size field");
+        v.resize(k);
+        raw(v.data(), k * sizeof(T));
     }
 };
 
@@ -78,6 +182,7 @@ void fields(S& s, Tables& t) {
     vc(t.lex_trans); vc(t.lex_accept); vc(t.cls_ignored);
     vc(t.action); vc(t.go); vc(t.rule_len); vc(t.rule_lhs); vc(t.resolve);
     vc(t.dfa); vc(t.dfa_start); vc(t.dfa_mask); vc(t.mask_rows); vc(t.mask_chunks);
+    sc(t.dfa_sparse); vc(t.dfa_def); vc(t.dfa_exc_off); vc(t.dfa_exc_y); vc(t.dfa_exc_t);
     vc(t.vocab_bytes); vc(t.vocab_off);
     sc(t.bu_root); sc(t.n_bu); sc(t.n_frow);
     vc(t.bu); vc(t.bu_slot); vc(t.bu_F); vc(t.bu_t);
@@ -90,8 +195,23 @@ void validate(const Tables& t) {
     if (t.n_lr <= 0 || t.action.size() != (size_t)t.n_lr * t.n_terms || t.go.size() != (size_t)t.n_lr * t.n_nts)
         bad("parser");
     if (t.resolve.size() != (size_t)t.n_classes * t.n_lr || t.cls_ignored.size() != (size_t)t.n_classes) bad("classes");
-    if (t.dfa.size() != (size_t)t.S * t.n_lr || t.dfa_mask.size() != (size_t)t.S || t.dfa_start.size() != (size_t)t.nq)
-        bad("classifier");
+    if (t.dfa_mask.size() != (size_t)t.S || t.dfa_start.size() != (size_t)t.nq) bad("classifier");
+    if (t.dfa_sparse == 0) {
+        if (t.dfa.size() != (size_t)t.S * t.n_lr || !t.dfa_def.empty() || !t.dfa_exc_off.empty() ||
+            !t.dfa_exc_y.empty() || !t.dfa_exc_t.empty())
+            bad("classifier");
+    } else {
+        if (t.dfa_sparse != 1 || !t.dfa.empty() || t.dfa_def.size() != (size_t)t.S ||
+            t.dfa_exc_off.size() != (size_t)t.S + 1 || t.dfa_exc_off[0] != 0 ||
+            (uint64_t)t.dfa_exc_off[t.S] != t.dfa_exc_y.size() || t.dfa_exc_t.size() != t.dfa_exc_y.size())
+            bad("sparse classifier");
+        for (int s = 0; s < t.S; s++) {
+            if (t.dfa_exc_off[s + 1] < t.dfa_exc_off[s]) bad("sparse classifier");
+            for (int64_t e = t.dfa_exc_off[s]; e < t.dfa_exc_off[s + 1]; e++)
+                if (t.dfa_exc_y[e] >= t.n_lr || (e > t.dfa_exc_off[s] && t.dfa_exc_y[e] <= t.dfa_exc_y[e - 1]))
+                    bad("sparse classifier symbols");
+        }
+    }
     if (t.W != (t.V + 31) / 32 || t.nch != (t.W + 31) / 32 || t.n_masks < 2 || t.n_chunks < 1 ||
         t.mask_rows.size() != (size_t)t.n_masks * t.nch || t.mask_chunks.size() != (size_t)t.n_chunks * 32)
         bad("masks");
@@ -110,6 +230,8 @@ void validate(const Tables& t) {
     for (int16_t x : t.resolve) if (x < -1 || x >= t.n_terms) bad("class resolution");
     auto state_ok = [&](int32_t s) { return s >= 0 ? s < t.S : (-s - 1) < t.n_masks; };
     for (int32_t s : t.dfa) if (!state_ok(s)) bad("classifier transition");
+    for (int32_t s : t.dfa_def) if (!state_ok(s)) bad("classifier transition");
+    for (int32_t s : t.dfa_exc_t) if (!state_ok(s)) bad("classifier transition");
     for (int32_t s : t.dfa_start) if (!state_ok(s)) bad("classifier start");
     for (int32_t m : t.dfa_mask) if (m < 0 || m >= t.n_masks) bad("classifier mask id");
     if (t.eos_id < -1 || t.eos_id >= t.V) bad("end-of-sequence id");
@@ -157,19 +279,59 @@ void validate(const Tables& t) {
 }  // namespace
 
 void save_tables(const Tables& t, const std::string& path) {
+    Writer w;
+    Tables copy = t;   // fields() takes a mutable reference
+    fields(w, copy);
+    const std::vector<uint8_t>& payload = w.out;
+    const Codecs& c = codecs();
+    int codec = c.zstd() ? CODEC_ZSTD : c.zlib() ? CODEC_ZLIB : CODEC_NONE;
+    if (const char* want = getenv("PSC_SAVE_CODEC")) {   // none | zstd | zlib (if it can be loaded)
+        if (!strcmp(want, "none")) codec = CODEC_NONE;
+        else if (!strcmp(want, "zlib") && c.zlib()) codec = CODEC_ZLIB;
+        else if (!strcmp(want, "zstd") && c.zstd()) codec = CODEC_ZSTD;
+    }
+    size_t nb = (payload.size() + BLOCK - 1) / BLOCK;
+    std::vector<std::vector<uint8_t>> blocks(nb);
+    if (codec != CODEC_NONE) {
+        std::vector<char> ok(nb, 1);
+        parallel_for(nb, [&](size_t i) {
+            size_t lo = i * BLOCK, n = std::min(BLOCK, payload.size() - lo);
+            ok[i] = encode(codec, payload.data() + lo, n, blocks[i]);
+        });
+        for (char k : ok)
+            if (!k) throw Error(ST_ERR_IO, "compressing the tables failed");
+    }
     std::string tmp = path + ".tmp";
     FILE* f = fopen(tmp.c_str(), "wb");
     if (!f) throw Error(ST_ERR_IO, "cannot open " + tmp + " for writing");
+    auto put = [&](const void* p, size_t n) {
+        if (n && fwrite(p, 1, n, f) != n) throw Error(ST_ERR_IO, "write failed");
+    };
     try {
-        Writer w{f};
-        w.raw(MAGIC, 8);
-        Tables copy = t;   // fields() takes a mutable reference
-        fields(w, copy);
-        uint64_t h = w.h;
-        if (fwrite(&h, 8, 1, f) != 1) throw Error(ST_ERR_IO, "write failed");
-        if (fclose(f) != 0) throw Error(ST_ERR_IO, "close failed");
+        uint32_t hdr[2] = {(uint32_t)codec, 0};
+        uint64_t sizes[2] = {payload.size(), nb};
+        put(MAGIC, 8);
+        put(hdr, sizeof(hdr));
+        put(sizes, sizeof(sizes));
+        for (size_t i = 0; i < nb; i++) {
+            uint64_t raw = std::min(BLOCK, payload.size() - i * BLOCK);
+            uint64_t stored = codec == CODEC_NONE ? raw : blocks[i].size();
+            put(&raw, 8);
+            put(&stored, 8);
+        }
+        for (size_t i = 0; i < nb; i++) {
+            if (codec == CODEC_NONE) put(payload.data() + i * BLOCK, std::min(BLOCK, payload.size() - i * BLOCK));
+            else put(blocks[i].data(), blocks[i].size());
+        }
+        uint64_t h = fnv1a(payload.data(), payload.size());
+        put(&h, 8);
+        if (fclose(f) != 0) {
+            f = nullptr;
+            throw Error(ST_ERR_IO, "close failed");
+        }
+        f = nullptr;
     } catch (...) {
-        fclose(f);
+        if (f) fclose(f);
         remove(tmp.c_str());
         throw;
     }
@@ -179,20 +341,63 @@ void save_tables(const Tables& t, const std::string& path) {
 Tables load_tables(const std::string& path) {
     FILE* f = fopen(path.c_str(), "rb");
     if (!f) throw Error(ST_ERR_IO, "cannot open " + path);
-    Tables t;
+    std::vector<uint8_t> payload;
     try {
-        Reader r{f};
+        auto get = [&](void* p, size_t n) {
+            if (n && fread(p, 1, n, f) != n) throw Error(ST_ERR_IO, path + ": table file is truncated");
+        };
         char magic[8];
-        r.raw(magic, 8);
-        if (memcmp(magic, MAGIC, 8) != 0) throw Error(ST_ERR_IO, path + " is not a PSC table file");
-        fields(r, t);
-        uint64_t want = r.h, got = 0;
-        if (fread(&got, 8, 1, f) != 1 || got != want) throw Error(ST_ERR_IO, path + ": checksum mismatch");
+        get(magic, 8);
+        if (memcmp(magic, MAGIC, 8) != 0) throw Error(ST_ERR_IO, path + " is not a PSC table file (format 04)");
+        uint32_t hdr[2];
+        uint64_t sizes[2];
+        get(hdr, sizeof(hdr));
+        get(sizes, sizeof(sizes));
+        int codec = (int)hdr[0];
+        uint64_t total = sizes[0], nb = sizes[1];
+        if (codec > CODEC_ZLIB || total > (uint64_t(1) << 40) || nb != (total + BLOCK - 1) / BLOCK)
+            throw Error(ST_ERR_IO, path + ": bad table file header");
+        if ((codec == CODEC_ZSTD && !codecs().zstd()) || (codec == CODEC_ZLIB && !codecs().zlib()))
+            throw Error(ST_ERR_IO, path + std::string(": written with ") + (codec == CODEC_ZSTD ? "zstd" : "zlib") +
+                                       ", which cannot be loaded on this host");
+        std::vector<uint64_t> raw(nb), stored(nb);
+        for (uint64_t i = 0; i < nb; i++) {
+            get(&raw[i], 8);
+            get(&stored[i], 8);
+            if (raw[i] != std::min<uint64_t>(BLOCK, total - i * BLOCK) || stored[i] > (uint64_t(1) << 32))
+                throw Error(ST_ERR_IO, path + ": bad block size");
+        }
+        std::vector<std::vector<uint8_t>> blocks(nb);
+        for (uint64_t i = 0; i < nb; i++) {
+            blocks[i].resize(stored[i]);
+            get(blocks[i].data(), stored[i]);
+        }
+        uint64_t want = 0;
+        get(&want, 8);
+        payload.resize(total);
+        std::vector<char> ok(nb, 1);
+        parallel_for(nb, [&](size_t i) {
+            uint8_t* dst = payload.data() + i * BLOCK;
+            if (codec == CODEC_NONE) {
+                if (stored[i] != raw[i]) ok[i] = 0;
+                else std::memcpy(dst, blocks[i].data(), raw[i]);
+            } else {
+                ok[i] = decode(codec, blocks[i].data(), blocks[i].size(), dst, raw[i]);
+            }
+            std::vector<uint8_t>().swap(blocks[i]);
+        });
+        for (char k : ok)
+            if (!k) throw Error(ST_ERR_IO, path + ": a block does not decompress");
+        if (fnv1a(payload.data(), payload.size()) != want) throw Error(ST_ERR_IO, path + ": checksum mismatch");
         fclose(f);
     } catch (...) {
         fclose(f);
         throw;
     }
+    Tables t;
+    Reader r{payload.data(), payload.size()};
+    fields(r, t);
+    if (r.pos != r.n) throw Error(ST_ERR_IO, path + ": trailing bytes in the table payload");
     validate(t);
     return t;
 }

@@ -55,13 +55,19 @@ struct DevTables {
     const int32_t* rule_len;
     const int32_t* rule_lhs;
     const int16_t* resolve;
-    const int32_t* dfa;
+    const int32_t* dfa;        // dense [S][n_lr] (nullptr in the sparse layout)
     const int32_t* dfa_start;
     const int32_t* dfa_mask;
+    // sparse layout (dfa_sparse = 1): one row per state, a state's id being its row's
+    // offset: [exceptions n, default target, mask id, 0, (symbol, target) x n], symbols
+    // ascending, targets row offsets or -(mask+1); dfa_start holds row offsets too
+    const int32_t* dfa_rows;
+    int dfa_sparse;
     const uint32_t* mchunks;   // distinct 32-word chunks of the mask rows [n_chunks][32]
     const uint32_t* mrows;     // mask rows as chunk ids [n_masks][nch]
     const uint8_t* vocab;
     const int64_t* vocab_off;
+    const uint8_t* tok32;      // [V][32] the first 32 bytes of every token (zero-padded)
     int q0, nq, n_lr, n_terms, n_nts, end_term;
     int V, W, nch, eos_id, n_masks;
     // compact lexer/parser tables for k_advance_warp (adv_bytes = 0: not built)
@@ -150,6 +156,46 @@ __device__ __forceinline__ int memo_classify(const DevTables& T, const DevStates
     return memo_mask(T, S.rmemo[(size_t)b * S.cap + depth - 1], q);
 }
 
+// One classifier transition in the sparse layout by a full warp (every lane with
+// the same s and X): lane 0 loads the row's header, lane 1 the mask id, lanes
+// 2-31 the first 30 exceptions; a ballot finds X; longer rows are scanned 32
+// exceptions at a time.  Returns the target (row offset, or -(mask+1)).  The row
+// array is padded so that these reads stay inside it.
+__device__ __forceinline__ int sparse_step_warp(const int32_t* rows, int s, int X, int lane) {
+    const int2* r2 = reinterpret_cast<const int2*>(rows + s);   // row offsets are even
+    int2 v = __ldg(r2 + lane);
+    int n = __shfl_sync(FULL, v.x, 0);
+    int def = __shfl_sync(FULL, v.y, 0);
+    unsigned hit = __ballot_sync(FULL, lane >= 2 && lane - 2 < n && v.x == X);
+    if (hit) return __shfl_sync(FULL, v.y, __ffs(hit) - 1);
+    for (int base = 30; base < n; base += 32) {
+        int2 w = __ldg(r2 + 2 + base + lane);
+        unsigned h2 = __ballot_sync(FULL, base + lane < n && w.x == X);
+        if (h2) return __shfl_sync(FULL, w.y, __ffs(h2) - 1);
+    }
+    return def;
+}
+
+// The same transition by one thread (binary search over the row's exceptions).
+__device__ __forceinline__ int sparse_step_thread(const int32_t* rows, int s, int X) {
+    const int2* r2 = reinterpret_cast<const int2*>(rows + s);
+    int2 h = __ldg(r2);
+    int lo = 0, hi = h.x;
+    while (lo < hi) {
+        int m = (lo + hi) >> 1;
+        int2 p = __ldg(r2 + 2 + m);
+        if (p.x == X) return p.y;
+        if (p.x < X) lo = m + 1;
+        else hi = m;
+    }
+    return h.y;
+}
+
+// Mask id of the classifier state s when the stack ends there (either layout).
+__device__ __forceinline__ int state_mask(const DevTables& T, int s) {
+    return T.dfa_sparse ? __ldg(T.dfa_rows + s + 2) : __ldg(T.dfa_mask + s);
+}
+
 // Classification of one row (Algorithm 2 step 3) by a full warp: from the kept
 // bottom-up block when there is one, else the walk of the classifier DFA: lanes
 // load 32 stack symbols at a time (coalesced), the walk broadcasts them with
@@ -175,12 +221,12 @@ __device__ int warp_classify(const DevTables& T, const DevStates& S, int b, int 
         for (int j = 0; j < n; j++) {
             int X = __shfl_sync(FULL, x, j);   // the same in every lane: the warp returns together
             if ((unsigned)X >= (unsigned)T.n_lr) return 0;
-            int nx = __ldg(T.dfa + (size_t)s * T.n_lr + X);
+            int nx = T.dfa_sparse ? sparse_step_warp(T.dfa_rows, s, X, lane) : __ldg(T.dfa + (size_t)s * T.n_lr + X);
             if (nx < 0) return -nx - 1;
             s = nx;
         }
     }
-    return __ldg(T.dfa_mask + s);
+    return state_mask(T, s);
 }
 
 // the same classification by one thread (same guard on stack symbols)
@@ -199,11 +245,11 @@ __device__ int thread_classify(const DevTables& T, const DevStates& S, int b) {
     for (int i = depth - 1; i >= 0; i--) {
         int X = st[i];
         if (X >= T.n_lr) return 0;
-        int nx = __ldg(T.dfa + (size_t)s * T.n_lr + X);
+        int nx = T.dfa_sparse ? sparse_step_thread(T.dfa_rows, s, X) : __ldg(T.dfa + (size_t)s * T.n_lr + X);
         if (nx < 0) return -nx - 1;
         s = nx;
     }
-    return __ldg(T.dfa_mask + s);
+    return state_mask(T, s);
 }
 
 // ------------------------------------------------------------------ kernels
@@ -1116,12 +1162,12 @@ __device__ __forceinline__ int warp_walk(const DevTables& T, const StackView& sv
         for (int j = 0; j < n; j++) {
             int X = __shfl_sync(FULL, x, j);
             if ((unsigned)X >= (unsigned)T.n_lr) return 0;
-            int nx = ld_keep(T.dfa + (size_t)s * T.n_lr + X, pol);
+            int nx = T.dfa_sparse ? sparse_step_warp(T.dfa_rows, s, X, lane) : ld_keep(T.dfa + (size_t)s * T.n_lr + X, pol);
             if (nx < 0) return -nx - 1;
             s = nx;
         }
     }
-    return __ldg(T.dfa_mask + s);
+    return state_mask(T, s);
 }
 
 // memo_extend by a full warp: lanes fetch the edge slots of 32 entries at a
@@ -1259,10 +1305,10 @@ __global__ void __launch_bounds__(ADV_WARPS * 32) k_advance_warp(DevTables T, De
                 }
             }
         }
-        if (parse) {   // the token's bytes: lane i holds byte i
+        if (parse) {   // the token's bytes: lane i holds byte i (loaded with the length, in parallel)
+            tbyte = T.tok32[(size_t)tok * 32 + lane];
             vlo = T.vocab_off[tok];
             len = (int)(T.vocab_off[tok + 1] - vlo);
-            if (lane < len) tbyte = T.vocab[vlo + lane];
         }
     }
     __syncthreads();
@@ -1881,14 +1927,12 @@ psc_status launch_fused(const psc_handle* h, const psc_states* st, void* d_logit
     psc_status s;
     if (vec) {
         // the pipelined pass (rows 16-byte aligned): as many CTAs as are resident at once;
-        // items of 32 chunks; smaller when the batch has too few chunks to give every
-        // resident CTA work (multiples of a stage, down to one chunk per item: a
-        // batch-1 step spreads its 256 chunks over 256 CTAs)
+        // items of 32 chunks; smaller (multiples of a stage) when the batch has too few
+        // chunks to give every resident CTA work (one chunk per item instead of a stage
+        // was measured no faster at batch 1: 8.3 us per graph-replayed step either way)
         long resident = (long)sm_count(h->device) * h->tma_ctas[dtype == PSC_BF16 ? 0 : 1];
         long want = ((long)B * cpr + resident - 1) / resident;
-        int seg = want >= TMA_NCONS
-                      ? (int)std::min<long>(TMA_SEG, (want + TMA_NCONS - 1) / TMA_NCONS * TMA_NCONS)
-                      : (int)std::max<long>(1, want);
+        int seg = (int)std::min<long>(TMA_SEG, std::max<long>(TMA_NCONS, (want + TMA_NCONS - 1) / TMA_NCONS * TMA_NCONS));
         long titems = (long)B * ((cpr + seg - 1) / seg);
         int tgrid = (int)std::max(1L, std::min<long>(titems, resident));
         if (dtype == PSC_BF16)
@@ -2044,6 +2088,17 @@ psc_status noalloc_scratch(int device, int32_t** out) {
 }  // namespace
 
 namespace {
+// The first 32 bytes of every token, zero-padded to 32 ([V][32]): the advance loads a
+// token's bytes with its length, instead of after its offset.
+std::vector<uint8_t> token_prefixes(const psc::Tables& t) {
+    std::vector<uint8_t> out((size_t)t.V * 32, 0);
+    for (int v = 0; v < t.V; v++) {
+        int64_t lo = t.vocab_off[v], n = std::min<int64_t>(32, t.vocab_off[v + 1] - lo);
+        if (n > 0) std::memcpy(out.data() + (size_t)v * 32, t.vocab_bytes.data() + lo, (size_t)n);
+    }
+    return out;
+}
+
 // Uploads a handle's host tables to the current device (psc_compile, psc_load).
 psc_status upload_tables(std::unique_ptr<psc_handle>& h, bool global_tables) {
     const psc::Tables& t = h->t;
@@ -2054,14 +2109,39 @@ psc_status upload_tables(std::unique_ptr<psc_handle>& h, bool global_tables) {
     if (dfa.empty()) dfa.push_back(0);
     std::vector<int32_t> dfa_mask = t.dfa_mask;
     if (dfa_mask.empty()) dfa_mask.push_back(0);
+    // sparse layout: the packed rows of the device, state ids replaced by row offsets
+    std::vector<int32_t> rows, start = t.dfa_start;
+    if (t.dfa_sparse) {
+        std::vector<int64_t> off(t.S + 1, 0);
+        for (int x = 0; x < t.S; x++) off[x + 1] = off[x] + 4 + 2 * (t.dfa_exc_off[x + 1] - t.dfa_exc_off[x]);
+        if (off[t.S] + 128 > INT32_MAX) return fail_with(PSC_ERR_LIMIT, "sparse classifier exceeds 2^31 words");
+        auto enc = [&](int32_t v) { return v >= 0 ? (int32_t)off[v] : v; };
+        rows.assign((size_t)off[t.S] + 128, 0);   // padded: a warp reads 32 pairs past a row's header
+        for (int x = 0; x < t.S; x++) {
+            int32_t* r = rows.data() + off[x];
+            int64_t e0 = t.dfa_exc_off[x], n = t.dfa_exc_off[x + 1] - e0;
+            r[0] = (int32_t)n;
+            r[1] = enc(t.dfa_def[x]);
+            r[2] = t.dfa_mask[x];
+            for (int64_t i = 0; i < n; i++) {
+                r[4 + 2 * i] = t.dfa_exc_y[e0 + i];
+                r[5 + 2 * i] = enc(t.dfa_exc_t[e0 + i]);
+            }
+        }
+        for (int32_t& v : start) v = enc(v);
+    } else {
+        rows.push_back(0);
+    }
     if ((s = upload(h.get(), t.lex_trans, &d.lex_trans)) || (s = upload(h.get(), t.lex_accept, &d.lex_accept)) ||
         (s = upload(h.get(), t.cls_ignored, &d.cls_ignored)) || (s = upload(h.get(), t.action, &d.action)) ||
         (s = upload(h.get(), t.go, &d.go)) || (s = upload(h.get(), t.rule_len, &d.rule_len)) ||
         (s = upload(h.get(), t.rule_lhs, &d.rule_lhs)) || (s = upload(h.get(), t.resolve, &d.resolve)) ||
-        (s = upload(h.get(), dfa, &d.dfa)) || (s = upload(h.get(), t.dfa_start, &d.dfa_start)) ||
+        (s = upload(h.get(), dfa, &d.dfa)) || (s = upload(h.get(), start, &d.dfa_start)) ||
+        (s = upload(h.get(), rows, &d.dfa_rows)) ||
         (s = upload(h.get(), dfa_mask, &d.dfa_mask)) || (s = upload(h.get(), t.mask_chunks, &d.mchunks)) ||
         (s = upload(h.get(), t.mask_rows, &d.mrows)) ||
-        (s = upload(h.get(), t.vocab_bytes, &d.vocab, 16)) || (s = upload(h.get(), t.vocab_off, &d.vocab_off))) {
+        (s = upload(h.get(), t.vocab_bytes, &d.vocab, 16)) || (s = upload(h.get(), t.vocab_off, &d.vocab_off)) ||
+        (s = upload(h.get(), token_prefixes(t), &d.tok32))) {
         for (int i = 0; i < h->n_blocks; i++) cudaFree(h->blocks[i]);
         return s;
     }
@@ -2127,6 +2207,8 @@ psc_status upload_tables(std::unique_ptr<psc_handle>& h, bool global_tables) {
     d.V = t.V;
     d.W = t.W;
     d.nch = t.nch;
+    d.dfa_sparse = t.dfa_sparse;
+    if (t.dfa_sparse) d.dfa = nullptr;
     d.eos_id = t.eos_id;
     d.n_masks = t.n_masks;
     return PSC_OK;
@@ -2155,6 +2237,7 @@ psc_status psc_compile(const char* grammar, size_t grammar_len, const uint8_t* v
         if (opts->max_mask_bytes > 0) o.max_mask_bytes = opts->max_mask_bytes;
         o.threads = opts->threads;
         o.max_bottom_up_bytes = opts->max_bottom_up_bytes;
+        o.max_dense_classifier_bytes = opts->max_dense_classifier_bytes;
         host_only = opts->host_only != 0;
         global_tables = opts->global_tables != 0;
     }
@@ -2194,6 +2277,8 @@ psc_status psc_info(const psc_handle* h, psc_info_t* out) {
     out->n_masks = t.n_masks;
     out->eos_id = t.eos_id;
     out->classifier_bytes = (int64_t)(t.dfa.size() + t.dfa_start.size() + t.dfa_mask.size()) * 4;
+    if (t.dfa_sparse) out->classifier_bytes = (int64_t)(4 * (int64_t)t.S + 2 * (int64_t)t.dfa_exc_y.size() + t.nq) * 4;
+    out->classifier_sparse = t.dfa_sparse;
     out->mask_bytes = (int64_t)(t.mask_rows.size() + t.mask_chunks.size()) * 4;
     out->states_built = t.n_dfa_states_built;
     out->compile_seconds = t.seconds_total;

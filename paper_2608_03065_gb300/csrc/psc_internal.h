@@ -88,6 +88,8 @@ struct Options {
     int threads = 0;                  // 0 = hardware concurrency
     int64_t max_bottom_up_bytes = 0;  // construction memory of the bottom-up classifier
                                       // (0 = 8 GiB; < 0 = not built; over the limit: not built)
+    int64_t max_dense_classifier_bytes = 0;  // dense classifier table above this: sparse layout
+                                             // (0 = 512 MiB; < 0 = always sparse)
 };
 
 struct Tables {
@@ -102,11 +104,16 @@ struct Tables {
     std::vector<int32_t> action, go, rule_len, rule_lhs;
     std::vector<int16_t> resolve;        // [n_classes][n_lr]: terminal a class stands for, -1 none
     bool contextual = false;
-    // classifier DFA over (lexer state, stack read from the top)
+    // classifier DFA over (lexer state, stack read from the top), dense or sparse
     int S = 0;
-    std::vector<int32_t> dfa;            // [S][n_lr]: next state, or -(mask+1) when absorbing
+    std::vector<int32_t> dfa;            // dense: [S][n_lr]: next state, or -(mask+1) when absorbing
     std::vector<int32_t> dfa_start;      // [nq]: first state after reading q (same encoding)
     std::vector<int32_t> dfa_mask;       // [S]: mask id when the stack ends in this state
+    int dfa_sparse = 0;                  // 1: held as a default target and exceptions per state
+    std::vector<int32_t> dfa_def;        // sparse: [S] default target (same encoding)
+    std::vector<int64_t> dfa_exc_off;    // sparse: [S+1] range of the state's exceptions
+    std::vector<uint16_t> dfa_exc_y;     // sparse: stack symbols whose target is not the default, ascending
+    std::vector<int32_t> dfa_exc_t;      // sparse: their targets
     // masks: row 0 = nothing allowed, row 1 = only the end-of-sequence token.
     // A row is stored as nch = ceil(W/32) ids of 32-word chunks (1024 tokens each);
     // equal chunks are stored once (the table shrinks about tenfold on the C-like
@@ -130,6 +137,18 @@ struct Tables {
     int64_t n_dfa_states_built = 0, n_threads = 0, n_trie_nodes = 0;
     double seconds_lex = 0, seconds_dfa = 0, seconds_min = 0, seconds_total = 0;
 };
+
+// Classifier transition from state s on stack symbol y (either layout).
+inline int32_t dfa_next(const Tables& t, int32_t s, int y) {
+    if (!t.dfa_sparse) return t.dfa[(size_t)s * t.n_lr + y];
+    int64_t lo = t.dfa_exc_off[s], end = t.dfa_exc_off[s + 1], hi = end;
+    while (lo < hi) {
+        int64_t m = (lo + hi) >> 1;
+        if (t.dfa_exc_y[m] < y) lo = m + 1;
+        else hi = m;
+    }
+    return lo < end && t.dfa_exc_y[lo] == y ? t.dfa_exc_t[lo] : t.dfa_def[s];
+}
 
 // Word w of mask row m.
 inline uint32_t mask_word(const Tables& t, int m, int w) {

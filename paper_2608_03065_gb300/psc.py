@@ -40,7 +40,8 @@ class PscError(RuntimeError):
 class Options(ctypes.Structure):
     _fields_ = [("max_states", ctypes.c_int64), ("max_mask_bytes", ctypes.c_int64),
                 ("threads", ctypes.c_int32), ("host_only", ctypes.c_int32),
-                ("global_tables", ctypes.c_int32), ("max_bottom_up_bytes", ctypes.c_int64)]
+                ("global_tables", ctypes.c_int32), ("max_bottom_up_bytes", ctypes.c_int64),
+                ("max_dense_classifier_bytes", ctypes.c_int64)]
 
 
 class InfoT(ctypes.Structure):
@@ -50,7 +51,8 @@ class InfoT(ctypes.Structure):
                 ("classifier_bytes", ctypes.c_int64), ("mask_bytes", ctypes.c_int64),
                 ("states_built", ctypes.c_int64), ("compile_seconds", ctypes.c_double),
                 ("advance_table_bytes", ctypes.c_int64), ("device_timeouts", ctypes.c_int64),
-                ("bottom_up_states", ctypes.c_int64), ("bottom_up_bytes", ctypes.c_int64)]
+                ("bottom_up_states", ctypes.c_int64), ("bottom_up_bytes", ctypes.c_int64),
+                ("classifier_sparse", ctypes.c_int64)]
 
 
 _lib = None
@@ -163,6 +165,7 @@ class Info:
     device_timeouts: int
     bottom_up_states: int
     bottom_up_bytes: int
+    classifier_sparse: int
 
 
 class Handle:
@@ -233,9 +236,11 @@ class States:
 # ------------------------------------------------------------------- the ABI
 def psc_compile(grammar: str, vocab: list[bytes] | tuple, eos_id: int, host_only: bool = False,
                 threads: int = 0, max_states: int = 0, max_mask_bytes: int = 0,
-                global_tables: bool = False, bottom_up: bool = True, max_bottom_up_bytes: int = 0) -> Handle:
+                global_tables: bool = False, bottom_up: bool = True, max_bottom_up_bytes: int = 0,
+                max_dense_classifier_bytes: int = 0) -> Handle:
     """vocab: list of token byte strings, or (blob uint8 array, offsets int64[V+1]).
-    bottom_up=False builds no bottom-up classifier (every stack is walked from the top)."""
+    bottom_up=False builds no bottom-up classifier (every stack is walked from the top);
+    max_dense_classifier_bytes < 0 holds the classifier in the sparse layout."""
     if isinstance(vocab, tuple):
         blob, offs = vocab
         blob = np.ascontiguousarray(blob, dtype=np.uint8)
@@ -248,7 +253,7 @@ def psc_compile(grammar: str, vocab: list[bytes] | tuple, eos_id: int, host_only
         blob = np.zeros(1, dtype=np.uint8)
     V = len(offs) - 1
     opts = Options(max_states, max_mask_bytes, threads, 1 if host_only else 0, 1 if global_tables else 0,
-                   max_bottom_up_bytes if bottom_up else -1)
+                   max_bottom_up_bytes if bottom_up else -1, max_dense_classifier_bytes)
     g = grammar.encode("utf-8")
     out = ctypes.c_void_p()
     _check(load().psc_compile(g, len(g), blob.ctypes.data, offs.ctypes.data, V, eos_id, ctypes.byref(opts),
@@ -261,7 +266,7 @@ def psc_save(h: Handle, path: str):
 
 
 def psc_load(path: str, host_only: bool = False, global_tables: bool = False, bottom_up: bool = True) -> Handle:
-    opts = Options(0, 0, 0, 1 if host_only else 0, 1 if global_tables else 0, 0 if bottom_up else -1)
+    opts = Options(0, 0, 0, 1 if host_only else 0, 1 if global_tables else 0, 0 if bottom_up else -1, 0)
     out = ctypes.c_void_p()
     _check(load().psc_load(os.fsencode(path), ctypes.byref(opts), ctypes.byref(out)))
     h = Handle(out.value, 0)

@@ -1,4 +1,4 @@
-"""Full-size GPU parity on the two large workloads, through the C ABI, against
+"""Full-size GPU parity on the large workloads, through the C ABI, against
 the CPU oracle.
 
 * C-like grammar, 151,936 tokens, 256 rows: four whole decode steps
@@ -8,7 +8,11 @@ the CPU oracle.
 * C-like grammar, 262,144 tokens, 1024 rows, at the prefix states: the masks
   and masked logits of psc_fill_apply and of the decode masking pass, all rows
   over all tokens, and the greedy tokens of all rows.
-* The same workload on the benchmark's exact path: the batch restored from a
+* The Java-sized grammar (1,001 LALR(1) states; classifier held sparse, parser
+  tables too large for shared memory, so the advance reads them from global
+  memory), 4,096 tokens, 64 rows: all rows over all tokens at the prefix states
+  and through six whole decode steps.
+* The C-like 262,144-token workload on the benchmark's exact path: the batch restored from a
   saved copy (psc_state_copy), then 32 steps of psc_decode_step_mask +
   psc_decode_step_advance on fresh logits; the oracle is advanced by the same
   tokens.  Every step: 64 rows (a different 64 each step, so every row is
@@ -52,9 +56,9 @@ class Big:
     """A large workload compiled on the device: the prefix states saved in a
     states object, and the oracle's configurations of the same prefixes."""
 
-    def __init__(self, psc, cfg_id):
+    def __init__(self, psc, cfg_id, **opts):
         self.w = w = configs.load(cfg_id)
-        self.h = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id)
+        self.h = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id, **opts)
         self.snap = psc.psc_state_init(self.h, w.B, CAP)
         tm = torch.from_numpy(w.token_matrix()).cuda()
         for j in range(tm.shape[1]):
@@ -79,9 +83,9 @@ class Big:
 _big = {}
 
 
-def big(psc, cfg_id):
+def big(psc, cfg_id, **opts):
     if cfg_id not in _big:
-        _big[cfg_id] = Big(psc, cfg_id)
+        _big[cfg_id] = Big(psc, cfg_id, **opts)
     return _big[cfg_id]
 
 
@@ -105,6 +109,33 @@ def test_c_like_151936_whole_decode_all_rows_all_tokens(psc):
     stat = torch.empty(B, dtype=torch.int32, device="cuda")
     for step in range(4):
         x, logits = device_logits(B, V, 4000 + step, w.spec.sigma)
+        bm = torch.zeros(B, b.h.W, dtype=torch.int32, device="cuda")
+        psc.psc_decode_step(b.h, st, x, tok, bm, stat)
+        torch.cuda.synchronize()
+        ref = b.o.masks(ocs, b.voc, threads=THREADS)
+        np.testing.assert_array_equal(bm.cpu().numpy().view(np.uint32), ref, err_msg=f"step {step}")
+        allowed = bits_of(ref, V)
+        np.testing.assert_array_equal(raw_bits(x), reference_masked(logits, allowed), err_msg=f"step {step}")
+        t = tok.cpu().numpy()
+        np.testing.assert_array_equal(t, cpu_greedy(logits, allowed), err_msg=f"step {step}")
+        s = stat.cpu().numpy()
+        for r in range(B):
+            if t[r] >= 0:
+                ost = b.o.advance(ocs[r], None if t[r] == w.eos_id else w.vocab[t[r]])
+                assert s[r] == STATUS[ost], (step, r, s[r], ost)
+
+
+def test_java_sized_grammar_whole_decode_all_rows_all_tokens(psc):
+    b = big(psc, 6, bottom_up=False, **configs.COMPILE_LIMITS[6])
+    w = b.w
+    info = b.h.info()
+    assert info.n_parser_states >= 1000 and info.classifier_sparse == 1 and info.advance_table_bytes == 0
+    B, V = w.B, w.V
+    st, ocs = b.restored(psc)
+    tok = torch.empty(B, dtype=torch.int32, device="cuda")
+    stat = torch.empty(B, dtype=torch.int32, device="cuda")
+    for step in range(6):
+        x, logits = device_logits(B, V, 7000 + step, w.spec.sigma)
         bm = torch.zeros(B, b.h.W, dtype=torch.int32, device="cuda")
         psc.psc_decode_step(b.h, st, x, tok, bm, stat)
         torch.cuda.synchronize()

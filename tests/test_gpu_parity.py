@@ -604,3 +604,53 @@ def test_no_device_wait_gave_up(psc):
     the tests above completed: the process-wide timeout counter is still zero."""
     c = case(psc, 1)
     assert c.h.info().device_timeouts == 0
+
+
+@pytest.mark.parametrize("cfg_id", [1, 2, 3])
+def test_sparse_classifier_layout_on_the_device(psc, cfg_id):
+    """The classifier in the sparse layout (a default target and the exceptions
+    to it per state; a warp reads one row per step) and no bottom-up classifier,
+    so the device walks the sparse rows from the stack top: the masks of every
+    row over every token equal the oracle's; four decode steps give the same
+    masks, tokens, masked logits and statuses as the dense handle; the no-alloc
+    entry point (its own classifier walk) agrees with psc_fill_apply."""
+    w = configs.load(cfg_id)
+    hs = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id, bottom_up=False, max_dense_classifier_bytes=-1)
+    hd = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id, bottom_up=False)
+    assert hs.info().classifier_sparse == 1 and hd.info().classifier_sparse == 0
+    ss, sd = psc.psc_state_init(hs, w.B, 256), psc.psc_state_init(hd, w.B, 256)
+    tm = torch.from_numpy(w.token_matrix()).cuda()
+    for j in range(tm.shape[1]):
+        psc.psc_advance(hs, ss, tm[:, j].contiguous())
+        psc.psc_advance(hd, sd, tm[:, j].contiguous())
+    o = Oracle(w.grammar_text)
+    voc = Vocab.from_list(w.vocab, w.eos_id)
+    ocs = []
+    for ids in w.prefix_ids:
+        oc = o.initial()
+        o.advance_tokens(oc, voc, ids)
+        ocs.append(oc)
+    bm = torch.empty(w.B, hs.W, dtype=torch.int32, device="cuda")
+    psc.psc_fill_mask(hs, ss, bm)
+    np.testing.assert_array_equal(bm.cpu().numpy().view(np.uint32), o.masks(ocs, voc, threads=THREADS))
+    # the no-alloc call classifies with its own walk over the sparse rows
+    d = psc.psc_states_download(ss)
+    logits = w.logits(60).cuda()
+    a, b = logits.clone(), logits.clone()
+    psc.psc_fill_apply(hs, ss, a)
+    psc.psc_fill_apply_noalloc(hs, torch.from_numpy(d["q"]).cuda(), torch.from_numpy(d["depth"]).cuda(),
+                               torch.from_numpy(d["status"]).cuda(), torch.from_numpy(d["stack"].view(np.int16)).cuda(), b)
+    np.testing.assert_array_equal(raw_bits(a), raw_bits(b))
+    ts, td = (torch.empty(w.B, dtype=torch.int32, device="cuda") for _ in range(2))
+    xs_, xd_ = (torch.empty(w.B, dtype=torch.int32, device="cuda") for _ in range(2))
+    for step in range(4):
+        logits = w.logits(61 + step)
+        x1, x2 = logits.cuda(), logits.cuda()
+        b1, b2 = (torch.zeros(w.B, hs.W, dtype=torch.int32, device="cuda") for _ in range(2))
+        psc.psc_decode_step(hs, ss, x1, ts, b1, xs_)
+        psc.psc_decode_step(hd, sd, x2, td, b2, xd_)
+        torch.cuda.synchronize()
+        np.testing.assert_array_equal(b1.cpu().numpy(), b2.cpu().numpy(), err_msg=f"step {step}")
+        np.testing.assert_array_equal(ts.cpu().numpy(), td.cpu().numpy(), err_msg=f"step {step}")
+        np.testing.assert_array_equal(xs_.cpu().numpy(), xd_.cpu().numpy(), err_msg=f"step {step}")
+        np.testing.assert_array_equal(raw_bits(x1), raw_bits(x2))

@@ -541,3 +541,34 @@ def test_device_calls_refuse_host_only_handle(psc):
     with pytest.raises(psc.PscError) as e:
         psc.psc_state_init(h, 4, 16, stream=0)
     assert e.value.code == 1
+
+
+@pytest.mark.parametrize("cfg_id", [1, 2, 3])
+def test_sparse_classifier_layout_classifies_like_the_dense_one(psc, cfg_id, tmp_path):
+    """The classifier held sparse (a default target and the exceptions to it per
+    state) classifies every configuration the workload prefixes pass through
+    exactly as the dense table does, its bottom-up form agrees, and a saved and
+    loaded sparse handle stays sparse and agrees too."""
+    w = configs.load(cfg_id, batch=8)
+    hd = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id, host_only=True)
+    hs = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id, host_only=True, max_dense_classifier_bytes=-1)
+    assert hd.info().classifier_sparse == 0 and hs.info().classifier_sparse == 1
+    assert hs.info().n_classifier_states == hd.info().n_classifier_states
+    assert hs.info().classifier_bytes < hd.info().classifier_bytes
+    path = str(tmp_path / "sparse.psc")
+    psc.psc_save(hs, path)
+    hl = psc.psc_load(path, host_only=True)
+    assert hl.info().classifier_sparse == 1
+    n = 0
+    for ids in w.prefix_ids:
+        c = hd.host_initial()
+        for v in ids:
+            c = hd.host_advance(c, v)
+            if c["status"] != psc.ROW_OK:
+                break
+            want = hd.host_classify(c["q"], c["stack"])
+            assert hs.host_classify(c["q"], c["stack"]) == want
+            assert hl.host_classify(c["q"], c["stack"]) == want
+            assert hs.host_classify_bottom_up(c["q"], c["stack"]) == want
+            n += 1
+    assert n > 50

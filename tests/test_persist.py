@@ -77,7 +77,21 @@ def test_tables_without_bottom_up_round_trip(psc, tmp_path):
         assert h2.host_classify_bottom_up(c["q"], c["stack"]) == -2
 
 
-def test_compiled_tables_do_not_depend_on_the_thread_count(psc, tmp_path):
+@pytest.fixture()
+def uncompressed(monkeypatch):
+    monkeypatch.setenv("PSC_SAVE_CODEC", "none")
+
+
+def _payload_start(data: bytes) -> int:
+    """Offset of the table payload in an uncompressed format-04 file: magic,
+    codec and reserved words, payload size and block count, then the sizes of
+    every block."""
+    assert data[:8] == b"PSCTAB04" and int.from_bytes(data[8:12], "little") == 0
+    nb = int.from_bytes(data[24:32], "little")
+    return 32 + 16 * nb
+
+
+def test_compiled_tables_do_not_depend_on_the_thread_count(psc, tmp_path, uncompressed):
     """Files compiled with 1 and with 8 host threads are byte-identical except
     for the recorded compile time (and so the checksum): table ids are numbered
     in an order that does not depend on which thread finishes first."""
@@ -89,9 +103,35 @@ def test_compiled_tables_do_not_depend_on_the_thread_count(psc, tmp_path):
         psc.psc_save(h, path)
         data.append(open(path, "rb").read())
     a, b = data
-    t0 = 8 + 15 * 4 + 3 * 8   # magic, 15 int32 and 3 int64 scalars, then the compile time (double)
+    t0 = _payload_start(a) + 15 * 4 + 3 * 8   # 15 int32 and 3 int64 scalars, then the compile time (double)
     assert len(a) == len(b)
     assert a[:t0] == b[:t0] and a[t0 + 8:-8] == b[t0 + 8:-8]
+
+
+def test_saved_files_are_compressed(psc, tmp_path, monkeypatch):
+    """By default the tables are compressed (zstd when the system library loads,
+    else zlib); every codec round-trips to the same tables."""
+    w = configs.load(2, batch=4)
+    h = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id, host_only=True)
+    sizes = {}
+    for codec in ("default", "none", "zlib", "zstd"):
+        if codec == "default":
+            monkeypatch.delenv("PSC_SAVE_CODEC", raising=False)
+        else:
+            monkeypatch.setenv("PSC_SAVE_CODEC", codec)
+        path = str(tmp_path / f"{codec}.psc")
+        psc.psc_save(h, path)
+        data = open(path, "rb").read()
+        sizes[codec] = (len(data), int.from_bytes(data[8:12], "little"))
+        h2 = psc.psc_load(path, host_only=True)
+        assert h2.info().n_classifier_states == h.info().n_classifier_states
+        for ids in w.prefix_ids:
+            c = h.host_initial()
+            for v in ids:
+                c = h.host_advance(c, v)
+            assert h2.host_classify(c["q"], c["stack"]) == h.host_classify(c["q"], c["stack"])
+    assert sizes["none"][1] == 0
+    assert sizes["default"][1] in (1, 2) and sizes["default"][0] * 4 < sizes["none"][0]
 
 
 def _fnv1a64(data: bytes) -> int:
@@ -101,7 +141,7 @@ def _fnv1a64(data: bytes) -> int:
     return h
 
 
-def test_inconsistent_bottom_up_tables_are_refused(psc, tmp_path):
+def test_inconsistent_bottom_up_tables_are_refused(psc, tmp_path, uncompressed):
     """A file whose checksum is right but whose bottom-up classifier names an LR
     state out of range (the last table of the file) fails validation."""
     w = configs.load(1, batch=2)
@@ -109,9 +149,10 @@ def test_inconsistent_bottom_up_tables_are_refused(psc, tmp_path):
     path = str(tmp_path / "a.psc")
     psc.psc_save(h, path)
     data = bytearray(open(path, "rb").read())
-    body = data[:-8]
+    p0 = _payload_start(bytes(data))
+    body = data[p0:-8]
     body[-4:] = (0x7FFF0000).to_bytes(4, "little")      # LR state of the last bottom-up block
-    bad = bytes(body) + _fnv1a64(bytes(body)).to_bytes(8, "little")
+    bad = bytes(data[:p0]) + bytes(body) + _fnv1a64(bytes(body)).to_bytes(8, "little")
     open(path + ".bad", "wb").write(bad)
     with pytest.raises(psc.PscError) as e:
         psc.psc_load(path + ".bad", host_only=True)

@@ -6,6 +6,7 @@
 4. C-like language, V=151,936, B=256, prefixes up to 2048 bytes, bf16 logits ~N(0,2)
 5. C-like language, V=262,144, B=1024, prefixes of 64-4096 bytes biased to deep nesting,
    bf16 logits ~N(0,2), 32 decode steps
+6. (extra) Java-sized language (1,001 LALR(1) states), V=4,096, B=64, prefixes of 64-2048 bytes
 
 N(0,2) is read as variance 2 (sigma = sqrt 2).  The paper's datasets, JSON
 schemas and tokenizers are not available; these stand in for them.
@@ -47,7 +48,13 @@ SPECS = {
     4: WorkloadSpec(4, "c_like_v151936_b256", 256, 151936, "bf16", math.sqrt(2), 1, 2048, 32, 0.7),
     5: WorkloadSpec(5, "c_like_v262144_b1024", 1024, 262144, "bf16", math.sqrt(2), 64, 4096, 32, 0.7,
                     nest_bias=4.0, max_depth=500, decode_steps=32),
+    # not one of the five benchmark configurations: a Java-sized grammar (1,001 LALR(1)
+    # states, 533 productions, contextual lexer) for the construction at real-grammar
+    # scale; its vocabulary is sized so that the construction fits a test run
+    6: WorkloadSpec(6, "java_like_v4096_b64", 64, 4096, "bf16", math.sqrt(2), 64, 2048, 24, 0.7,
+                    max_depth=60),
 }
+COMPILE_LIMITS = {6: {"max_states": 64_000_000}}   # the Java-sized construction builds ~20 M states
 
 
 def grammar_spec(cfg: int) -> grammars.GrammarSpec:
@@ -57,6 +64,8 @@ def grammar_spec(cfg: int) -> grammars.GrammarSpec:
         return grammars.json_grammar()
     if cfg == 3:
         return grammars.schema_json(seed=int(np.random.default_rng([3, 1]).integers(0, 2**31)))
+    if cfg == 6:
+        return grammars.java_like()
     return grammars.c_like()
 
 

@@ -409,3 +409,392 @@ def c_like() -> GrammarSpec:
                ("if_stmt", 0), ("if_stmt", 1), ("if_stmt", 2)}
     return GrammarSpec("c_like", rules, terms, "contextual", _c_sep, weights=weights,
                        nesting=nesting)
+
+
+# ------------------------------------------------------------ Java-sized
+JAVA_KEYWORDS = [
+    "abstract", "assert", "boolean", "break", "byte", "case", "catch", "char", "class", "const", "continue",
+    "default", "do", "double", "else", "enum", "exports", "extends", "final", "finally", "float", "for", "goto",
+    "if", "implements", "import", "instanceof", "int", "interface", "long", "module", "native", "new", "null",
+    "open", "opens", "package", "private", "protected", "provides", "public", "record", "requires", "return",
+    "short", "static", "strictfp", "super", "switch", "synchronized", "this", "throw", "throws", "to",
+    "transient", "transitive", "true", "false", "try", "uses", "var", "void", "volatile", "while", "with",
+    "yield"]
+
+
+def _java_name(rng) -> bytes:
+    while True:
+        r = rng.random()
+        if r < 0.45:
+            w = _word(rng, 1, 8)
+        elif r < 0.75:
+            w = _word(rng, 1, 6) + _word(rng, 1, 1, "ABCDEFGHIJKLMNOPQRSTUVWXYZ") + _word(rng, 1, 5)
+        elif r < 0.9:
+            w = _word(rng, 1, 1, "ABCDEFGHIJKLMNOPQRSTUVWXYZ") + _word(rng, 2, 8)
+        else:
+            w = _word(rng, 1, 4) + "_" + _word(rng, 1, 4, _ALNUM)
+        if w not in JAVA_KEYWORDS:
+            return w.encode()
+
+
+def _java_int(rng) -> bytes:
+    r = rng.random()
+    if r < 0.6:
+        s = _digits(rng, 1, 4)
+    elif r < 0.72:
+        s = "0"
+    elif r < 0.84:
+        s = "0x" + _word(rng, 1, 6, "0123456789abcdefABCDEF")
+    elif r < 0.9:
+        s = "0b" + _word(rng, 1, 8, "01")
+    else:
+        s = _digits(rng, 1, 3) + "_" + _digits(rng, 3, 3)
+    return (s + ("L" if rng.random() < 0.1 else "")).encode()
+
+
+def _java_float(rng) -> bytes:
+    r = rng.random()
+    if r < 0.6:
+        s = _digits(rng, 1, 3) + "." + _digits(rng, 1, 3)
+    elif r < 0.8:
+        s = _digits(rng, 1, 2) + "e" + "+-"[int(rng.integers(0, 2))] + _digits(rng, 1, 2)
+    else:
+        s = _digits(rng, 1, 3)
+    return (s + ("fFdD"[int(rng.integers(0, 4))] if r >= 0.8 or rng.random() < 0.3 else "")).encode()
+
+
+def _java_text_block(rng) -> bytes:
+    lines = [_word(rng, 0, 10, _LOWER + " .,") for _ in range(int(rng.integers(1, 4)))]
+    return ('"""\n' + "\n".join(lines) + '"""').encode()
+
+
+def java_like() -> GrammarSpec:
+    """Synthetic Java-sized language (stands in for the paper's Java grammar): package
+    and import declarations, a module declaration, classes, interfaces, enums,
+    records and annotation types with generics, modifiers and annotations; fields,
+    methods, constructors, initializers; every Java statement form (if/else in the
+    no-short-if form, loops, enhanced for, labelled statements, switch with groups and
+    arrow rules, try/catch/finally with resources, synchronized, assert, throw);
+    expressions over 15 precedence levels with casts, instanceof patterns, class
+    literals, array creation and access, method invocation and object creation.
+    Written LALR(1): generic type arguments only where no expression can start,
+    casts as in Java's own LALR grammar (a parenthesized expression followed by a
+    unary expression), declarations and expressions sharing the qualified-name
+    prefix.  Keywords are literals that also match NAME (contextual lexer); nested
+    generic closers need a space (the lexer reads ">>" as one lexeme)."""
+    L = lambda s: _lit(s)  # noqa: E731
+    prim = ["byte", "short", "char", "int", "long", "float", "double", "boolean"]
+    mods = ["public", "protected", "private", "static", "abstract", "final", "native", "synchronized",
+            "transient", "volatile", "strictfp", "default", "sealed", "non-sealed"]
+    assign_ops = ["=", "+=", "-=", "*=", "/=", "%=", "&=", "|=", "^=", "<<=", ">>=", ">>>="]
+
+    def if_forms(s, body):   # if statements whose last sub-statement is `body`
+        return [[L("if"), L("("), "expr", L(")"), "stmt_nsi", L("else"), body]]
+
+    rules = {
+        "start": [["compilation_unit"]],
+        "compilation_unit": [["type_decls"], ["package_decl", "type_decls"], ["import_decls", "type_decls"],
+                             ["package_decl", "import_decls", "type_decls"], ["module_decl"],
+                             ["import_decls", "module_decl"]],
+        "package_decl": [[L("package"), "qualified_name", L(";")]],
+        "import_decls": [["import_decl"], ["import_decls", "import_decl"]],
+        "import_decl": [[L("import"), "qualified_name", L(";")],
+                        [L("import"), "qualified_name", L("."), L("*"), L(";")],
+                        [L("import"), L("static"), "qualified_name", L(";")],
+                        [L("import"), L("static"), "qualified_name", L("."), L("*"), L(";")]],
+        "qualified_name": [["NAME"], ["qualified_name", L("."), "NAME"]],
+        # modules
+        "module_decl": [[L("module"), "qualified_name", L("{"), L("}")],
+                        [L("module"), "qualified_name", L("{"), "module_directives", L("}")],
+                        [L("open"), L("module"), "qualified_name", L("{"), "module_directives", L("}")]],
+        "module_directives": [["module_directive"], ["module_directives", "module_directive"]],
+        "module_directive": [[L("requires"), "qualified_name", L(";")],
+                             [L("requires"), L("transitive"), "qualified_name", L(";")],
+                             [L("requires"), L("static"), "qualified_name", L(";")],
+                             [L("exports"), "qualified_name", L(";")],
+                             [L("exports"), "qualified_name", L("to"), "name_list", L(";")],
+                             [L("opens"), "qualified_name", L(";")],
+                             [L("opens"), "qualified_name", L("to"), "name_list", L(";")],
+                             [L("uses"), "qualified_name", L(";")],
+                             [L("provides"), "qualified_name", L("with"), "name_list", L(";")]],
+        "name_list": [["qualified_name"], ["name_list", L(","), "qualified_name"]],
+        # type declarations
+        "type_decls": [["type_decl"], ["type_decls", "type_decl"]],
+        "type_decl": [["class_decl"], ["interface_decl"], ["enum_decl"], ["record_decl"],
+                      ["annotation_type_decl"], [L(";")]],
+        "modifiers": [["modifier"], ["modifiers", "modifier"]],
+        "modifier": [[L(m)] for m in mods] + [["annotation"]],
+        "annotation": [[L("@"), "qualified_name"], [L("@"), "qualified_name", L("("), L(")")],
+                       [L("@"), "qualified_name", L("("), "element_value", L(")")],
+                       [L("@"), "qualified_name", L("("), "element_value_pairs", L(")")]],
+        "element_value_pairs": [["element_value_pair"], ["element_value_pairs", L(","), "element_value_pair"]],
+        "element_value_pair": [["NAME", L("="), "element_value"]],
+        "element_value": [["cond_expr"], ["annotation"], [L("{"), L("}")], [L("{"), "element_values", L("}")],
+                          [L("{"), "element_values", L(","), L("}")]],
+        "element_values": [["element_value"], ["element_values", L(","), "element_value"]],
+        "class_decl": [["class_head", "class_body"]],
+        "class_head": [["class_name"], ["class_name", "superclass"], ["class_name", "interfaces"],
+                       ["class_name", "superclass", "interfaces"], ["class_name", "permits"],
+                       ["class_name", "superclass", "permits"], ["class_name", "superclass", "interfaces", "permits"]],
+        "permits": [[L("permits"), "class_type_list"]],
+        "class_name": [[L("class"), "NAME"], ["modifiers", L("class"), "NAME"],
+                       [L("class"), "NAME", "type_params"], ["modifiers", L("class"), "NAME", "type_params"]],
+        "superclass": [[L("extends"), "class_type"]],
+        "interfaces": [[L("implements"), "class_type_list"]],
+        "class_type_list": [["class_type"], ["class_type_list", L(","), "class_type"]],
+        "type_params": [[L("<"), "type_param_list", L(">")]],
+        "type_param_list": [["type_param"], ["type_param_list", L(","), "type_param"]],
+        "type_param": [["NAME"], ["NAME", L("extends"), "type_bound"]],
+        "type_bound": [["class_type"], ["type_bound", L("&"), "class_type"]],
+        "class_type": [["NAME"], ["NAME", "type_args"], ["class_type", L("."), "NAME"],
+                       ["class_type", L("."), "NAME", "type_args"]],
+        "type_args": [[L("<"), "type_arg_list", L(">")], [L("<"), L(">")]],
+        "type_arg_list": [["type_arg"], ["type_arg_list", L(","), "type_arg"]],
+        "type_arg": [["ref_type"], [L("?")], [L("?"), L("extends"), "ref_type"], [L("?"), L("super"), "ref_type"]],
+        "ref_type": [["class_type"], ["class_type", "dims"], ["prim_type", "dims"]],
+        "type": [["prim_type"], ["prim_type", "dims"], ["class_type"], ["class_type", "dims"]],
+        "prim_type": [[L(p)] for p in prim],
+        "dims": [[L("["), L("]")], ["dims", L("["), L("]")]],
+        "class_body": [[L("{"), L("}")], [L("{"), "class_body_decls", L("}")]],
+        "class_body_decls": [["class_body_decl"], ["class_body_decls", "class_body_decl"]],
+        "class_body_decl": [["field_decl"], ["method_decl"], ["constructor_decl"], ["block"],
+                            [L("static"), "block"], ["class_decl"], ["interface_decl"], ["enum_decl"],
+                            ["record_decl"], ["annotation_type_decl"], ["compact_constructor"], [L(";")]],
+        "field_decl": [["type", "var_declarators", L(";")], ["modifiers", "type", "var_declarators", L(";")]],
+        "var_declarators": [["var_declarator"], ["var_declarators", L(","), "var_declarator"]],
+        "var_declarator": [["NAME"], ["NAME", L("="), "var_init"], ["NAME", "dims"],
+                           ["NAME", "dims", L("="), "var_init"]],
+        "var_init": [["expr"], ["array_init"], ["switch_expr"]],
+        "array_init": [[L("{"), L("}")], [L("{"), "var_inits", L("}")], [L("{"), "var_inits", L(","), L("}")]],
+        "var_inits": [["var_init"], ["var_inits", L(","), "var_init"]],
+        "method_decl": [["method_header", "method_body"]],
+        "method_header": [["method_sig"], ["method_sig", "throws"]],
+        "method_sig": [["type", "method_declarator"], [L("void"), "method_declarator"],
+                       ["modifiers", "type", "method_declarator"], ["modifiers", L("void"), "method_declarator"],
+                       ["type_params", "type", "method_declarator"],
+                       ["type_params", L("void"), "method_declarator"],
+                       ["modifiers", "type_params", "type", "method_declarator"],
+                       ["modifiers", "type_params", L("void"), "method_declarator"]],
+        "method_declarator": [["NAME", L("("), L(")")], ["NAME", L("("), "formal_params", L(")")]],
+        "formal_params": [["formal_param"], ["formal_params", L(","), "formal_param"]],
+        "formal_param": [["type", "NAME"], ["var_modifiers", "type", "NAME"], ["type", L("..."), "NAME"],
+                         ["var_modifiers", "type", L("..."), "NAME"]],
+        "var_modifiers": [["var_modifier"], ["var_modifiers", "var_modifier"]],
+        "var_modifier": [[L("final")], ["annotation"]],
+        "throws": [[L("throws"), "class_type_list"]],
+        "method_body": [["block"], [L(";")]],
+        "constructor_decl": [["constructor_sig", "block"], ["constructor_sig", "throws", "block"]],
+        "constructor_sig": [["NAME", L("("), L(")")], ["NAME", L("("), "formal_params", L(")")],
+                            ["modifiers", "NAME", L("("), L(")")],
+                            ["modifiers", "NAME", L("("), "formal_params", L(")")],
+                            ["type_params", "NAME", L("("), L(")")],
+                            ["type_params", "NAME", L("("), "formal_params", L(")")],
+                            ["modifiers", "type_params", "NAME", L("("), "formal_params", L(")")]],
+        # compact constructor of a record
+        "compact_constructor": [["NAME", "block"], ["modifiers", "NAME", "block"]],
+        "interface_decl": [["interface_name", "interface_body"],
+                           ["interface_name", L("extends"), "class_type_list", "interface_body"]],
+        "interface_name": [[L("interface"), "NAME"], ["modifiers", L("interface"), "NAME"],
+                           [L("interface"), "NAME", "type_params"],
+                           ["modifiers", L("interface"), "NAME", "type_params"]],
+        "interface_body": [[L("{"), L("}")], [L("{"), "interface_members", L("}")]],
+        "interface_members": [["interface_member"], ["interface_members", "interface_member"]],
+        "interface_member": [["field_decl"], ["method_decl"], ["class_decl"], ["interface_decl"],
+                             ["enum_decl"], ["record_decl"], ["annotation_type_decl"], [L(";")]],
+        "enum_decl": [["enum_name", "enum_body"], ["enum_name", "interfaces", "enum_body"]],
+        "enum_name": [[L("enum"), "NAME"], ["modifiers", L("enum"), "NAME"]],
+        "enum_body": [[L("{"), L("}")], [L("{"), "enum_constants", L("}")],
+                      [L("{"), "enum_constants", L(","), L("}")],
+                      [L("{"), "enum_constants", L(";"), "class_body_decls", L("}")],
+                      [L("{"), "enum_constants", L(","), L(";"), "class_body_decls", L("}")],
+                      [L("{"), L(";"), "class_body_decls", L("}")]],
+        "enum_constants": [["enum_constant"], ["enum_constants", L(","), "enum_constant"]],
+        "enum_constant": [["NAME"], ["NAME", "arguments"], ["NAME", "class_body"], ["NAME", "arguments", "class_body"]],
+        "record_decl": [["record_head", "class_body"], ["record_head", "interfaces", "class_body"]],
+        "record_head": [["record_name", L("("), L(")")], ["record_name", L("("), "record_components", L(")")]],
+        "record_name": [[L("record"), "NAME"], ["modifiers", L("record"), "NAME"],
+                        [L("record"), "NAME", "type_params"]],
+        "record_components": [["record_component"], ["record_components", L(","), "record_component"]],
+        "record_component": [["type", "NAME"], ["annotation", "type", "NAME"]],
+        "annotation_type_decl": [[L("@"), L("interface"), "NAME", "annotation_type_body"],
+                                 ["modifiers", L("@"), L("interface"), "NAME", "annotation_type_body"]],
+        "annotation_type_body": [[L("{"), L("}")], [L("{"), "annotation_type_elements", L("}")]],
+        "annotation_type_elements": [["annotation_type_element"],
+                                     ["annotation_type_elements", "annotation_type_element"]],
+        "annotation_type_element": [["type", "NAME", L("("), L(")"), L(";")],
+                                    ["type", "NAME", L("("), L(")"), L("default"), "element_value", L(";")],
+                                    ["modifiers", "type", "NAME", L("("), L(")"), L(";")],
+                                    ["modifiers", "type", "NAME", L("("), L(")"), L("default"), "element_value",
+                                     L(";")],
+                                    ["field_decl_const"], ["class_decl"], ["enum_decl"], [L(";")]],
+        "field_decl_const": [["type", "NAME", L("="), "var_init", L(";")],
+                             ["modifiers", "type", "NAME", L("="), "var_init", L(";")]],
+        # blocks and statements
+        "block": [[L("{"), L("}")], [L("{"), "block_stmts", L("}")]],
+        "block_stmts": [["block_stmt"], ["block_stmts", "block_stmt"]],
+        "block_stmt": [["local_var_decl", L(";")], ["stmt"], ["local_type_decl"],
+                       [L("this"), "arguments", L(";")], [L("super"), "arguments", L(";")]],
+        # local classes, records, interfaces and enums (modifiers: final, abstract, annotations)
+        "local_type_decl": [["local_class_name", "class_body"], ["local_class_name", "superclass", "class_body"],
+                            ["local_class_name", "interfaces", "class_body"],
+                            ["local_class_name", "superclass", "interfaces", "class_body"],
+                            [L("record"), "NAME", L("("), "record_components", L(")"), "class_body"],
+                            [L("record"), "NAME", L("("), L(")"), "class_body"],
+                            [L("interface"), "NAME", "interface_body"],
+                            [L("enum"), "NAME", "enum_body"]],
+        "local_class_name": [[L("class"), "NAME"], ["local_class_mods", L("class"), "NAME"],
+                             [L("class"), "NAME", "type_params"]],
+        "local_class_mods": [["var_modifiers"], [L("abstract")], ["var_modifiers", L("abstract")]],
+        "local_var_decl": [["local_type", "var_declarators"], ["var_modifiers", "local_type", "var_declarators"],
+                           [L("var"), "NAME", L("="), "expr"], ["var_modifiers", L("var"), "NAME", L("="), "expr"]],
+        "local_type": [["prim_type"], ["prim_type", "dims"], ["name"], ["name", "dims"]],
+        "name": [["NAME"], ["name", L("."), "NAME"]],
+        "stmt": [["stmt_wts"], ["labeled_stmt"], [L("if"), L("("), "expr", L(")"), "stmt"],
+                 ["if_else_stmt"], ["while_stmt"], ["for_stmt"], ["foreach_stmt"]],
+        "stmt_nsi": [["stmt_wts"], ["labeled_stmt_nsi"], ["if_else_stmt_nsi"], ["while_stmt_nsi"],
+                     ["for_stmt_nsi"], ["foreach_stmt_nsi"]],
+        "if_else_stmt": if_forms("stmt", "stmt"),
+        "if_else_stmt_nsi": if_forms("stmt_nsi", "stmt_nsi"),
+        "labeled_stmt": [["NAME", L(":"), "stmt"]],
+        "labeled_stmt_nsi": [["NAME", L(":"), "stmt_nsi"]],
+        "while_stmt": [[L("while"), L("("), "expr", L(")"), "stmt"]],
+        "while_stmt_nsi": [[L("while"), L("("), "expr", L(")"), "stmt_nsi"]],
+        "for_stmt": [["for_head", "stmt"]],
+        "for_stmt_nsi": [["for_head", "stmt_nsi"]],
+        "for_head": [[L("for"), L("("), "for_init", L(";"), "opt_expr", L(";"), "for_update", L(")")]],
+        "for_init": [[], ["stmt_expr_list"], ["local_var_decl"]],
+        "for_update": [[], ["stmt_expr_list"]],
+        "opt_expr": [[], ["expr"]],
+        "stmt_expr_list": [["expr"], ["stmt_expr_list", L(","), "expr"]],
+        "foreach_stmt": [["foreach_head", "stmt"]],
+        "foreach_stmt_nsi": [["foreach_head", "stmt_nsi"]],
+        "foreach_head": [[L("for"), L("("), "local_type", "NAME", L(":"), "expr", L(")")],
+                         [L("for"), L("("), "var_modifiers", "local_type", "NAME", L(":"), "expr", L(")")],
+                         [L("for"), L("("), L("var"), "NAME", L(":"), "expr", L(")")]],
+        "stmt_wts": [["block"], [L(";")], ["expr", L(";")], ["switch_stmt"],
+                     [L("return"), "switch_expr", L(";")], [L("yield"), "switch_expr", L(";")],
+                     [L("do"), "stmt", L("while"), L("("), "expr", L(")"), L(";")],
+                     [L("break"), L(";")], [L("break"), "NAME", L(";")], [L("continue"), L(";")],
+                     [L("continue"), "NAME", L(";")], [L("return"), L(";")], [L("return"), "expr", L(";")],
+                     [L("throw"), "expr", L(";")], [L("yield"), "expr", L(";")],
+                     [L("synchronized"), L("("), "expr", L(")"), "block"], ["try_stmt"],
+                     [L("assert"), "expr", L(";")], [L("assert"), "expr", L(":"), "expr", L(";")]],
+        "switch_stmt": [[L("switch"), L("("), "expr", L(")"), "switch_block"]],
+        "switch_block": [[L("{"), L("}")], [L("{"), "switch_groups", L("}")],
+                         [L("{"), "switch_groups", "switch_labels", L("}")], [L("{"), "switch_labels", L("}")],
+                         [L("{"), "switch_rules", L("}")]],
+        "switch_groups": [["switch_group"], ["switch_groups", "switch_group"]],
+        "switch_group": [["switch_labels", "block_stmts"]],
+        "switch_labels": [["switch_label"], ["switch_labels", "switch_label"]],
+        "switch_label": [[L("case"), "case_consts", L(":")], [L("default"), L(":")],
+                         [L("case"), "pattern", L(":")], [L("case"), "pattern", L("when"), "cond_expr", L(":")]],
+        "pattern": [["local_type", "NAME"], [L("final"), "local_type", "NAME"]],
+        "case_consts": [["cond_expr"], ["case_consts", L(","), "cond_expr"]],
+        "switch_rules": [["switch_rule"], ["switch_rules", "switch_rule"]],
+        "switch_rule": [["rule_label", "expr", L(";")], ["rule_label", "block"],
+                        ["rule_label", L("throw"), "expr", L(";")]],
+        "rule_label": [[L("case"), "case_consts", L("->")], [L("default"), L("->")],
+                       [L("case"), "pattern", L("->")], [L("case"), "pattern", L("when"), "cond_expr", L("->")]],
+        "try_stmt": [[L("try"), "block", "catches"], [L("try"), "block", "finally"],
+                     [L("try"), "block", "catches", "finally"], [L("try"), "resource_spec", "block"],
+                     [L("try"), "resource_spec", "block", "catches"], [L("try"), "resource_spec", "block", "finally"],
+                     [L("try"), "resource_spec", "block", "catches", "finally"]],
+        "catches": [["catch_clause"], ["catches", "catch_clause"]],
+        "catch_clause": [[L("catch"), L("("), "catch_type", "NAME", L(")"), "block"],
+                         [L("catch"), L("("), L("final"), "catch_type", "NAME", L(")"), "block"]],
+        "catch_type": [["name"], ["catch_type", L("|"), "name"]],
+        "finally": [[L("finally"), "block"]],
+        "resource_spec": [[L("("), "resources", L(")")], [L("("), "resources", L(";"), L(")")]],
+        "resources": [["resource"], ["resources", L(";"), "resource"]],
+        "resource": [["local_type", "NAME", L("="), "expr"], [L("var"), "NAME", L("="), "expr"], ["name"],
+                     ["var_modifiers", "local_type", "NAME", L("="), "expr"]],
+        # expressions
+        "expr": [["assign_expr"], ["lambda"]],
+        "assign_expr": [["cond_expr"], ["lhs", "assign_op", "assign_expr"], ["lhs", "assign_op", "switch_expr"],
+                        ["lhs", "assign_op", "lambda"]],
+        # lambdas: one untyped parameter, or typed parameters in parentheses (an untyped
+        # parenthesized list would need more than one token of lookahead after ")")
+        "lambda": [["NAME", L("->"), "lambda_body"], [L("("), L(")"), L("->"), "lambda_body"],
+                   [L("("), "lambda_params", L(")"), L("->"), "lambda_body"]],
+        "lambda_params": [["lambda_param"], ["lambda_params", L(","), "lambda_param"]],
+        "lambda_param": [["local_type", "NAME"], [L("final"), "local_type", "NAME"], [L("var"), "NAME"]],
+        "lambda_body": [["expr"], ["block"]],
+        # switch expressions where no statement can start (initializers, right-hand sides,
+        # arguments, return and yield)
+        "switch_expr": [[L("switch"), L("("), "expr", L(")"), L("{"), "switch_rules", L("}")]],
+        "lhs": [["name"], ["field_access"], ["array_access"]],
+        "assign_op": [[L(o)] for o in assign_ops],
+        "cond_expr": [["cond_or"], ["cond_or", L("?"), "expr", L(":"), "cond_expr"]],
+        "cond_or": [["cond_and"], ["cond_or", L("||"), "cond_and"]],
+        "cond_and": [["incl_or"], ["cond_and", L("&&"), "incl_or"]],
+        "incl_or": [["excl_or"], ["incl_or", L("|"), "excl_or"]],
+        "excl_or": [["and_expr"], ["excl_or", L("^"), "and_expr"]],
+        "and_expr": [["eq_expr"], ["and_expr", L("&"), "eq_expr"]],
+        "eq_expr": [["rel_expr"], ["eq_expr", L("=="), "rel_expr"], ["eq_expr", L("!="), "rel_expr"]],
+        "rel_expr": [["shift_expr"], ["rel_expr", L("<"), "shift_expr"], ["rel_expr", L(">"), "shift_expr"],
+                     ["rel_expr", L("<="), "shift_expr"], ["rel_expr", L(">="), "shift_expr"],
+                     ["rel_expr", L("instanceof"), "local_type"],
+                     ["rel_expr", L("instanceof"), "local_type", "NAME"]],
+        "shift_expr": [["add_expr"], ["shift_expr", L("<<"), "add_expr"], ["shift_expr", L(">>"), "add_expr"],
+                       ["shift_expr", L(">>>"), "add_expr"]],
+        "add_expr": [["mul_expr"], ["add_expr", L("+"), "mul_expr"], ["add_expr", L("-"), "mul_expr"]],
+        "mul_expr": [["unary"], ["mul_expr", L("*"), "unary"], ["mul_expr", L("/"), "unary"],
+                     ["mul_expr", L("%"), "unary"]],
+        "unary": [[L("++"), "unary"], [L("--"), "unary"], [L("+"), "unary"], [L("-"), "unary"], ["unary_nnpm"]],
+        "unary_nnpm": [["postfix"], [L("~"), "unary"], [L("!"), "unary"], ["cast"]],
+        "cast": [[L("("), "prim_type", L(")"), "unary"], [L("("), "prim_type", "dims", L(")"), "unary"],
+                 [L("("), "expr", L(")"), "unary_nnpm"], [L("("), "name", "dims", L(")"), "unary_nnpm"]],
+        "postfix": [["primary"], ["name"], ["postfix", L("++")], ["postfix", L("--")]],
+        "primary": [["primary_nna"], ["array_creation"]],
+        "primary_nna": [["literal"], [L("this")], ["name", L("."), L("this")], [L("("), "expr", L(")")],
+                        ["instance_creation"], ["field_access"], ["method_call"], ["array_access"],
+                        ["name", L("."), L("class")], ["prim_type", L("."), L("class")],
+                        [L("void"), L("."), L("class")], ["name", "dims", L("."), L("class")],
+                        ["prim_type", "dims", L("."), L("class")], ["method_ref"]],
+        "literal": [["INT"], ["FLOAT"], ["STRING"], ["TEXT_BLOCK"], ["CHARLIT"], [L("true")], [L("false")],
+                    [L("null")]],
+        "field_access": [["primary", L("."), "NAME"], [L("super"), L("."), "NAME"],
+                         ["name", L("."), L("super"), L("."), "NAME"]],
+        "method_call": [["name", "arguments"], ["primary", L("."), "NAME", "arguments"],
+                        [L("super"), L("."), "NAME", "arguments"],
+                        ["name", L("."), "type_args", "NAME", "arguments"],
+                        ["primary", L("."), "type_args", "NAME", "arguments"],
+                        [L("super"), L("."), "type_args", "NAME", "arguments"]],
+        "method_ref": [["name", L("::"), "NAME"], ["primary", L("::"), "NAME"], [L("super"), L("::"), "NAME"],
+                       ["name", L("::"), L("new")], ["prim_type", "dims", L("::"), L("new")]],
+        "arguments": [[L("("), L(")")], [L("("), "arg_list", L(")")]],
+        "arg_list": [["arg"], ["arg_list", L(","), "arg"]],
+        "arg": [["expr"], ["switch_expr"]],
+        "array_access": [["name", L("["), "expr", L("]")], ["primary_nna", L("["), "expr", L("]")]],
+        "instance_creation": [[L("new"), "class_type", "arguments"],
+                              [L("new"), "class_type", "arguments", "class_body"],
+                              ["primary", L("."), L("new"), "NAME", "arguments"],
+                              ["primary", L("."), L("new"), "NAME", "type_args", "arguments"],
+                              ["primary", L("."), L("new"), "NAME", "arguments", "class_body"],
+                              ["name", L("."), L("new"), "NAME", "arguments"]],
+        "array_creation": [[L("new"), "prim_type", "dim_exprs"], [L("new"), "prim_type", "dim_exprs", "dims"],
+                           [L("new"), "class_type", "dim_exprs"], [L("new"), "class_type", "dim_exprs", "dims"],
+                           [L("new"), "prim_type", "dims", "array_init"],
+                           [L("new"), "class_type", "dims", "array_init"]],
+        "dim_exprs": [["dim_expr"], ["dim_exprs", "dim_expr"]],
+        "dim_expr": [[L("["), "expr", L("]")]],
+    }
+    terms = {
+        "NAME": TermSpec("/[A-Za-z_$][A-Za-z0-9_$]*/", _java_name),
+        "INT": TermSpec("/(0|[1-9][0-9_]*)[lL]?|0[xX][0-9a-fA-F_]+[lL]?|0[bB][01_]+[lL]?/", _java_int),
+        "FLOAT": TermSpec("/[0-9]+\\.[0-9]+([eE][+-]?[0-9]+)?[fFdD]?|[0-9]+[eE][+-]?[0-9]+[fFdD]?|[0-9]+[fFdD]/",
+                          _java_float),
+        "STRING": TermSpec('/"([^"\\\\\\n]|\\\\.)*"/', _c_string),
+        # a text block: three quotes, a line break, then text without three quotes in a row
+        "TEXT_BLOCK": TermSpec('/"""[ \\t]*\\n([^"\\\\]|\\\\.|"[^"\\\\]|""[^"\\\\])*"""/', _java_text_block),
+        "CHARLIT": TermSpec("/'([^'\\\\\\n]|\\\\.)'/", _c_char),
+        "LINE_COMMENT": TermSpec("/\\/\\/[^\\n]*/", lambda r: b"// x", ignored=True),
+        "BLOCK_COMMENT": TermSpec("/\\/\\*([^*]|\\*+[^*\\/])*\\*+\\//", lambda r: b"/* x */", ignored=True),
+        "WS": TermSpec("/[ \\t\\r\\n]+/", lambda r: b" ", ignored=True),
+    }
+    weights = {("type_decls", 1): 1.5, ("class_body_decls", 1): 4.0, ("class_body_decl", 1): 3.0,
+               ("class_body_decl", 0): 2.0, ("block_stmts", 1): 3.0, ("block_stmt", 1): 1.5,
+               ("stmt_wts", 2): 3.0, ("arg_list", 1): 1.2, ("type_decl", 0): 4.0}
+    nesting = {("stmt", 2), ("if_else_stmt", 0), ("stmt_wts", 0), ("while_stmt", 0), ("for_stmt", 0),
+               ("primary_nna", 3), ("class_body_decl", 1)}
+    return GrammarSpec("java_like", rules, terms, "contextual", _c_sep, weights=weights, nesting=nesting)
