@@ -491,6 +491,133 @@ def run_sweep(args):
                       "points": pts}))
 
 
+# ------------------------------------------------------------- compile mode
+def compile_one(cfg: int, vocab: int | None):
+    """(child process) Compile one workload's tables on the host and print their
+    sizes, the compile time and this process's peak RSS (nothing else runs in it)."""
+    import resource
+    import tempfile
+    from paper_2608_03065_gb300 import build, psc
+    from workloads import configs, sample
+    build.build()
+    spec = configs.SPECS[cfg]
+    g = configs.grammar_spec(cfg)
+    V = vocab or spec.V
+    toks = sample.build_vocab(g, sample.VocabSpec(V, spec.vocab_max_len, spec.frac_grammar), [cfg, 2])
+    opts = dict(configs.COMPILE_LIMITS.get(cfg, {}))
+    t0 = time.time()
+    h = psc.psc_compile(g.text(), toks, len(toks) - 1, host_only=True, **opts)
+    secs = time.time() - t0
+    i = h.info()
+    out = {"workload": spec.name if vocab is None else f"{spec.name.split('_v')[0]}_v{V}", "vocab": V,
+           "compile_s": round(secs, 2), "threads": os.cpu_count(),
+           "lalr_states": i.n_parser_states, "lexer_states": i.n_lexer_states,
+           "states_built": i.states_built, "classifier_states": i.n_classifier_states,
+           "classifier_layout": "sparse" if i.classifier_sparse else "dense",
+           "classifier_bytes": i.classifier_bytes,
+           "dense_classifier_bytes": i.n_classifier_states * i.n_parser_states * 4,
+           "masks": i.n_masks, "mask_bytes": i.mask_bytes, "bottom_up_states": i.bottom_up_states,
+           "bottom_up_bytes": i.bottom_up_bytes}
+    with tempfile.TemporaryDirectory() as d:
+        for codec in ("default", "none"):
+            if codec == "none":
+                os.environ["PSC_SAVE_CODEC"] = "none"
+            path = os.path.join(d, f"{codec}.psc")
+            t0 = time.time()
+            psc.psc_save(h, path)
+            with open(path, "rb") as f:
+                head = f.read(12)
+            key = "file_bytes" if codec == "default" else "file_bytes_uncompressed"
+            out[key] = os.path.getsize(path)
+            if codec == "default":
+                out["codec"] = {0: "none", 1: "zstd", 2: "zlib"}[int.from_bytes(head[8:12], "little")]
+                out["save_s"] = round(time.time() - t0, 2)
+                t0 = time.time()
+                psc.psc_load(path, host_only=True)
+                out["load_s"] = round(time.time() - t0, 2)
+    out["peak_rss_gb"] = round(resource.getrusage(resource.RUSAGE_SELF).ru_maxrss / 2**20, 2)
+    print(json.dumps(out))
+
+
+def graph_step_us(psc, h, w, B, n=16, cap=256):
+    """Device time of one decode step at batch B on the workload's prefix states:
+    a CUDA graph of n steps (psc_decode_step on n logits buffers), replayed."""
+    import torch
+    dev = torch.device("cuda", 0)
+    tm = torch.from_numpy(w.token_matrix()).to(dev)
+    snap = psc.psc_state_init(h, B, cap)
+    for j in range(tm.shape[1]):
+        psc.psc_advance(h, snap, tm[:B, j].contiguous())
+    st = psc.psc_state_init(h, B, cap)
+    gen = torch.Generator(device=dev).manual_seed(B)
+    xs = [(torch.randn(B, w.V, generator=gen, device=dev) * w.spec.sigma).to(torch.bfloat16) for _ in range(n)]
+    toks = [torch.empty(B, dtype=torch.int32, device=dev) for _ in range(n)]
+    psc.psc_state_copy(st, snap)
+    psc.psc_decode_step(h, st, xs[0].clone(), toks[0])
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        cs = torch.cuda.current_stream()
+        psc.psc_state_copy(st, snap, stream=cs)
+        for i in range(n):
+            psc.psc_decode_step(h, st, xs[i], toks[i], stream=cs)
+    reps = []
+    for r in range(6):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        g.replay()
+        b.record()
+        torch.cuda.synchronize()
+        if r >= 2:
+            reps.append(a.elapsed_time(b) * 1000.0 / n)
+    return round(sorted(reps)[len(reps) // 2], 2)
+
+
+def run_compile(args):
+    """Construction at scale (the paper's preprocessing cost and runtime memory,
+    Section 5, Tables 6 and 7, report the same quantities for its Python
+    implementation): each workload compiled in its own process on the host cores
+    (compile time, peak RSS, classifier and mask sizes, saved file sizes); then,
+    on the GPU, the decode step on the Java-sized tables (sparse classifier,
+    parser tables read from global memory) and on the 262,144-token C-like
+    tables with the advance's tables staged in shared memory or read from
+    global memory."""
+    jobs = [(2, None), (3, None), (4, None), (5, None), (6, 1024), (6, 2048), (6, 4096)]
+    if args.steps > 1000:   # --steps above 1000: also the 8,192-token Java-sized vocabulary
+        jobs.append((6, 8192))
+    rows = []
+    for cfg, voc in jobs:
+        cmd = [sys.executable, os.path.abspath(__file__), "--mode", "compile-one", "--cfg", str(cfg)]
+        if voc:
+            cmd += ["--vocab", str(voc)]
+        r = subprocess.run(cmd, capture_output=True, text=True)
+        line = [x for x in r.stdout.splitlines() if x.startswith("{")]
+        rows.append(json.loads(line[-1]) if r.returncode == 0 and line else
+                    {"workload": f"config {cfg} vocab {voc}", "error": (r.stderr or r.stdout)[-400:]})
+    out = {"mode": "compile", "metric": "construction time, peak RSS and table sizes", "compile": rows}
+    try:
+        import torch
+        if torch.cuda.is_available():
+            from paper_2608_03065_gb300 import build, psc
+            from workloads import configs
+            build.build()
+            w6 = configs.load(6)
+            h6 = psc.psc_compile(w6.grammar_text, w6.vocab, w6.eos_id, bottom_up=False, **configs.COMPILE_LIMITS[6])
+            out["java_like_decode_step_us"] = {"batch": w6.B, "vocab": w6.V, "graph_us": graph_step_us(psc, h6, w6, w6.B),
+                                               "advance_table_bytes": h6.info().advance_table_bytes,
+                                               "classifier_sparse": h6.info().classifier_sparse}
+            del h6
+            w5 = configs.load(5)
+            for gt in (False, True):
+                h5 = psc.psc_compile(w5.grammar_text, w5.vocab, w5.eos_id, global_tables=gt)
+                out.setdefault("c_like_262144_decode_step_us", {})[
+                    "global_tables" if gt else "staged_tables"] = graph_step_us(psc, h5, w5, w5.B)
+                del h5
+    except Exception as e:   # the construction numbers stand without a GPU
+        out["gpu_error"] = str(e)[:300]
+    print(json.dumps(out))
+
+
 # ------------------------------------------------------------- profile mode
 def run_profile(args):
     """A small case for profiler captures: the workload's tables and prefix states,
@@ -528,11 +655,15 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="gb300")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--mode", default="decode", choices=["decode", "teacher", "sweep", "profile"],
+    ap.add_argument("--cfg", type=int, default=WORKLOAD)
+    ap.add_argument("--vocab", type=int, default=0)
+    ap.add_argument("--mode", default="decode", choices=["decode", "teacher", "sweep", "profile", "compile",
+                                                         "compile-one"],
                     help="decode: the benchmark line; teacher: teacher-forcing pass rates and "
                          "batch-1 step latency (the paper's RQ1/RQ2 measurements on these workloads); "
                          "sweep: decode-step time over batch sizes and logit types on config 5's tables; "
-                         "profile: three decode steps in NVTX ranges, a small case for profiler captures")
+                         "profile: three decode steps in NVTX ranges, a small case for profiler captures; "
+                         "compile: construction time, peak RSS and table sizes at real-grammar scale")
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)
@@ -542,6 +673,10 @@ def main():
         return run_sweep(args)
     if args.mode == "profile":
         return run_profile(args)
+    if args.mode == "compile":
+        return run_compile(args)
+    if args.mode == "compile-one":
+        return compile_one(args.cfg, args.vocab or None)
 
     import torch
     import torch.distributed as dist
