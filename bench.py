@@ -2,7 +2,8 @@
 
 One step = one pass of the whole per-step path over the batch, psc_decode_step
 (called as its two halves, psc_decode_step_mask + psc_decode_step_advance, so
-that the masking kernel can be timed on its own):
+that the masking kernel can be timed on its own; the same steps replayed from a
+CUDA graph are reported beside the timed region):
   k_step_tma       apply every row's precomputed mask to the bf16 logits in
                    place, write the packed bitmask [B][V/32] and pick the greedy
                    token among the allowed ones, in one TMA-pipelined pass
@@ -231,7 +232,8 @@ def config_block(w, n):
             "batch": w.B, "vocab": w.V, "logit_dtype": "bf16", "grammar": "synthetic C-like (150 rules)",
             "parallelism": f"replicas x{n}", "l2": "inputs larger than L2 (512 MiB logits per step)",
             "decode": f"sequences of {SEQ} greedy steps from the prefix states (restored from a device "
-                      "copy before each sequence, inside the timed region); fresh logits every step"}
+                      "copy before each sequence, inside the timed region); each step on its own logits "
+                      "buffer"}
 
 
 def code_only(src: str) -> str:
@@ -721,23 +723,50 @@ def main():
     n_ev = min(K, SEQ)
     ev = [tuple(torch.cuda.Event(enable_timing=True) for _ in range(3)) for _ in range(n_ev)]
 
-    def step(i, timed=None):
+    def step(i, timed=None, cs=None):
+        cs = stream if cs is None else cs
         x = bufs[i]
         if timed is not None:
-            ev[timed][0].record(stream)
-        psc.psc_decode_step_mask(h, st, x, bitmask, stream=stream)
+            ev[timed][0].record(cs)
+        psc.psc_decode_step_mask(h, st, x, bitmask, stream=cs)
         if timed is not None:
-            ev[timed][1].record(stream)
-        psc.psc_decode_step_advance(h, st, tok, stat, stream=stream)
+            ev[timed][1].record(cs)
+        psc.psc_decode_step_advance(h, st, tok, stat, stream=cs)
         if timed is not None:
-            ev[timed][2].record(stream)
+            ev[timed][2].record(cs)
 
-    def restore():
-        psc.psc_state_copy(st, snap, stream=stream)
+    def restore(cs=None):
+        psc.psc_state_copy(st, snap, stream=stream if cs is None else cs)
 
     restore()
     for i in range(Wm):
         step(i)
+    # per-kernel times: one decode sequence with CUDA events between the kernels (an event
+    # between two kernels stops the second from starting during the first one's tail)
+    restore()
+    for i in range(n_ev):
+        step(Wm + i, timed=i)
+    torch.cuda.synchronize()
+    # the same K steps (restores included, each step on its own logits buffer) captured once
+    # in a CUDA graph and replayed (reported beside the timed region: at this batch the GPU
+    # is the bottleneck either way)
+    graph = torch.cuda.CUDAGraph()
+    torch.cuda.synchronize()
+    with torch.cuda.graph(graph):
+        cs = torch.cuda.current_stream()
+        for i in range(K):
+            if i % SEQ == 0:
+                restore(cs)
+            step(Wm + i, cs=cs)
+    torch.cuda.synchronize()
+    g_a, g_b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    g_a.record(stream)
+    graph.replay()
+    g_b.record(stream)
+    torch.cuda.synchronize()
+    graph_ms = max_over_ranks(g_a.elapsed_time(g_b), dev)
+    del graph
+    # the timed region: the K steps called one at a time
     torch.cuda.synchronize()
     barrier()
     torch.cuda.synchronize()
@@ -748,7 +777,7 @@ def main():
         for i in range(K):
             if i % SEQ == 0:
                 restore()
-            step(Wm + i, timed=i if i < n_ev else None)
+            step(Wm + i)
         t_end.record(stream)
         torch.cuda.synchronize()
         torch.cuda.nvtx.range_pop()
@@ -857,6 +886,10 @@ def main():
         "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "u32", "data": "synthetic", "config": config_block(w, world),
         "us_per_step": ms_per_step * 1000.0,
+        "timing": "the K steps called one at a time between CUDA events; per-kernel times from a separate "
+                  "decode sequence with events between the kernels",
+        "graph": {"value": whole_job_rate(world, K, graph_ms), "unit": UNIT, "ms_per_step": graph_ms / K,
+                  "note": "the same K steps captured once in a CUDA graph and replayed"},
         "decode_step_us": step_avg_ms * 1000.0,
         "k_step_tma_us": mask_avg_ms * 1000.0,
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
