@@ -505,7 +505,7 @@ def compile_one(cfg: int, vocab: int | None):
     spec = configs.SPECS[cfg]
     g = configs.grammar_spec(cfg)
     V = vocab or spec.V
-    toks = sample.build_vocab(g, sample.VocabSpec(V, spec.vocab_max_len, spec.frac_grammar), [cfg, 2])
+    toks = configs.vocab_for(cfg, V)
     opts = dict(configs.COMPILE_LIMITS.get(cfg, {}))
     t0 = time.time()
     h = psc.psc_compile(g.text(), toks, len(toks) - 1, host_only=True, **opts)
@@ -580,11 +580,12 @@ def run_compile(args):
     Section 5, Tables 6 and 7, report the same quantities for its Python
     implementation): each workload compiled in its own process on the host cores
     (compile time, peak RSS, classifier and mask sizes, saved file sizes); then,
-    on the GPU, the decode step on the Java-sized tables (sparse classifier,
-    parser tables read from global memory) and on the 262,144-token C-like
+    on the GPU, the decode step on the Java-sized tables at 4,096 and 262,144
+    tokens (sparse classifier, parser tables read from global memory, stacks
+    walked from the top) and on the 262,144-token C-like
     tables with the advance's tables staged in shared memory or read from
     global memory."""
-    jobs = [(2, None), (3, None), (4, None), (5, None), (6, 1024), (6, 2048), (6, 4096)]
+    jobs = [(2, None), (3, None), (4, None), (5, None), (6, 1024), (6, 2048), (6, 4096), (7, 131072), (7, None)]
     if args.steps > 1000:   # --steps above 1000: also the 8,192-token Java-sized vocabulary
         jobs.append((6, 8192))
     rows = []
@@ -609,6 +610,13 @@ def run_compile(args):
                                                "advance_table_bytes": h6.info().advance_table_bytes,
                                                "classifier_sparse": h6.info().classifier_sparse}
             del h6
+            w7 = configs.load(7)
+            h7 = psc.psc_compile(w7.grammar_text, w7.vocab, w7.eos_id, bottom_up=False, **configs.COMPILE_LIMITS[7])
+            out["java_like_pretok_262144_decode_step_us"] = {
+                "batch": w7.B, "vocab": w7.V, "graph_us": graph_step_us(psc, h7, w7, w7.B),
+                "advance_table_bytes": h7.info().advance_table_bytes,
+                "classifier_sparse": h7.info().classifier_sparse}
+            del h7
             w5 = configs.load(5)
             for gt in (False, True):
                 h5 = psc.psc_compile(w5.grammar_text, w5.vocab, w5.eos_id, global_tables=gt)

@@ -960,13 +960,17 @@ Tables compile_tables(const std::string& text, const uint8_t* vb, const int64_t*
     double t7 = now();
     // optional: empty tables when a size limit or the host's memory stops it (the device
     // then walks stacks from the top)
+    bool built = false;
     try {
-        build_bottom_up(T, opt);
+        built = build_bottom_up(T, opt);
     } catch (const std::bad_alloc&) {
         Options off = opt;
         off.max_bottom_up_bytes = -1;
         build_bottom_up(T, off);   // clears the partial tables
     }
+    if (!built && getenv("PSC_LOG"))
+        fprintf(stderr, "psc: no bottom-up classifier (switched off, or over max_bottom_up_bytes or "
+                        "max_states): stacks are walked from the top\n");
     T.seconds_total = now() - t0;
     if (getenv("PSC_LOG"))
         fprintf(stderr, "psc: compile %.2f s: grammar+lexer+LALR %.2f s, token tries %.2f s, classifier %.2f s, "

@@ -12,6 +12,9 @@ the CPU oracle.
   tables too large for shared memory, so the advance reads them from global
   memory), 4,096 tokens, 64 rows: all rows over all tokens at the prefix states
   and through six whole decode steps.
+* The same grammar with a pre-tokenized vocabulary of 262,144 tokens, 256 rows:
+  all rows over all tokens at the prefix states (fused masking pass with the
+  greedy choice) and through four whole decode steps.
 * The C-like 262,144-token workload on the benchmark's exact path: the batch restored from a
   saved copy (psc_state_copy), then 32 steps of psc_decode_step_mask +
   psc_decode_step_advance on fresh logits; the oracle is advanced by the same
@@ -100,15 +103,18 @@ def device_logits(B, V, seed, sigma):
 STATUS = {ST_OK: 0, ST_DONE: 1, ST_ERROR: 2}
 
 
-def test_c_like_151936_whole_decode_all_rows_all_tokens(psc):
-    b = big(psc, 4)
+def whole_decode_all_rows_all_tokens(psc, b, steps, seed):
+    """``steps`` whole decode steps (psc_decode_step) on fresh logits from the
+    restored prefix states; after every step the bitmask, the masked logits and
+    the greedy tokens of all rows over all tokens, and the statuses of all rows,
+    equal the oracle's."""
     w = b.w
     B, V = w.B, w.V
     st, ocs = b.restored(psc)
     tok = torch.empty(B, dtype=torch.int32, device="cuda")
     stat = torch.empty(B, dtype=torch.int32, device="cuda")
-    for step in range(4):
-        x, logits = device_logits(B, V, 4000 + step, w.spec.sigma)
+    for step in range(steps):
+        x, logits = device_logits(B, V, seed + step, w.spec.sigma)
         bm = torch.zeros(B, b.h.W, dtype=torch.int32, device="cuda")
         psc.psc_decode_step(b.h, st, x, tok, bm, stat)
         torch.cuda.synchronize()
@@ -123,33 +129,43 @@ def test_c_like_151936_whole_decode_all_rows_all_tokens(psc):
             if t[r] >= 0:
                 ost = b.o.advance(ocs[r], None if t[r] == w.eos_id else w.vocab[t[r]])
                 assert s[r] == STATUS[ost], (step, r, s[r], ost)
+
+
+def test_c_like_151936_whole_decode_all_rows_all_tokens(psc):
+    whole_decode_all_rows_all_tokens(psc, big(psc, 4), 4, 4000)
 
 
 def test_java_sized_grammar_whole_decode_all_rows_all_tokens(psc):
     b = big(psc, 6, bottom_up=False, **configs.COMPILE_LIMITS[6])
+    info = b.h.info()
+    assert info.n_parser_states >= 1000 and info.classifier_sparse == 1 and info.advance_table_bytes == 0
+    whole_decode_all_rows_all_tokens(psc, b, 6, 7000)
+
+
+def test_java_sized_grammar_262144_pretokenized_all_rows_all_tokens(psc):
+    """The Java-sized grammar at the paper's largest vocabulary size, with a
+    pre-tokenized vocabulary: the fused masking pass at the prefix states, then
+    four whole decode steps, every row over every token.  (The bottom-up
+    classifier is left out: on this grammar it passes its memory budget, and the
+    device walks the stacks from the top, which is what the default compile
+    falls back to.)"""
+    b = big(psc, 7, bottom_up=False, **configs.COMPILE_LIMITS[7])
     w = b.w
     info = b.h.info()
     assert info.n_parser_states >= 1000 and info.classifier_sparse == 1 and info.advance_table_bytes == 0
-    B, V = w.B, w.V
-    st, ocs = b.restored(psc)
-    tok = torch.empty(B, dtype=torch.int32, device="cuda")
-    stat = torch.empty(B, dtype=torch.int32, device="cuda")
-    for step in range(6):
-        x, logits = device_logits(B, V, 7000 + step, w.spec.sigma)
-        bm = torch.zeros(B, b.h.W, dtype=torch.int32, device="cuda")
-        psc.psc_decode_step(b.h, st, x, tok, bm, stat)
-        torch.cuda.synchronize()
-        ref = b.o.masks(ocs, b.voc, threads=THREADS)
-        np.testing.assert_array_equal(bm.cpu().numpy().view(np.uint32), ref, err_msg=f"step {step}")
-        allowed = bits_of(ref, V)
-        np.testing.assert_array_equal(raw_bits(x), reference_masked(logits, allowed), err_msg=f"step {step}")
-        t = tok.cpu().numpy()
-        np.testing.assert_array_equal(t, cpu_greedy(logits, allowed), err_msg=f"step {step}")
-        s = stat.cpu().numpy()
-        for r in range(B):
-            if t[r] >= 0:
-                ost = b.o.advance(ocs[r], None if t[r] == w.eos_id else w.vocab[t[r]])
-                assert s[r] == STATUS[ost], (step, r, s[r], ost)
+    assert w.V == 262144 and w.B == 256
+    ref = b.o.masks(b.ocs0, b.voc, threads=THREADS)
+    st, _ = b.restored(psc)
+    x, logits = device_logits(w.B, w.V, 7500, w.spec.sigma)
+    bm = torch.zeros(w.B, b.h.W, dtype=torch.int32, device="cuda")
+    tok = torch.empty(w.B, dtype=torch.int32, device="cuda")
+    psc.psc_fill_apply_argmax(b.h, st, x, tok, bm)
+    torch.cuda.synchronize()
+    allowed = bits_of(ref, w.V)
+    np.testing.assert_array_equal(bm.cpu().numpy().view(np.uint32), ref)
+    np.testing.assert_array_equal(raw_bits(x), reference_masked(logits, allowed))
+    np.testing.assert_array_equal(tok.cpu().numpy(), cpu_greedy(logits, allowed))
+    whole_decode_all_rows_all_tokens(psc, b, 4, 7600)
 
 
 def test_c_like_262144_prefix_states_all_rows_all_tokens(psc):

@@ -13,7 +13,7 @@ torch = pytest.importorskip("torch")
 SINGLES = {bytes([b]) for b in list(range(0x20, 0x7F)) + [9, 10, 13]}
 
 
-@pytest.mark.parametrize("cfg_id,batch", [(1, None), (2, None), (3, 16), (4, 16), (5, 16), (6, 16)])
+@pytest.mark.parametrize("cfg_id,batch", [(1, None), (2, None), (3, 16), (4, 16), (5, 16), (6, 16), (7, 16)])
 def test_vocabulary_and_prefixes(cfg_id, batch):
     w = configs.load(cfg_id, batch=batch)
     s = configs.SPECS[cfg_id]
@@ -30,6 +30,24 @@ def test_vocabulary_and_prefixes(cfg_id, batch):
         assert w.eos_id not in ids
     m = w.token_matrix()
     assert m.shape[0] == w.B and m.dtype == np.int32
+
+
+def test_pretokenized_vocabulary_follows_the_splitting_rule():
+    """Workload 7's tokens are each one pre-token of the byte-level BPE splitting
+    rule (single bytes aside): no token mixes letters with punctuation, numbers
+    have at most three digits; about 3 % are punctuation runs, the structure
+    that makes a token span several grammar symbols."""
+    import re
+    from workloads import sample
+    w = configs.load(7, batch=16)
+    toks = [t for t in w.vocab[:-1] if len(t) > 1]
+    assert all(sample.PRETOKEN.fullmatch(t) for t in toks)
+    assert not any(re.search(rb"[A-Za-z][^A-Za-z]|[0-9][^0-9]", t) for t in toks)
+    assert not any(re.fullmatch(rb"[0-9]{4,}", t) for t in toks)
+    punct = [t for t in toks if re.fullmatch(rb" ?[!-/:-@\[-`{-~]+\n*", t)]
+    assert 0.02 * w.V < len(punct) < 0.06 * w.V
+    assert {b");", b"()", b" {"} <= set(toks) | set(w.vocab)
+    assert configs.vocab_for(7, 4096)[:-1] != w.vocab[:4095]   # the size is part of the recipe
 
 
 @pytest.mark.parametrize("cfg_id", [1, 2])

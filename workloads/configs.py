@@ -1,4 +1,4 @@
-"""The five seeded synthetic workloads (grammar, vocabulary, batch of prefixes, logits).
+"""The seeded synthetic workloads (grammar, vocabulary, batch of prefixes, logits).
 
 1. tiny arithmetic grammar, V=512, B=8, prefixes of 1-64 bytes, fp32 logits ~N(0,1)
 2. JSON (RFC 8259), V=32,000, B=64, prefixes up to 512 bytes, bf16 logits ~N(0,2)
@@ -7,6 +7,8 @@
 5. C-like language, V=262,144, B=1024, prefixes of 64-4096 bytes biased to deep nesting,
    bf16 logits ~N(0,2), 32 decode steps
 6. (extra) Java-sized language (1,001 LALR(1) states), V=4,096, B=64, prefixes of 64-2048 bytes
+7. (extra) the same language with a pre-tokenized vocabulary of V=262,144 (the size of the
+   paper's largest tokenizer), B=256, prefixes of 64-2048 bytes
 
 N(0,2) is read as variance 2 (sigma = sqrt 2).  The paper's datasets, JSON
 schemas and tokenizers are not available; these stand in for them.
@@ -20,7 +22,7 @@ from dataclasses import dataclass
 import numpy as np
 
 from . import grammars
-from .sample import TrieTokenizer, VocabSpec, build_prefixes, build_vocab
+from .sample import TrieTokenizer, VocabSpec, build_prefixes, build_vocab, build_vocab_pretokenized
 
 
 @dataclass(frozen=True)
@@ -38,6 +40,7 @@ class WorkloadSpec:
     nest_bias: float = 1.0
     max_depth: int = 40
     decode_steps: int = 1
+    vocab_style: str = "fragments"   # "fragments" or "pretokenized" (see sample.py)
 
 
 SPECS = {
@@ -53,8 +56,14 @@ SPECS = {
     # scale; its vocabulary is sized so that the construction fits a test run
     6: WorkloadSpec(6, "java_like_v4096_b64", 64, 4096, "bf16", math.sqrt(2), 64, 2048, 24, 0.7,
                     max_depth=60),
+    # not a benchmark configuration either: the Java-sized grammar at the vocabulary size of
+    # the paper's Java runs, with tokens that never mix letters and punctuation (the rule of
+    # the byte-level BPE tokenizers the paper uses); 3 % of the tokens are punctuation runs
+    7: WorkloadSpec(7, "java_like_pretok_v262144_b256", 256, 262144, "bf16", math.sqrt(2), 64, 2048, 24,
+                    0.0, max_depth=60, vocab_style="pretokenized"),
 }
-COMPILE_LIMITS = {6: {"max_states": 64_000_000}}   # the Java-sized construction builds ~20 M states
+# the Java-sized constructions build ~20 M states (6) and ~16 M states (7)
+COMPILE_LIMITS = {6: {"max_states": 64_000_000}, 7: {"max_states": 64_000_000}}
 
 
 def grammar_spec(cfg: int) -> grammars.GrammarSpec:
@@ -64,7 +73,7 @@ def grammar_spec(cfg: int) -> grammars.GrammarSpec:
         return grammars.json_grammar()
     if cfg == 3:
         return grammars.schema_json(seed=int(np.random.default_rng([3, 1]).integers(0, 2**31)))
-    if cfg == 6:
+    if cfg in (6, 7):
         return grammars.java_like()
     return grammars.c_like()
 
@@ -109,12 +118,24 @@ class Workload:
         return x if self.spec.dtype == "f32" else x.to(torch.bfloat16)
 
 
+def vocab_spec(cfg: int, V: int | None = None) -> VocabSpec:
+    s = SPECS[cfg]
+    return VocabSpec(V or s.V, s.vocab_max_len, s.frac_grammar, style=s.vocab_style)
+
+
+def vocab_for(cfg: int, V: int | None = None) -> list[bytes]:
+    """Workload ``cfg``'s vocabulary (optionally at another size V)."""
+    vs = vocab_spec(cfg, V)
+    build = build_vocab_pretokenized if vs.style == "pretokenized" else build_vocab
+    return build(grammar_spec(cfg), vs, [cfg, 2])
+
+
 @functools.lru_cache(maxsize=8)
 def load(cfg: int, batch: int | None = None) -> Workload:
     """Build workload ``cfg`` (optionally with only the first ``batch`` rows)."""
     s = SPECS[cfg]
     g = grammar_spec(cfg)
-    vocab = build_vocab(g, VocabSpec(s.V, s.vocab_max_len, s.frac_grammar), [cfg, 2])
+    vocab = vocab_for(cfg)
     B = s.B if batch is None else batch
     prefixes = build_prefixes(g, B, s.prefix_min, s.prefix_max, [cfg, 3],
                               max_depth=s.max_depth, nest_bias=s.nest_bias)

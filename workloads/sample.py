@@ -10,6 +10,8 @@ generator seeded with ``1000 * config_id + 4``).
 """
 from __future__ import annotations
 
+import collections
+import re
 from dataclasses import dataclass
 
 import numpy as np
@@ -110,6 +112,8 @@ class VocabSpec:
     max_len: int
     frac_grammar: float          # fraction of fragments cut from grammar sentences
     unicode: bool = True
+    style: str = "fragments"     # "fragments" or "pretokenized"
+    frac_punct: float = 0.03     # pretokenized: fraction of punctuation-run tokens
 
 
 PRINTABLE = [bytes([b]) for b in range(0x20, 0x7F)] + [b"\t", b"\n", b"\r"]
@@ -167,6 +171,101 @@ def build_vocab(spec: GrammarSpec, vs: VocabSpec, seed_key) -> list[bytes]:
         if len(frag) <= vs.max_len and frag not in seen:
             seen.add(frag)
             toks.append(frag)
+    perm = rng.permutation(len(toks))
+    toks = [toks[int(i)] for i in perm]
+    toks.append(b"")          # end of sequence
+    return toks
+
+
+# The splitting rule of byte-level BPE tokenizers of the GPT / Llama 3 / Qwen2.5
+# kind (ASCII form): text is cut into words with at most one leading non-letter,
+# numbers of up to three digits, punctuation runs with an optional leading space
+# and trailing newlines, and whitespace runs; merges never cross a cut, so no
+# token mixes letters with punctuation.
+PRETOKEN = re.compile(rb"[^\r\nA-Za-z0-9]?[A-Za-z]+|[0-9]{1,3}| ?[^\sA-Za-z0-9]+[\r\n]*|\s*[\r\n]+|\s+(?!\S)|\s+")
+_PUNCT_RUN = re.compile(rb" ?[^\sA-Za-z0-9]+[\r\n]*")
+_PUNCT_CHARS = b"(){}[];,.=<>+-*/%&|^!~?:@\"'#$\\"
+
+
+def build_vocab_pretokenized(spec: GrammarSpec, vs: VocabSpec, seed_key,
+                             corpus_bytes: int = 1 << 20) -> list[bytes]:
+    """A vocabulary shaped like a pre-tokenized byte-level BPE vocabulary of
+    ``vs.size`` unique byte strings: every single printable byte; the pre-tokens
+    of sampled grammar sentences and their prefixes (the intermediate merges) by
+    frequency; punctuation runs (a fraction ``vs.frac_punct`` of the vocabulary:
+    the corpus's own, then random runs over code punctuation); numbers 0-999;
+    indentation runs; and, for the rest, natural-language words with at most one
+    leading non-letter and some non-ASCII pieces.  Every token but the single
+    bytes is one pre-token (PRETOKEN matches it whole).  The last id is the
+    end-of-sequence token (empty bytes)."""
+    rng = np.random.default_rng(seed_key)
+    sampler = SentenceSampler(spec, max_depth=30)
+    cnt: collections.Counter = collections.Counter()
+    n = 0
+    while n < corpus_bytes:
+        txt, _ = sampler.text(rng, 4096)
+        n += len(txt)
+        for m in PRETOKEN.finditer(txt):
+            p = m.group(0)
+            cnt[p] += 1.0
+            for k in range(2, len(p)):
+                cnt[p[:k]] += 0.2
+    toks: list[bytes] = list(PRINTABLE)
+    seen = set(toks)
+    n_target = vs.size - 1
+
+    def add(t: bytes) -> bool:
+        if t and t not in seen and len(t) <= vs.max_len and len(toks) < n_target \
+                and PRETOKEN.fullmatch(t):
+            seen.add(t)
+            toks.append(t)
+            return True
+        return False
+
+    ranked = [p for p, _ in sorted(cnt.items(), key=lambda kv: (-kv[1], kv[0]))]
+    n_punct = int(vs.size * vs.frac_punct)
+    k = 0
+    for p in ranked:
+        if k < n_punct and _PUNCT_RUN.fullmatch(p) and add(p):
+            k += 1
+    stall = 0
+    while k < n_punct and stall < 100000:
+        ln = 1 + int(min(rng.geometric(0.35), 7))
+        r = bytes(_PUNCT_CHARS[int(i)] for i in rng.integers(0, len(_PUNCT_CHARS), ln))
+        if rng.random() < 0.3:
+            r = b" " + r
+        if rng.random() < 0.2:
+            r += b"\n" * int(rng.integers(1, 3))
+        if add(r):
+            k += 1
+            stall = 0
+        else:
+            stall += 1
+    for p in ranked:
+        if len(toks) >= n_target // 4:
+            break
+        if not _PUNCT_RUN.fullmatch(p):
+            add(p)
+    for i in range(1000):
+        add(str(i).encode())
+    for w in range(2, 17):
+        add(b" " * w)
+        add(b"\n" + b" " * w)
+        add(b"\t" * (w // 2))
+    lead = [b"", b" ", b" ", b" ", b".", b"(", b"_", b"@", b"\"", b"'"]
+    stall = 0
+    while len(toks) < n_target and stall < 100000:
+        if vs.unicode and rng.random() < 0.05:
+            w = b" " + "".join(_UNI[int(i)] for i in rng.integers(0, len(_UNI), int(rng.integers(1, 4)))).encode()
+        else:
+            ln = int(rng.integers(1, 11))
+            w = bytes(int(c) for c in rng.integers(ord("a"), ord("z") + 1, ln))
+            if rng.random() < 0.3:
+                w = w[:1].upper() + w[1:]
+            w = lead[int(rng.integers(0, len(lead)))] + w
+        stall = 0 if add(w) else stall + 1
+    if len(toks) < n_target:
+        raise ValueError(f"pretokenized vocabulary stalled at {len(toks)} of {n_target} tokens")
     perm = rng.permutation(len(toks))
     toks = [toks[int(i)] for i in perm]
     toks.append(b"")          # end of sequence
