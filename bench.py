@@ -632,13 +632,17 @@ def run_compile(args):
 def run_profile(args):
     """A small case for profiler captures: the workload's tables and prefix states,
     then three decode steps (psc_decode_step_mask + psc_decode_step_advance) on
-    fresh logits, each inside an NVTX range named "decode" (about 2 GB on the device)."""
+    fresh logits, each inside an NVTX range named "decode" (config 5 by default, about
+    2 GB on the device; --cfg picks another workload)."""
     import torch
     from paper_2608_03065_gb300 import build, psc
     from workloads import configs
     build.build()
-    w = configs.load(WORKLOAD)
-    h = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id)
+    w = configs.load(args.cfg)
+    opts = dict(configs.COMPILE_LIMITS.get(args.cfg, {}))
+    if args.cfg in (6, 7):
+        opts["bottom_up"] = False   # over its construction budget on the Java-sized grammar
+    h = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id, **opts)
     st = psc.psc_state_init(h, w.B, 256)
     tm = torch.from_numpy(w.token_matrix()).cuda()
     for j in range(tm.shape[1]):

@@ -73,9 +73,15 @@ typedef struct {
     int64_t max_mask_bytes;  /* host bytes of distinct mask rows before PSC_ERR_LIMIT (0 = 24 GiB) */
     int32_t threads;         /* host threads for compilation (0 = all cores) */
     int32_t host_only;       /* 1: build host tables only (no GPU needed; device calls fail) */
-    int32_t global_tables;   /* 1: psc_advance reads its tables from global memory even when they
-                                would fit in shared memory (0 = stage them when they fit) */
-    int64_t max_bottom_up_bytes;  /* host memory for building the bottom-up classifier (0 = 8 GiB);
+    int32_t global_tables;   /* where the advance kernel reads the lexer and parser tables:
+                                0 = staged in shared memory, dense when they fit in 200 KiB, else
+                                packed (ACTION and GOTO row-displaced into one table of owner-
+                                checked entries, lexeme classes resolved through candidate lists)
+                                when those fit, else global memory; 1 = global memory;
+                                2 = staged packed tables whenever they fit.  Other values:
+                                PSC_ERR_ARG. */
+    int64_t max_bottom_up_bytes;  /* host memory for building the bottom-up classifier (0 = 16 GiB,
+                                     at most half of the machine's memory);
                                      negative: not built (psc_load: dropped), and the device walks
                                      every stack from the top.  Over the limit it is not built
                                      (no error). */
@@ -98,12 +104,14 @@ typedef struct {
                                   held as ids of 1024-token chunks, equal chunks stored once */
     int64_t states_built;      /* classifier states before minimisation */
     double compile_seconds;
-    int64_t advance_table_bytes;  /* bytes psc_advance stages in shared memory (0: it reads global memory) */
+    int64_t advance_table_bytes;  /* bytes psc_advance stages in shared memory (0: it reads global memory;
+                                     a host_only handle: what a device upload would stage) */
     int64_t device_timeouts;      /* bounded in-kernel waits that gave up since the library was loaded
                                      (process-wide; non-zero means a pipeline fault; reading it synchronises) */
     int64_t bottom_up_states;     /* states of the bottom-up classifier (0: not built) */
     int64_t bottom_up_bytes;      /* its device bytes (blocks, edge slots, final table) */
     int64_t classifier_sparse;    /* 1: the classifier DFA is held in the sparse layout */
+    int64_t advance_tables_packed;  /* 1: the staged parser tables are in the packed layout */
 } psc_info_t;
 
 /* Offline construction (Algorithm 1, Section 3).  Reads the grammar text (a

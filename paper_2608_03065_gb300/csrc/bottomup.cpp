@@ -36,6 +36,8 @@
 #include <thread>
 #include <unordered_map>
 
+#include <unistd.h>
+
 #include "psc_internal.h"
 
 namespace psc {
@@ -91,7 +93,11 @@ bool build_bottom_up(Tables& T, const Options& opt) {
     T.n_bu = 0;
     T.n_frow = 0;
     if (opt.max_bottom_up_bytes < 0) return false;
-    const int64_t budget = opt.max_bottom_up_bytes > 0 ? opt.max_bottom_up_bytes : (int64_t(8) << 30);
+    // default budget: 16 GiB, at most half of the machine's memory
+    int64_t dflt = int64_t(16) << 30;
+    long pages = sysconf(_SC_PHYS_PAGES), psize = sysconf(_SC_PAGESIZE);
+    if (pages > 0 && psize > 0) dflt = std::min<int64_t>(dflt, (int64_t)pages * psize / 2);
+    const int64_t budget = opt.max_bottom_up_bytes > 0 ? opt.max_bottom_up_bytes : dflt;
     const int n = T.n_lr, S = T.S, nq = T.nq;
     if (n <= 0 || n > 32767 || (int64_t)n * n * 2 > (int64_t(64) << 20)) return false;
     int threads = opt.threads > 0 ? opt.threads : (int)std::max(1u, std::thread::hardware_concurrency());
@@ -373,9 +379,11 @@ bool build_bottom_up(Tables& T, const Options& opt) {
     T.n_bu = R;
     T.n_frow = (int)(T.bu_F.size() / nq);
     if (log)
-        fprintf(stderr, "psc: bottom-up classifier: %d states, %d final rows; domains %.2f s, steps %.2f s, "
-                        "states %.2f s (%d batches: parallel %.2f s, serial %.2f s), final %.2f s\n",
-                R, T.n_frow, t1 - t0, t2 - t1, t3 - t2, n_batches, t_par, t_ser, seconds() - t3);
+        fprintf(stderr, "psc: bottom-up classifier: %d states, %d final rows, %.2f GiB of construction vectors; "
+                        "domains %.2f s, steps %.2f s, states %.2f s (%d batches: parallel %.2f s, serial %.2f s), "
+                        "final %.2f s\n",
+                R, T.n_frow, ((double)arena.n * 4 + (double)tr.size() * 4 + (double)step_bytes) / (1 << 30),
+                t1 - t0, t2 - t1, t3 - t2, n_batches, t_par, t_ser, seconds() - t3);
     return true;
 }
 

@@ -635,6 +635,13 @@ Tables compile_tables(const std::string& text, const uint8_t* vb, const int64_t*
     std::vector<int> rank = terminal_rank(g);
     Lexer L = build_lexer(g, rank);
     Parser P = build_lalr(g);
+    if (getenv("PSC_LOG")) {
+        size_t na = 0, ng = 0, nr = 0;
+        for (int32_t x : P.action) na += act_kind(x) != ACT_ERR, nr += act_kind(x) == ACT_REDUCE;
+        for (int32_t x : P.go) ng += x >= 0;
+        fprintf(stderr, "psc: LALR(1): %d states, %d terminals, %d nonterminals, %zu actions (%zu reduce), %zu gotos, "
+                        "%zu lexeme classes\n", P.n_states, P.n_terms, P.n_nts, na, nr, ng, L.classes.size());
+    }
     int threads = opt.threads > 0 ? opt.threads : (int)std::max(1u, std::thread::hardware_concurrency());
     int ncls = (int)L.classes.size();
     int end_cls = ncls;   // pseudo class of the end marker

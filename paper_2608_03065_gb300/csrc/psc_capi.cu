@@ -25,7 +25,10 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <cstdio>
+#include <cstdlib>
 #include <cstring>
+#include <map>
 #include <memory>
 #include <mutex>
 #include <new>
@@ -74,6 +77,12 @@ struct DevTables {
     const uint8_t* adv;
     int adv_bytes, o_bc, o_trans, o_accept, o_ign, o_resolve, o_action, o_go, o_rlen, o_rlhs, nbc;
     int adv_packed;   // reduce entries of the compact ACTION hold (rule length << 10 | lhs) instead of the rule
+    // packed (row-displaced) parser tables, for grammars whose dense compact tables do not
+    // fit in shared memory: ACTION and GOTO each as a table of uint32 entries (row id << 16
+    // | int16 entry) with equal rows stored once, and per state a word (row id << 17 | base):
+    // the entry (s, x) is the one at base + x when its row id is the state's; lexeme
+    // classes resolved through candidate terminal lists
+    int adv_comb, o_cand, o_abase, o_gbase, o_acmb, o_gcmb, kc;
     // bottom-up classifier (bu = nullptr: not built; the root block, for the stack [0], is at 0)
     const int32_t* bu;        // blocks [final row, next block per successor slot]
     const int16_t* bu_slot;   // [n_lr][n_lr] slot of the LR edge t -> u, -1 none
@@ -103,6 +112,7 @@ struct psc_handle {
     void* blocks[32] = {};
     int n_blocks = 0;
     int tma_ctas[2] = {1, 1};   // resident k_step_tma CTAs per SM (bf16, f32)
+    int tables = 0;             // psc_options.global_tables the handle was made with
 };
 
 struct psc_states {
@@ -985,6 +995,7 @@ __global__ void k_finalize_tokens(unsigned long long* __restrict__ best_key, int
 constexpr int ADV_WARPS = 8;     // rows per CTA
 constexpr int ADV_WIN = 256;     // stack entries held per row
 constexpr int ADV_KEEP = 192;    // entries copied in (the rest is room for pushes)
+constexpr size_t ADV_TABLE_MAX = 200 * 1024;   // staged tables at most (one CTA of 8 rows per SM)
 
 // Dynamic shared memory of k_advance_warp: the staged tables, then the stack windows.
 int adv_smem(const DevTables& d) { return d.adv_bytes + ADV_WARPS * ADV_WIN * 2; }
@@ -1036,6 +1047,16 @@ __device__ __forceinline__ int lds_u8(uint32_t a) {
     asm volatile("ld.shared.u8 %0, [%1];" : "=h"(v) : "r"(a));
     return v;
 }
+__device__ __forceinline__ int lds_s32(uint32_t a) {
+    int v;
+    asm volatile("ld.shared.s32 %0, [%1];" : "=r"(v) : "r"(a));
+    return v;
+}
+__device__ __forceinline__ uint32_t lds_u32(uint32_t a) {
+    uint32_t v;
+    asm volatile("ld.shared.u32 %0, [%1];" : "=r"(v) : "r"(a));
+    return v;
+}
 __device__ __forceinline__ void sts_u16(uint32_t a, int v) {
     asm volatile("st.shared.u16 [%0], %1;" ::"r"(a), "h"((unsigned short)v) : "memory");
 }
@@ -1063,11 +1084,14 @@ struct StackView {
 struct AdvTabs {
     uint32_t bc, trans, acc, ign, res, act, go, rlen, rlhs;
     uint32_t trans_row, res_row, act_row, go_row;   // bytes per row: nbc, n_lr, n_terms, n_nts int16 entries
-    int q0;
+    uint32_t cand, abase, gbase, acmb, gcmb;       // packed layout
+    int q0, kc;
     __device__ __forceinline__ AdvTabs(uint32_t sb, const DevTables& T)
         : bc(sb + T.o_bc), trans(sb + T.o_trans), acc(sb + T.o_accept), ign(sb + T.o_ign), res(sb + T.o_resolve),
           act(sb + T.o_action), go(sb + T.o_go), rlen(sb + T.o_rlen), rlhs(sb + T.o_rlhs),
-          trans_row(2u * T.nbc), res_row(2u * T.n_lr), act_row(2u * T.n_terms), go_row(2u * T.n_nts), q0(T.q0) {}
+          trans_row(2u * T.nbc), res_row(2u * T.n_lr), act_row(2u * T.n_terms), go_row(2u * T.n_nts),
+          cand(sb + T.o_cand), abase(sb + T.o_abase), gbase(sb + T.o_gbase), acmb(sb + T.o_acmb),
+          gcmb(sb + T.o_gcmb), q0(T.q0), kc(T.kc) {}
 };
 
 // Feed one lexeme class to the parser: resolve it to a terminal with the
@@ -1137,6 +1161,92 @@ __device__ __forceinline__ int feed_class_win(const AdvTabs& A, StackView& sv, i
         top = g;
     }
     return ROW_LIMIT;
+}
+
+// Entry x of a packed table's row (w = the state's word, row id << 17 | base): the
+// int16 entry when the slot belongs to the row, else `miss` (an ACTION error is 0,
+// a missing GOTO -1).
+__device__ __forceinline__ int comb_get(uint32_t tab, uint32_t w, int x, int miss) {
+    uint32_t e = lds_u32(tab + 4u * ((w & 0x1FFFFu) + (uint32_t)x));
+    return (e >> 16) == (w >> 17) ? (int)(int16_t)(e & 0xFFFFu) : miss;
+}
+
+// feed_class_win over the packed tables: the class is resolved by trying its
+// candidate terminals in order (the first with an action in the top state); the
+// ACTION word of the top stays in a register, each GOTO lookup first reads the
+// word of the uncovered state (once per run of one-symbol reductions).
+template <bool PACKED>
+__device__ __forceinline__ int feed_class_comb(const AdvTabs& A, StackView& sv, int& depth, int& top, int& below,
+                                               int cap, int cls) {
+    uint32_t tw = lds_u32(A.abase + 4u * top);
+    int t = -1, a = 0;
+    for (int k = 0; k < A.kc; k++) {
+        int c = lds_s16(A.cand + 2u * (cls * A.kc + k));
+        if (c < 0) break;
+        a = comb_get(A.acmb, tw, c, 0);
+        if ((a & 3) != psc::ACT_ERR) {
+            t = c;
+            break;
+        }
+    }
+    if (t < 0) return ROW_REJECTED;
+    bool dirty = false;
+    for (int guard = 0; guard < 4 * cap + 64; guard++) {
+        if (guard > 0) a = comb_get(A.acmb, tw, t, 0);
+        if (PACKED && (a & 0xF003) == 0x1002 && depth >= 2) {
+            const uint32_t bw = lds_u32(A.gbase + 4u * below);
+            do {   // one-symbol reductions: GOTO[below][lhs], lhs in bits 2-11
+                int g = comb_get(A.gcmb, bw, (a >> 2) & 1023, -1);
+                if (g < 0) return ROW_REJECTED;
+                if (++guard >= 4 * cap + 64) return ROW_LIMIT;
+                top = g;
+                dirty = true;
+                tw = lds_u32(A.abase + 4u * top);
+                a = comb_get(A.acmb, tw, t, 0);
+            } while ((a & 0xF003) == 0x1002);
+        }
+        int kind = a & 3, val = (a >> 2) & 0x3FFF;
+        if (kind == psc::ACT_SHIFT) {
+            if (depth >= cap) return ROW_OVERFLOW;
+            if (dirty) sv.set(depth - 1, top);
+            sv.set(depth++, val);
+            below = top;
+            top = val;
+            return ROW_OK;
+        }
+        if (kind != psc::ACT_REDUCE) return ROW_REJECTED;
+        int k, lhs;
+        if (PACKED) {
+            k = val >> 10;
+            lhs = val & 1023;
+        } else {
+            k = lds_u8(A.rlen + val);
+            lhs = lds_s16(A.rlhs + 2u * val);
+        }
+        if (depth - k < 1) return ROW_REJECTED;
+        if (k == 0 && dirty) sv.set(depth - 1, top);
+        dirty = false;
+        depth -= k;
+        int under;
+        if (k == 1) under = below;
+        else if (k == 0) under = top;
+        else under = sv.get(depth - 1);
+        int g = comb_get(A.gcmb, lds_u32(A.gbase + 4u * under), lhs, -1);
+        if (g < 0) return ROW_REJECTED;
+        if (depth >= cap) return ROW_OVERFLOW;
+        sv.set(depth++, g);
+        below = under;
+        top = g;
+        tw = lds_u32(A.abase + 4u * top);
+    }
+    return ROW_LIMIT;
+}
+
+template <bool PACKED, bool COMB>
+__device__ __forceinline__ int feed_class(const AdvTabs& A, StackView& sv, int& depth, int& top, int& below, int cap,
+                                          int cls) {
+    if (COMB) return feed_class_comb<PACKED>(A, sv, depth, top, below, cap, cls);
+    return feed_class_win<PACKED>(A, sv, depth, top, below, cap, cls);
 }
 
 // Classifier walk of a configuration (lexer state q, stack of the given depth
@@ -1214,7 +1324,7 @@ __device__ __forceinline__ int warp_memo_extend(const DevTables& T, const StackV
 // kernel start only after its own wait for the advance before it, which wrote the
 // rows; the host sets `early` only when the masking pass is the last work on
 // these states and took the mask ids as they were.
-template <bool PACKED>
+template <bool PACKED, bool COMB>
 __global__ void __launch_bounds__(ADV_WARPS * 32) k_advance_warp(DevTables T, DevStates S, const int32_t* tokens,
                                                                  int B, int use_mid, int32_t* status_out,
                                                                  int from_keys, int32_t* tokens_out, int early) {
@@ -1402,7 +1512,7 @@ __global__ void __launch_bounds__(ADV_WARPS * 32) k_advance_warp(DevTables T, De
             int below = depth >= 2 ? sv.get(depth - 2) : 0;
             if (ncls >= 0) {
                 for (int k = 0; k < ncls && status == ROW_OK; k++)
-                    status = feed_class_win<PACKED>(A, sv, nd, top, below, S.cap, lds_u16(la + 2u * k));
+                    status = feed_class<PACKED, COMB>(A, sv, nd, top, below, S.cap, lds_u16(la + 2u * k));
             } else {
                 // one byte (as its byte class) through the lexer DFA; a completed lexeme
                 // goes to the parser
@@ -1417,7 +1527,7 @@ __global__ void __launch_bounds__(ADV_WARPS * 32) k_advance_warp(DevTables T, De
                         status = ROW_REJECTED;
                         return;
                     }
-                    if (!lds_u8(A.ign + cls)) status = feed_class_win<PACKED>(A, sv, nd, top, below, S.cap, cls);
+                    if (!lds_u8(A.ign + cls)) status = feed_class<PACKED, COMB>(A, sv, nd, top, below, S.cap, cls);
                     nq = lds_s16(A.trans + A.q0 * A.trans_row + 2u * c);
                     if (nq < 0) status = ROW_REJECTED;
                 };
@@ -1889,6 +1999,12 @@ psc_status launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t sm
 // Algorithm 2 steps 1-2 for every row (the token given, or the fused pass's greedy
 // choice when d_tokens_out is set), then step 3 for the new configurations: the
 // rows' mask ids are current afterwards.
+using AdvanceKernel = void (*)(DevTables, DevStates, const int32_t*, int, int, int32_t*, int, int32_t*, int);
+AdvanceKernel advance_kernel(const DevTables& d) {
+    if (d.adv_comb) return d.adv_packed ? k_advance_warp<true, true> : k_advance_warp<false, true>;
+    return d.adv_packed ? k_advance_warp<true, false> : k_advance_warp<false, false>;
+}
+
 psc_status launch_advance(const psc_handle* h, psc_states* st, const int32_t* d_tokens, int use_mid,
                           int32_t* d_row_status, int32_t* d_tokens_out, cudaStream_t cs) {
     int B = st->d.B;
@@ -1897,7 +2013,7 @@ psc_status launch_advance(const psc_handle* h, psc_states* st, const int32_t* d_
     st->after_mask = false;
     psc_status s;
     if (h->d.adv_bytes > 0) {
-        s = launch_pdl(h->d.adv_packed ? k_advance_warp<true> : k_advance_warp<false>,
+        s = launch_pdl(advance_kernel(h->d),
                        dim3((B + ADV_WARPS - 1) / ADV_WARPS), dim3(ADV_WARPS * 32), adv_smem(h->d), cs,
                        "k_advance_warp", h->d, st->d, d_tokens, B, use_mid, d_row_status, from_keys, d_tokens_out,
                        early);
@@ -1992,9 +2108,64 @@ int host_feed(const psc::Tables& T, uint16_t* st, int& depth, int cap, int cls) 
 namespace {
 // Compact int16 lexer/parser tables for k_advance_warp, or an empty blob when
 // the grammar is too large for shared memory (k_advance then reads global memory).
-std::vector<uint8_t> build_advance_blob(const psc::Tables& t, DevTables& d) {
+// Candidate terminals of each lexeme class in an order such that, in every parser
+// state s, the first candidate with an action in s is resolve[c][s] (or, where
+// resolve gives -1 or a terminal without an action, none has one): resolution by
+// trying the candidates in turn then picks what the resolve table picks.  Empty
+// when no such order exists.
+std::vector<std::vector<int>> class_candidates(const psc::Tables& t) {
+    const int ncls = t.n_classes, n = t.n_lr;
+    auto has = [&](int s, int x) { return psc::act_kind(t.action[(size_t)s * t.n_terms + x]) != psc::ACT_ERR; };
+    std::vector<std::vector<int>> out(ncls);
+    for (int c = 0; c < ncls; c++) {
+        std::vector<int> L;
+        for (int s = 0; s < n; s++) {
+            int r = t.resolve[(size_t)c * n + s];
+            if (r >= 0 && std::find(L.begin(), L.end(), r) == L.end()) L.push_back(r);
+        }
+        std::sort(L.begin(), L.end());
+        const int m = (int)L.size();
+        // r must come before x wherever resolve picks r while x has an action too
+        std::vector<std::vector<char>> before(m, std::vector<char>(m, 0));
+        for (int s = 0; s < n; s++) {
+            int r = t.resolve[(size_t)c * n + s];
+            if (r < 0) continue;
+            int i = (int)(std::find(L.begin(), L.end(), r) - L.begin());
+            for (int j = 0; j < m; j++)
+                if (j != i && has(s, L[j])) before[i][j] = 1;
+        }
+        std::vector<char> done(m, 0);
+        for (int k = 0; k < m; k++) {
+            int pick = -1;
+            for (int i = 0; i < m && pick < 0; i++) {
+                if (done[i]) continue;
+                bool free = true;
+                for (int j = 0; j < m && free; j++) free = done[j] || j == i || !before[j][i];
+                if (free) pick = i;
+            }
+            if (pick < 0) return {};   // a cycle: no order reproduces the table
+            done[pick] = 1;
+            out[c].push_back(L[pick]);
+        }
+        for (int s = 0; s < n; s++) {
+            int r = t.resolve[(size_t)c * n + s], f = -1;
+            for (int x : out[c])
+                if (has(s, x)) {
+                    f = x;
+                    break;
+                }
+            if (!(r == f || (f < 0 && (r < 0 || !has(s, r))))) return {};
+        }
+    }
+    return out;
+}
+
+// layout: 0 = the dense compact tables when they fit in shared memory, else the packed
+// ones when those fit; 2 = the packed tables whenever they fit.
+std::vector<uint8_t> build_advance_blob(const psc::Tables& t, DevTables& d, int layout) {
     std::vector<uint8_t> blob;
     d.adv_bytes = 0;
+    d.adv_comb = 0;
     int n_rules = (int)t.rule_len.size();
     if (t.n_lr >= 8192 || n_rules >= 8192 || t.nq >= 32768 || t.n_terms >= 32768) return blob;
     for (int L : t.rule_len)
@@ -2029,7 +2200,160 @@ std::vector<uint8_t> build_advance_blob(const psc::Tables& t, DevTables& d) {
     d.o_go = take((size_t)t.n_lr * t.n_nts * 2);
     d.o_rlen = take((size_t)n_rules);
     d.o_rlhs = take((size_t)n_rules * 2);
-    if (off > 200 * 1024) return blob;
+    if (getenv("PSC_LOG"))
+        fprintf(stderr, "psc: advance tables %zu B (lexer %d x %d classes, resolve %d x %d, action %d x %d, goto %d x %d)%s\n",
+                off, t.nq, nbc, ncls, t.n_lr, t.n_lr, t.n_terms, t.n_lr, t.n_nts,
+                off > ADV_TABLE_MAX ? ": too large for shared memory" : "");
+    int max_len = 0;
+    for (int L : t.rule_len) max_len = std::max(max_len, L);
+    d.adv_packed = (max_len < 16 && t.n_nts <= 1024) ? 1 : 0;
+    auto enc_action = [&](int32_t a) {
+        int kind = psc::act_kind(a), val = psc::act_val(a);
+        if (d.adv_packed && kind == psc::ACT_REDUCE) val = (t.rule_len[val] << 10) | t.rule_lhs[val];
+        return (int16_t)(((val & 0x3FFF) << 2) | kind);
+    };
+    if (layout == 2 || off > ADV_TABLE_MAX) {
+        // ---- packed layout: the lexer as above, then candidates, bases, the packed entries
+        std::vector<std::vector<int>> cands = class_candidates(t);
+        if (cands.empty() && ncls > 0) return blob;
+        int kc = 1;
+        for (auto& L : cands) kc = std::max(kc, (int)L.size());
+        if (kc > 16) return blob;
+        const int n = t.n_lr;
+        // one packed table each for ACTION and GOTO: equal rows are stored once, rows are
+        // placed first fit (fullest first) at the lowest base where all their entries land
+        // on free slots; an entry records its row's id, so a lookup in another row misses.
+        // Per state one word (row id << 17 | base).
+        struct Packed {
+            std::vector<uint32_t> slots;
+            std::vector<uint32_t> word;   // per state
+            int entries = 0;
+        };
+        auto pack = [&](int ncol, auto&& entry) -> Packed {   // entry(s, x, &v): has (s, x) an entry
+            Packed P;
+            std::vector<std::vector<std::pair<int, int16_t>>> rows;
+            std::map<std::vector<std::pair<int, int16_t>>, int> ids;
+            std::vector<int> rid(n);
+            for (int s = 0; s < n; s++) {
+                std::vector<std::pair<int, int16_t>> r;
+                for (int x = 0; x < ncol; x++) {
+                    int16_t v;
+                    if (entry(s, x, &v)) r.push_back({x, v});
+                }
+                auto it = ids.find(r);
+                if (it == ids.end()) {
+                    it = ids.emplace(r, (int)rows.size()).first;
+                    rows.push_back(r);
+                }
+                rid[s] = it->second;
+            }
+            const int nr = (int)rows.size();
+            std::vector<int> order(nr), base(nr, 0);
+            for (int r = 0; r < nr; r++) order[r] = r;
+            std::stable_sort(order.begin(), order.end(), [&](int a, int b) { return rows[a].size() > rows[b].size(); });
+            std::vector<char> used;
+            int len = ncol, first_free = 0;
+            for (int r : order) {
+                if (rows[r].empty()) continue;
+                int lo = rows[r].front().first;
+                for (int b = std::max(0, first_free - lo);; b++) {
+                    if ((size_t)b + ncol > used.size()) used.resize((size_t)b + ncol + 4096, 0);
+                    bool ok = true;
+                    for (auto& e : rows[r])
+                        if (used[b + e.first]) {
+                            ok = false;
+                            break;
+                        }
+                    if (!ok) continue;
+                    for (auto& e : rows[r]) used[b + e.first] = 1;
+                    base[r] = b;
+                    len = std::max(len, b + ncol);
+                    break;
+                }
+                while (first_free < (int)used.size() && used[first_free]) first_free++;
+            }
+            P.slots.assign((size_t)len, 0xFFFFFFFFu);
+            for (int r = 0; r < nr; r++)
+                for (auto& e : rows[r]) {
+                    P.slots[(size_t)base[r] + e.first] = ((uint32_t)r << 16) | (uint16_t)e.second;
+                    P.entries++;
+                }
+            if (nr >= (1 << 15) || len >= (1 << 17)) P.slots.clear();   // the state word cannot hold them
+            P.word.resize(n);
+            for (int s = 0; s < n; s++) P.word[s] = ((uint32_t)rid[s] << 17) | (uint32_t)base[rid[s]];
+            return P;
+        };
+        Packed PA = pack(t.n_terms, [&](int s, int x, int16_t* v) {
+            int32_t a = t.action[(size_t)s * t.n_terms + x];
+            if (psc::act_kind(a) == psc::ACT_ERR) return false;
+            *v = enc_action(a);
+            return true;
+        });
+        Packed PG = pack(t.n_nts, [&](int s, int x, int16_t* v) {
+            int32_t g = t.go[(size_t)s * t.n_nts + x];
+            if (g < 0) return false;
+            *v = (int16_t)g;
+            return true;
+        });
+        if (PA.slots.empty() || PG.slots.empty()) return blob;
+        // every lookup of the packed tables against the dense ones
+        auto look = [](const Packed& P, int s, int x, int miss) {
+            uint32_t w = P.word[s], e = P.slots[(size_t)(w & 0x1FFFFu) + x];
+            return (e >> 16) == (w >> 17) ? (int)(int16_t)(e & 0xFFFFu) : miss;
+        };
+        for (int s = 0; s < n; s++) {
+            for (int x = 0; x < t.n_terms; x++) {
+                int32_t a = t.action[(size_t)s * t.n_terms + x];
+                if (look(PA, s, x, 0) != (psc::act_kind(a) == psc::ACT_ERR ? 0 : (int)enc_action(a))) return blob;
+            }
+            for (int x = 0; x < t.n_nts; x++) {
+                int32_t g = t.go[(size_t)s * t.n_nts + x];
+                if (look(PG, s, x, -1) != (g >= 0 ? g : -1)) return blob;
+            }
+        }
+        off = (size_t)d.o_resolve;   // the lexer parts stay where they are
+        d.o_cand = take((size_t)std::max(ncls, 1) * kc * 2);
+        d.o_abase = take((size_t)n * 4);
+        d.o_gbase = take((size_t)n * 4);
+        d.o_acmb = take(PA.slots.size() * 4);
+        d.o_gcmb = take(PG.slots.size() * 4);
+        d.o_rlen = take((size_t)n_rules);
+        d.o_rlhs = take((size_t)n_rules * 2);
+        d.o_resolve = d.o_action = d.o_go = 0;
+        if (getenv("PSC_LOG"))
+            fprintf(stderr, "psc: packed advance tables %zu B (ACTION %d entries in %zu slots, GOTO %d in %zu, "
+                            "%d candidates per class)%s\n",
+                    off, PA.entries, PA.slots.size(), PG.entries, PG.slots.size(), kc,
+                    off > ADV_TABLE_MAX ? ": too large for shared memory" : "");
+        if (off > ADV_TABLE_MAX) return blob;
+        blob.assign(off, 0);
+        for (int b = 0; b < 256; b++) blob[d.o_bc + b] = (uint8_t)bc[b];
+        for (int q = 0; q < t.nq; q++) {
+            for (int b = 0; b < 256; b++)
+                reinterpret_cast<int16_t*>(blob.data() + d.o_trans)[(size_t)q * nbc + bc[b]] =
+                    (int16_t)t.lex_trans[(size_t)q * 256 + b];
+            reinterpret_cast<int16_t*>(blob.data() + d.o_accept)[q] = (int16_t)t.lex_accept[q];
+        }
+        for (int c = 0; c < ncls; c++) {
+            blob[d.o_ign + c] = t.cls_ignored[c];
+            for (int k = 0; k < kc; k++)
+                reinterpret_cast<int16_t*>(blob.data() + d.o_cand)[(size_t)c * kc + k] =
+                    (int16_t)(k < (int)cands[c].size() ? cands[c][k] : -1);
+        }
+        std::memcpy(blob.data() + d.o_abase, PA.word.data(), (size_t)n * 4);
+        std::memcpy(blob.data() + d.o_gbase, PG.word.data(), (size_t)n * 4);
+        std::memcpy(blob.data() + d.o_acmb, PA.slots.data(), PA.slots.size() * 4);
+        std::memcpy(blob.data() + d.o_gcmb, PG.slots.data(), PG.slots.size() * 4);
+        for (int r = 0; r < n_rules; r++) {
+            blob[d.o_rlen + r] = (uint8_t)t.rule_len[r];
+            reinterpret_cast<int16_t*>(blob.data() + d.o_rlhs)[r] = (int16_t)t.rule_lhs[r];
+        }
+        d.kc = kc;
+        d.nbc = nbc;
+        d.adv_comb = 1;
+        d.adv_bytes = (int)off;
+        return blob;
+    }
     blob.assign(off, 0);
     auto put16 = [&](int o, size_t i, int v) { reinterpret_cast<int16_t*>(blob.data() + o)[i] = (int16_t)v; };
     for (int b = 0; b < 256; b++) blob[d.o_bc + b] = (uint8_t)bc[b];
@@ -2043,15 +2367,7 @@ std::vector<uint8_t> build_advance_blob(const psc::Tables& t, DevTables& d) {
     }
     // a reduce entry carries its rule's length and left-hand side when they fit in 14 bits
     // (one dependent shared-memory read less per reduction)
-    int max_len = 0;
-    for (int L : t.rule_len) max_len = std::max(max_len, L);
-    d.adv_packed = (max_len < 16 && t.n_nts <= 1024) ? 1 : 0;
-    for (size_t i = 0; i < t.action.size(); i++) {
-        int32_t a = t.action[i];
-        int kind = psc::act_kind(a), val = psc::act_val(a);
-        if (d.adv_packed && kind == psc::ACT_REDUCE) val = (t.rule_len[val] << 10) | t.rule_lhs[val];
-        put16(d.o_action, i, ((val & 0x3FFF) << 2) | kind);
-    }
+    for (size_t i = 0; i < t.action.size(); i++) put16(d.o_action, i, enc_action(t.action[i]));
     for (size_t i = 0; i < t.go.size(); i++) put16(d.o_go, i, t.go[i]);
     for (int r = 0; r < n_rules; r++) {
         blob[d.o_rlen + r] = (uint8_t)t.rule_len[r];
@@ -2100,7 +2416,9 @@ std::vector<uint8_t> token_prefixes(const psc::Tables& t) {
 }
 
 // Uploads a handle's host tables to the current device (psc_compile, psc_load).
-psc_status upload_tables(std::unique_ptr<psc_handle>& h, bool global_tables) {
+// tables: 0 = staged (dense compact tables when they fit, else packed ones), 1 = global
+// memory, 2 = staged packed tables.
+psc_status upload_tables(std::unique_ptr<psc_handle>& h, int tables) {
     const psc::Tables& t = h->t;
     psc_status s = cuda_check(cudaGetDevice(&h->device), "cudaGetDevice");
     if (s != PSC_OK) return s;
@@ -2159,7 +2477,8 @@ psc_status upload_tables(std::unique_ptr<psc_handle>& h, bool global_tables) {
         d.n_frow = t.n_frow;
     }
     std::vector<uint8_t> blob;
-    if (!global_tables) blob = build_advance_blob(t, d);
+    d.adv_bytes = d.adv_comb = 0;
+    if (tables != 1) blob = build_advance_blob(t, d, tables);
     if (!blob.empty()) {
         if ((s = upload(h.get(), blob, &d.adv)) != PSC_OK) {
             for (int i = 0; i < h->n_blocks; i++) cudaFree(h->blocks[i]);
@@ -2170,7 +2489,7 @@ psc_status upload_tables(std::unique_ptr<psc_handle>& h, bool global_tables) {
         int optin = 0;
         cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, h->device);
         cudaFuncAttributes fa{};
-        auto kadv = d.adv_packed ? k_advance_warp<true> : k_advance_warp<false>;
+        auto kadv = advance_kernel(d);
         cudaFuncGetAttributes(&fa, kadv);
         optin -= (int)fa.sharedSizeBytes;   // the limit covers dynamic memory only
         if (optin < adv_smem(d)) {
@@ -2231,7 +2550,8 @@ psc_status psc_compile(const char* grammar, size_t grammar_len, const uint8_t* v
     for (int v = 0; v < V; v++)
         if (vocab_offsets[v + 1] < vocab_offsets[v]) return fail_with(PSC_ERR_ARG, "psc_compile: offsets decrease");
     psc::Options o;
-    bool host_only = false, global_tables = false;
+    bool host_only = false;
+    int tables = 0;
     if (opts) {
         if (opts->max_states > 0) o.max_states = opts->max_states;
         if (opts->max_mask_bytes > 0) o.max_mask_bytes = opts->max_mask_bytes;
@@ -2239,7 +2559,8 @@ psc_status psc_compile(const char* grammar, size_t grammar_len, const uint8_t* v
         o.max_bottom_up_bytes = opts->max_bottom_up_bytes;
         o.max_dense_classifier_bytes = opts->max_dense_classifier_bytes;
         host_only = opts->host_only != 0;
-        global_tables = opts->global_tables != 0;
+        tables = opts->global_tables;
+        if (tables < 0 || tables > 2) return fail_with(PSC_ERR_ARG, "psc_compile: global_tables must be 0, 1 or 2");
     }
     std::unique_ptr<psc_handle> h(new (std::nothrow) psc_handle());
     if (!h) return fail_with(PSC_ERR_OOM, "psc_compile: out of host memory");
@@ -2251,8 +2572,9 @@ psc_status psc_compile(const char* grammar, size_t grammar_len, const uint8_t* v
         return fail_with(PSC_ERR_OOM, "psc_compile: out of host memory");
     }
     h->host_only = host_only;
+    h->tables = tables;
     if (!host_only) {
-        psc_status s = upload_tables(h, global_tables);
+        psc_status s = upload_tables(h, tables);
         if (s != PSC_OK) return s;
     }
     *out = h.release();
@@ -2282,7 +2604,15 @@ psc_status psc_info(const psc_handle* h, psc_info_t* out) {
     out->mask_bytes = (int64_t)(t.mask_rows.size() + t.mask_chunks.size()) * 4;
     out->states_built = t.n_dfa_states_built;
     out->compile_seconds = t.seconds_total;
-    out->advance_table_bytes = h->host_only ? 0 : h->d.adv_bytes;
+    if (h->host_only) {   // what a device upload with the handle's placement would stage
+        DevTables tmp{};
+        if (h->tables != 1) build_advance_blob(t, tmp, h->tables);
+        out->advance_table_bytes = tmp.adv_bytes;
+        out->advance_tables_packed = tmp.adv_bytes > 0 && tmp.adv_comb;
+    } else {
+        out->advance_table_bytes = h->d.adv_bytes;
+        out->advance_tables_packed = h->d.adv_bytes > 0 && h->d.adv_comb;
+    }
     out->bottom_up_states = t.n_bu;
     out->bottom_up_bytes = (int64_t)(t.bu.size() + t.bu_F.size()) * 4 + (int64_t)t.bu_slot.size() * 2;
     out->device_timeouts = 0;
@@ -2696,8 +3026,10 @@ psc_status psc_load(const char* path, const psc_options* opts, psc_handle** out)
         t.n_bu = t.n_frow = 0;
     }
     h->host_only = opts && opts->host_only;
+    h->tables = opts ? opts->global_tables : 0;
+    if (h->tables < 0 || h->tables > 2) return fail_with(PSC_ERR_ARG, "psc_load: global_tables must be 0, 1 or 2");
     if (!h->host_only) {
-        psc_status s = upload_tables(h, opts && opts->global_tables);
+        psc_status s = upload_tables(h, h->tables);
         if (s != PSC_OK) return s;
     }
     *out = h.release();

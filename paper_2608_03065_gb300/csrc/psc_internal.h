@@ -87,7 +87,8 @@ struct Options {
     int64_t max_mask_bytes = int64_t(24) << 30;
     int threads = 0;                  // 0 = hardware concurrency
     int64_t max_bottom_up_bytes = 0;  // construction memory of the bottom-up classifier
-                                      // (0 = 8 GiB; < 0 = not built; over the limit: not built)
+                                      // (0 = 16 GiB, at most half the memory; < 0 = not built;
+                                      // over the limit: not built)
     int64_t max_dense_classifier_bytes = 0;  // dense classifier table above this: sparse layout
                                              // (0 = 512 MiB; < 0 = always sparse)
 };

@@ -52,7 +52,7 @@ class InfoT(ctypes.Structure):
                 ("states_built", ctypes.c_int64), ("compile_seconds", ctypes.c_double),
                 ("advance_table_bytes", ctypes.c_int64), ("device_timeouts", ctypes.c_int64),
                 ("bottom_up_states", ctypes.c_int64), ("bottom_up_bytes", ctypes.c_int64),
-                ("classifier_sparse", ctypes.c_int64)]
+                ("classifier_sparse", ctypes.c_int64), ("advance_tables_packed", ctypes.c_int64)]
 
 
 _lib = None
@@ -166,6 +166,7 @@ class Info:
     bottom_up_states: int
     bottom_up_bytes: int
     classifier_sparse: int
+    advance_tables_packed: int
 
 
 class Handle:
@@ -234,13 +235,21 @@ class States:
 
 
 # ------------------------------------------------------------------- the ABI
+def _tables(global_tables: bool, packed_tables: bool) -> int:
+    if global_tables and packed_tables:
+        raise ValueError("global_tables and packed_tables exclude each other")
+    return 1 if global_tables else 2 if packed_tables else 0
+
+
 def psc_compile(grammar: str, vocab: list[bytes] | tuple, eos_id: int, host_only: bool = False,
                 threads: int = 0, max_states: int = 0, max_mask_bytes: int = 0,
                 global_tables: bool = False, bottom_up: bool = True, max_bottom_up_bytes: int = 0,
-                max_dense_classifier_bytes: int = 0) -> Handle:
+                max_dense_classifier_bytes: int = 0, packed_tables: bool = False) -> Handle:
     """vocab: list of token byte strings, or (blob uint8 array, offsets int64[V+1]).
     bottom_up=False builds no bottom-up classifier (every stack is walked from the top);
-    max_dense_classifier_bytes < 0 holds the classifier in the sparse layout."""
+    max_dense_classifier_bytes < 0 holds the classifier in the sparse layout;
+    global_tables=True has the advance read its parser tables from global memory,
+    packed_tables=True stages them in the packed layout even when the dense one fits."""
     if isinstance(vocab, tuple):
         blob, offs = vocab
         blob = np.ascontiguousarray(blob, dtype=np.uint8)
@@ -252,7 +261,7 @@ def psc_compile(grammar: str, vocab: list[bytes] | tuple, eos_id: int, host_only
     if blob.size == 0:
         blob = np.zeros(1, dtype=np.uint8)
     V = len(offs) - 1
-    opts = Options(max_states, max_mask_bytes, threads, 1 if host_only else 0, 1 if global_tables else 0,
+    opts = Options(max_states, max_mask_bytes, threads, 1 if host_only else 0, _tables(global_tables, packed_tables),
                    max_bottom_up_bytes if bottom_up else -1, max_dense_classifier_bytes)
     g = grammar.encode("utf-8")
     out = ctypes.c_void_p()
@@ -265,8 +274,9 @@ def psc_save(h: Handle, path: str):
     _check(load().psc_save(h.ptr, os.fsencode(path)))
 
 
-def psc_load(path: str, host_only: bool = False, global_tables: bool = False, bottom_up: bool = True) -> Handle:
-    opts = Options(0, 0, 0, 1 if host_only else 0, 1 if global_tables else 0, 0 if bottom_up else -1, 0)
+def psc_load(path: str, host_only: bool = False, global_tables: bool = False, bottom_up: bool = True,
+             packed_tables: bool = False) -> Handle:
+    opts = Options(0, 0, 0, 1 if host_only else 0, _tables(global_tables, packed_tables), 0 if bottom_up else -1, 0)
     out = ctypes.c_void_p()
     _check(load().psc_load(os.fsencode(path), ctypes.byref(opts), ctypes.byref(out)))
     h = Handle(out.value, 0)

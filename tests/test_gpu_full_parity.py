@@ -8,13 +8,15 @@ the CPU oracle.
 * C-like grammar, 262,144 tokens, 1024 rows, at the prefix states: the masks
   and masked logits of psc_fill_apply and of the decode masking pass, all rows
   over all tokens, and the greedy tokens of all rows.
-* The Java-sized grammar (1,001 LALR(1) states; classifier held sparse, parser
-  tables too large for shared memory, so the advance reads them from global
-  memory), 4,096 tokens, 64 rows: all rows over all tokens at the prefix states
-  and through six whole decode steps.
-* The same grammar with a pre-tokenized vocabulary of 262,144 tokens, 256 rows:
-  all rows over all tokens at the prefix states (fused masking pass with the
-  greedy choice) and through four whole decode steps.
+* The Java-sized grammar (1,001 LALR(1) states; classifier held sparse and
+  walked from the top; parser tables packed to fit shared memory), 4,096 tokens,
+  64 rows: all rows over all tokens at the prefix states and through six whole
+  decode steps; then three more from the prefix states with the same tables read
+  from global memory.
+* The same grammar with a pre-tokenized vocabulary of 262,144 tokens, 256 rows,
+  default options (bottom-up classifier too): all rows over all tokens at the
+  prefix states (fused masking pass with the greedy choice) and through four
+  whole decode steps.
 * The C-like 262,144-token workload on the benchmark's exact path: the batch restored from a
   saved copy (psc_state_copy), then 32 steps of psc_decode_step_mask +
   psc_decode_step_advance on fresh logits; the oracle is advanced by the same
@@ -61,12 +63,7 @@ class Big:
 
     def __init__(self, psc, cfg_id, **opts):
         self.w = w = configs.load(cfg_id)
-        self.h = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id, **opts)
-        self.snap = psc.psc_state_init(self.h, w.B, CAP)
-        tm = torch.from_numpy(w.token_matrix()).cuda()
-        for j in range(tm.shape[1]):
-            psc.psc_advance(self.h, self.snap, tm[:, j].contiguous())
-        torch.cuda.synchronize()
+        self._prefix_states(psc, psc.psc_compile(w.grammar_text, w.vocab, w.eos_id, **opts))
         self.o = Oracle(w.grammar_text)
         self.voc = Vocab.from_list(w.vocab, w.eos_id)
         self.ocs0 = []
@@ -74,6 +71,23 @@ class Big:
             oc = self.o.initial()
             self.o.advance_tokens(oc, self.voc, ids)
             self.ocs0.append(oc)
+
+    def _prefix_states(self, psc, h):
+        self.h = h
+        self.snap = psc.psc_state_init(h, self.w.B, CAP)
+        tm = torch.from_numpy(self.w.token_matrix()).cuda()
+        for j in range(tm.shape[1]):
+            psc.psc_advance(h, self.snap, tm[:, j].contiguous())
+        torch.cuda.synchronize()
+
+    def reloaded(self, psc, path, **opts):
+        """The same workload on the tables saved and loaded back with other
+        placement options (prefix states rebuilt on the new handle)."""
+        psc.psc_save(self.h, path)
+        other = object.__new__(Big)
+        other.w, other.o, other.voc, other.ocs0 = self.w, self.o, self.voc, self.ocs0
+        other._prefix_states(psc, psc.psc_load(path, **opts))
+        return other
 
     def restored(self, psc):
         """A fresh states object restored from the saved prefix states, and
@@ -135,24 +149,31 @@ def test_c_like_151936_whole_decode_all_rows_all_tokens(psc):
     whole_decode_all_rows_all_tokens(psc, big(psc, 4), 4, 4000)
 
 
-def test_java_sized_grammar_whole_decode_all_rows_all_tokens(psc):
+def test_java_sized_grammar_whole_decode_all_rows_all_tokens(psc, tmp_path):
+    """Packed parser tables staged in shared memory (the default for this
+    grammar), then the same tables read from global memory (k_advance +
+    k_classify); the classifier sparse and walked from the top."""
     b = big(psc, 6, bottom_up=False, **configs.COMPILE_LIMITS[6])
     info = b.h.info()
-    assert info.n_parser_states >= 1000 and info.classifier_sparse == 1 and info.advance_table_bytes == 0
+    assert info.n_parser_states >= 1000 and info.classifier_sparse == 1
+    assert info.advance_tables_packed == 1 and info.advance_table_bytes > 0
     whole_decode_all_rows_all_tokens(psc, b, 6, 7000)
+    bg = b.reloaded(psc, str(tmp_path / "java.psc"), global_tables=True, bottom_up=False)
+    assert bg.h.info().advance_table_bytes == 0
+    whole_decode_all_rows_all_tokens(psc, bg, 3, 7100)
 
 
 def test_java_sized_grammar_262144_pretokenized_all_rows_all_tokens(psc):
     """The Java-sized grammar at the paper's largest vocabulary size, with a
-    pre-tokenized vocabulary: the fused masking pass at the prefix states, then
-    four whole decode steps, every row over every token.  (The bottom-up
-    classifier is left out: on this grammar it passes its memory budget, and the
-    device walks the stacks from the top, which is what the default compile
-    falls back to.)"""
-    b = big(psc, 7, bottom_up=False, **configs.COMPILE_LIMITS[7])
+    pre-tokenized vocabulary, compiled with the default options (sparse
+    classifier, bottom-up classifier, packed parser tables staged in shared
+    memory): the fused masking pass at the prefix states, then four whole decode
+    steps, every row over every token."""
+    b = big(psc, 7, **configs.COMPILE_LIMITS[7])
     w = b.w
     info = b.h.info()
-    assert info.n_parser_states >= 1000 and info.classifier_sparse == 1 and info.advance_table_bytes == 0
+    assert info.n_parser_states >= 1000 and info.classifier_sparse == 1 and info.bottom_up_states > 0
+    assert info.advance_tables_packed == 1
     assert w.V == 262144 and w.B == 256
     ref = b.o.masks(b.ocs0, b.voc, threads=THREADS)
     st, _ = b.restored(psc)

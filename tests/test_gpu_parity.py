@@ -34,10 +34,11 @@ class Case:
     """A workload compiled on the device, with device states and oracle configs
     advanced over the same prefix tokens."""
 
-    def __init__(self, psc, cfg_id, cap=256, global_tables=False):
+    def __init__(self, psc, cfg_id, cap=256, global_tables=False, packed_tables=False):
         self.w = configs.load(cfg_id)
         w = self.w
-        self.h = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id, global_tables=global_tables)
+        self.h = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id, global_tables=global_tables,
+                                 packed_tables=packed_tables)
         self.st = psc.psc_state_init(self.h, w.B, cap)
         tm = torch.from_numpy(w.token_matrix()).cuda()
         for j in range(tm.shape[1]):
@@ -213,12 +214,13 @@ def test_decode_loop_advance(psc, cfg_id, steps, mode):
     _decode_loop(psc, case(psc, cfg_id), steps, mode)
 
 
-@pytest.mark.parametrize("global_tables", [False, True])
-def test_decode_loop_table_paths(psc, global_tables):
-    """The advance kernel with its tables staged in shared memory and read from
-    global memory give the same states (JSON, whole decode steps)."""
-    c = Case(psc, 2, global_tables=global_tables)
-    assert (c.h.info().advance_table_bytes > 0) == (not global_tables)
+@pytest.mark.parametrize("tables", ["global", "packed"])
+def test_decode_loop_table_paths(psc, tables):
+    """The advance kernel with its tables read from global memory, or staged in
+    the packed layout, decodes as the oracle says (JSON, whole decode steps)."""
+    c = Case(psc, 2, global_tables=tables == "global", packed_tables=tables == "packed")
+    assert (c.h.info().advance_table_bytes > 0) == (tables == "packed")
+    assert c.h.info().advance_tables_packed == (tables == "packed")
     _decode_loop(psc, c, 5, "step")
 
 
@@ -455,8 +457,8 @@ def test_nan_payloads_and_infinities_kept(psc):
         np.testing.assert_array_equal(got, want)
 
 
-@pytest.mark.parametrize("global_tables", [False, True])
-def test_deep_stacks_and_long_pushes(psc, global_tables):
+@pytest.mark.parametrize("tables", ["staged", "global", "packed"])
+def test_deep_stacks_and_long_pushes(psc, tables):
     """Balanced parentheses with tokens of up to 32 brackets: stacks grow to
     thousands of entries, past the advance kernel's shared-memory window (192
     entries copied in, 256 held), pushes of one token run beyond the window into
@@ -465,7 +467,7 @@ def test_deep_stacks_and_long_pushes(psc, global_tables):
     g = 'start: s\ns: | s "(" s ")"\n'
     toks = [b"(" * n for n in (1, 2, 7, 16, 31, 32)] + [b")" * n for n in (1, 3, 16, 32)] + [b"()", b")(", b""]
     eos = len(toks) - 1
-    h = psc.psc_compile(g, toks, eos, global_tables=global_tables)
+    h = psc.psc_compile(g, toks, eos, global_tables=tables == "global", packed_tables=tables == "packed")
     o = Oracle(g)
     voc = Vocab.from_list(toks, eos)
     B, cap = 6, 8192

@@ -7,8 +7,9 @@ device by psc_advance with tokens drawn from the oracle's masks (so rows walk
 through the configurations the grammar reaches), and after every step:
 psc_fill_mask equals the oracle's masks, psc_fill_apply masks seeded logits
 exactly as the oracle's masks say (with the bitmask copy), and the statuses
-psc_advance reports equal the oracle's.  Both advance table paths (staged
-shared-memory tables and global tables) run.
+psc_advance reports equal the oracle's.  Every advance table path runs: dense
+tables staged in shared memory, packed tables staged in shared memory, tables
+read from global memory.
 """
 from __future__ import annotations
 
@@ -39,9 +40,9 @@ def _masked(raw, allowed):
     return out
 
 
-@pytest.mark.parametrize("global_tables", [False, True])
-def test_random_grammars_device_matches_the_oracle(psc, global_tables):
-    rng = np.random.default_rng(77 + global_tables)
+@pytest.mark.parametrize("tables", ["staged", "global", "packed"])
+def test_random_grammars_device_matches_the_oracle(psc, tables):
+    rng = np.random.default_rng({"staged": 77, "global": 78, "packed": 79}[tables])
     done, modes, configs_seen = 0, set(), 0
     while done < 40:
         text, vocab = random_grammar(rng, True), random_vocab(rng, True)
@@ -49,10 +50,13 @@ def test_random_grammars_device_matches_the_oracle(psc, global_tables):
             continue
         eos = len(vocab) - 1
         try:
-            h = psc.psc_compile(text, vocab, eos, global_tables=global_tables)
+            h = psc.psc_compile(text, vocab, eos, global_tables=tables == "global",
+                                packed_tables=tables == "packed")
         except psc.PscError as e:
             assert e.code == 3, (text, str(e))        # only LALR(1) conflicts are expected
             continue
+        assert (h.info().advance_table_bytes > 0) == (tables != "global")
+        assert h.info().advance_tables_packed == (tables == "packed")
         modes.add("contextual" if "%lexer contextual" in text else "basic")
         o = Oracle(text)
         voc = Vocab.from_list(vocab, eos)

@@ -572,3 +572,64 @@ def test_sparse_classifier_layout_classifies_like_the_dense_one(psc, cfg_id, tmp
             assert hs.host_classify_bottom_up(c["q"], c["stack"]) == want
             n += 1
     assert n > 50
+
+
+def test_packed_advance_tables(psc):
+    """The packed staged parser tables (ACTION and GOTO row-displaced, equal rows
+    stored once, lexeme classes resolved by trying candidate terminals in order)
+    are what the advance stages for the Java-sized grammar, whose dense compact
+    tables pass the shared-memory budget; the library builds them only after
+    every lookup of them equals the dense tables' entry and the candidate order
+    reproduces the class-resolution table in every parser state, so a packed
+    layout on the seeded random grammars (both lexer modes, classes with several
+    candidate terminals) means both checks passed.  A host_only handle reports
+    what a device upload would stage."""
+    from ._random_grammars import random_grammar, random_vocab
+    toks = configs.vocab_for(6, 300)
+    hj = psc.psc_compile(grammars.java_like().text(), toks, len(toks) - 1, host_only=True, bottom_up=False)
+    ij = hj.info()
+    assert ij.n_parser_states >= 1000 and ij.advance_tables_packed == 1
+    assert 0 < ij.advance_table_bytes <= 200 * 1024
+    w = configs.load(2, batch=4)
+    for kw, packed in (({}, 0), ({"packed_tables": True}, 1)):
+        i = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id, host_only=True, **kw).info()
+        assert i.advance_table_bytes > 0 and i.advance_tables_packed == packed
+    assert psc.psc_compile(w.grammar_text, w.vocab, w.eos_id, host_only=True,
+                           global_tables=True).info().advance_table_bytes == 0
+    with pytest.raises(ValueError):
+        psc.psc_compile(w.grammar_text, w.vocab, w.eos_id, host_only=True, global_tables=True, packed_tables=True)
+    rng = np.random.default_rng(5150)
+    modes, multi = set(), 0
+    done = 0
+    while done < 60:
+        text, vocab = random_grammar(rng, True), random_vocab(rng, True)
+        if text is None:
+            continue
+        try:
+            h = psc.psc_compile(text, vocab, len(vocab) - 1, host_only=True, packed_tables=True, bottom_up=False)
+        except psc.PscError as e:
+            assert e.code == 3
+            continue
+        i = h.info()
+        assert i.advance_tables_packed == 1 and i.advance_table_bytes > 0, text
+        modes.add("contextual" if "%lexer contextual" in text else "basic")
+        multi += "%lexer contextual" in text and re.search(r'"[a-z]+"', text) is not None
+        done += 1
+    assert modes == {"basic", "contextual"} and multi > 5
+
+
+def test_table_placement_values_are_checked(psc):
+    """psc_options.global_tables takes 0, 1 or 2; anything else is PSC_ERR_ARG."""
+    import ctypes
+    lib = psc.load()
+    g = b'start: "x"\n'
+    blob = (ctypes.c_uint8 * 1)(120)
+    offs = (ctypes.c_int64 * 3)(0, 1, 1)
+    out = ctypes.c_void_p()
+    for bad in (3, -1):
+        opts = psc.Options(0, 0, 0, 1, bad, 0, 0)
+        assert lib.psc_compile(g, len(g), blob, offs, 2, 1, ctypes.byref(opts), ctypes.byref(out)) == 1
+        assert b"global_tables" in lib.psc_last_error()
+    opts = psc.Options(0, 0, 0, 1, 2, 0, 0)
+    assert lib.psc_compile(g, len(g), blob, offs, 2, 1, ctypes.byref(opts), ctypes.byref(out)) == 0
+    lib.psc_destroy(out)
