@@ -581,8 +581,10 @@ def run_compile(args):
     implementation): each workload compiled in its own process on the host cores
     (compile time, peak RSS, classifier and mask sizes, saved file sizes); then,
     on the GPU, the decode step on the Java-sized tables at 4,096 and 262,144
-    tokens (sparse classifier, parser tables read from global memory, stacks
-    walked from the top) and on the 262,144-token C-like
+    tokens (sparse classifier, packed parser tables staged in shared memory; also
+    with the parser tables read from global memory, and at 262,144 tokens with
+    stacks walked from the top instead of the bottom-up classifier) and on the
+    262,144-token C-like
     tables with the advance's tables staged in shared memory or read from
     global memory."""
     jobs = [(2, None), (3, None), (4, None), (5, None), (6, 1024), (6, 2048), (6, 4096), (7, 131072), (7, None)]
@@ -604,19 +606,28 @@ def run_compile(args):
             from paper_2608_03065_gb300 import build, psc
             from workloads import configs
             build.build()
-            w6 = configs.load(6)
-            h6 = psc.psc_compile(w6.grammar_text, w6.vocab, w6.eos_id, bottom_up=False, **configs.COMPILE_LIMITS[6])
-            out["java_like_decode_step_us"] = {"batch": w6.B, "vocab": w6.V, "graph_us": graph_step_us(psc, h6, w6, w6.B),
-                                               "advance_table_bytes": h6.info().advance_table_bytes,
-                                               "classifier_sparse": h6.info().classifier_sparse}
-            del h6
-            w7 = configs.load(7)
-            h7 = psc.psc_compile(w7.grammar_text, w7.vocab, w7.eos_id, bottom_up=False, **configs.COMPILE_LIMITS[7])
-            out["java_like_pretok_262144_decode_step_us"] = {
-                "batch": w7.B, "vocab": w7.V, "graph_us": graph_step_us(psc, h7, w7, w7.B),
-                "advance_table_bytes": h7.info().advance_table_bytes,
-                "classifier_sparse": h7.info().classifier_sparse}
-            del h7
+            import tempfile
+            for cfg, key, opts in ((6, "java_like_decode_step_us", {"bottom_up": False}),
+                                   (7, "java_like_pretok_262144_decode_step_us", {})):
+                w = configs.load(cfg)
+                h = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id, **opts, **configs.COMPILE_LIMITS[cfg])
+                i = h.info()
+                rec = {"batch": w.B, "vocab": w.V, "classifier_sparse": i.classifier_sparse,
+                       "bottom_up_states": i.bottom_up_states, "advance_table_bytes": i.advance_table_bytes,
+                       "advance_tables_packed": i.advance_tables_packed,
+                       "graph_us": graph_step_us(psc, h, w, w.B)}
+                with tempfile.TemporaryDirectory() as d:
+                    path = os.path.join(d, "t.psc")
+                    psc.psc_save(h, path)
+                    del h
+                    hg = psc.psc_load(path, global_tables=True, bottom_up="bottom_up" not in opts)
+                    rec["graph_us_global_tables"] = graph_step_us(psc, hg, w, w.B)
+                    del hg
+                    if cfg == 7:
+                        ht = psc.psc_load(path, bottom_up=False)
+                        rec["graph_us_top_down"] = graph_step_us(psc, ht, w, w.B)
+                        del ht
+                out[key] = rec
             w5 = configs.load(5)
             for gt in (False, True):
                 h5 = psc.psc_compile(w5.grammar_text, w5.vocab, w5.eos_id, global_tables=gt)
@@ -640,8 +651,8 @@ def run_profile(args):
     build.build()
     w = configs.load(args.cfg)
     opts = dict(configs.COMPILE_LIMITS.get(args.cfg, {}))
-    if args.cfg in (6, 7):
-        opts["bottom_up"] = False   # over its construction budget on the Java-sized grammar
+    if args.cfg == 6:
+        opts["bottom_up"] = False   # over its construction budget on this grammar and vocabulary
     h = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id, **opts)
     st = psc.psc_state_init(h, w.B, 256)
     tm = torch.from_numpy(w.token_matrix()).cuda()
@@ -914,7 +925,7 @@ def main():
                      "algorithmic_bytes": alg_bytes, "peak_kind": peak_kind},
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": B * V * 2,
                 "d2h_bytes_per_step": B * 4},
-        "gpu_launches": 2 * K,
+        "gpu_launches": 2 * K + (K + SEQ - 1) // SEQ,   # two per step, one per restore (k_state_copy)
         "clocks": clocks.summary(),
         "cpu_baseline": cpu,
         "mask_paths": paths,

@@ -1015,6 +1015,29 @@ __device__ __forceinline__ uint64_t gmem_addr(const void* p) {
 __device__ __forceinline__ void grid_dep_launch() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 __device__ __forceinline__ void grid_dep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 
+// psc_state_copy: every array of one batch's states into another's in one launch,
+// once the previous kernel on the stream has completed (16-byte copies; a
+// segment's bytes past its last whole 16 one by one; every segment starts on an
+// allocation of its own, so 16-byte aligned).
+struct CopySegs {
+    const uint8_t* src[8];
+    uint8_t* dst[8];
+    unsigned long long bytes[8];
+    int n;
+};
+__global__ void k_state_copy(CopySegs c) {
+    grid_dep_wait();
+    grid_dep_launch();
+    const size_t tid = blockIdx.x * (size_t)blockDim.x + threadIdx.x, nt = (size_t)gridDim.x * blockDim.x;
+    for (int k = 0; k < c.n; k++) {
+        const size_t n16 = c.bytes[k] / 16;
+        const uint4* src = reinterpret_cast<const uint4*>(c.src[k]);
+        uint4* dst = reinterpret_cast<uint4*>(c.dst[k]);
+        for (size_t i = tid; i < n16; i += nt) dst[i] = src[i];
+        for (size_t i = n16 * 16 + tid; i < c.bytes[k]; i += nt) c.dst[k][i] = c.src[k][i];
+    }
+}
+
 // Bounded wait on phase 0 of an mbarrier; returns false if it did not complete.
 __device__ __forceinline__ bool mbar_wait0(uint32_t bar, int limit) {
     for (int it = 0; it < limit; it++) {
@@ -2683,24 +2706,24 @@ psc_status psc_state_copy(psc_states* dst, const psc_states* src, void* stream) 
     const DevStates& a = src->d;
     DevStates& b = dst->d;
     size_t B = (size_t)a.B;
-    psc_status s;
-    // one copy per array (no batched-copy call)
-    if ((s = cuda_check(cudaMemcpyAsync(b.q, a.q, B * 4, cudaMemcpyDeviceToDevice, cs), "psc_state_copy")) != PSC_OK ||
-        (s = cuda_check(cudaMemcpyAsync(b.depth, a.depth, B * 4, cudaMemcpyDeviceToDevice, cs), "psc_state_copy")) !=
-            PSC_OK ||
-        (s = cuda_check(cudaMemcpyAsync(b.status, a.status, B * 4, cudaMemcpyDeviceToDevice, cs), "psc_state_copy")) !=
-            PSC_OK ||
-        (s = cuda_check(cudaMemcpyAsync(b.stack, a.stack, B * (size_t)a.cap * 2, cudaMemcpyDeviceToDevice, cs),
-                        "psc_state_copy")) != PSC_OK ||
-        (s = cuda_check(cudaMemcpyAsync(b.mid, a.mid, B * 4, cudaMemcpyDeviceToDevice, cs), "psc_state_copy")) !=
-            PSC_OK ||
-        (s = cuda_check(cudaMemcpyAsync(b.best, a.best, B * 8, cudaMemcpyDeviceToDevice, cs), "psc_state_copy")) !=
-            PSC_OK)
-        return s;
-    if (a.rmemo && b.rmemo &&
-        (s = cuda_check(cudaMemcpyAsync(b.rmemo, a.rmemo, B * (size_t)a.cap * 4, cudaMemcpyDeviceToDevice, cs),
-                        "psc_state_copy")) != PSC_OK)
-        return s;
+    // one kernel for all the arrays (a copy per array costs a stream round trip each)
+    CopySegs c{};
+    auto add = [&](const void* src, void* dst, size_t bytes) {
+        c.src[c.n] = static_cast<const uint8_t*>(src);
+        c.dst[c.n] = static_cast<uint8_t*>(dst);
+        c.bytes[c.n++] = bytes;
+    };
+    add(a.q, b.q, B * 4);
+    add(a.depth, b.depth, B * 4);
+    add(a.status, b.status, B * 4);
+    add(a.stack, b.stack, B * (size_t)a.cap * 2);
+    add(a.mid, b.mid, B * 4);
+    if (a.best && b.best) add(a.best, b.best, B * 8);
+    if (a.rmemo && b.rmemo) add(a.rmemo, b.rmemo, B * (size_t)a.cap * 4);
+    size_t v16 = (B * (size_t)a.cap * 6 + B * 24) / 16;
+    int grid = (int)std::max<size_t>(1, std::min<size_t>((v16 + 255) / 256, (size_t)sm_count(dev) * 4));
+    psc_status s = launch_pdl(k_state_copy, dim3(grid), dim3(256), 0, cs, "k_state_copy", c);
+    if (s != PSC_OK) return s;
     dst->gen++;
     dst->mid_gen = src->mid_gen == src->gen ? dst->gen : 0;   // the mask ids are as current as src's
     dst->after_mask = false;
