@@ -7,6 +7,7 @@ CUDA graph are reported beside the timed region):
   k_step_tma       apply every row's precomputed mask to the bf16 logits in
                    place, write the packed bitmask [B][V/32] and pick the greedy
                    token among the allowed ones, in one TMA-pipelined pass
+                   (k_step_warp, a warp per 1024-column chunk, at small batches)
   k_advance_warp   lex + parse the chosen tokens on the device-resident stacks
                    and classify the new configurations (bottom-up classifier:
                    only the stack entries the step changed are re-read)
@@ -807,7 +808,7 @@ def main():
     barrier()
     torch.cuda.synchronize()
     elapsed_ms = t_start.elapsed_time(t_end)
-    mask_ms = [a.elapsed_time(b) for a, b, _ in ev]      # k_step_tma alone
+    mask_ms = [a.elapsed_time(b) for a, b, _ in ev]      # the masking kernel alone
     step_ms = [a.elapsed_time(c) for a, _, c in ev]      # the whole decode step
     elapsed_ms = max_over_ranks(elapsed_ms, dev)
     ms_per_step = elapsed_ms / K

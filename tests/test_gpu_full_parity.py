@@ -17,6 +17,8 @@ the CPU oracle.
   default options (bottom-up classifier too): all rows over all tokens at the
   prefix states (fused masking pass with the greedy choice) and through four
   whole decode steps.
+* The C-like 262,144-token workload at batches of 1, 3 and 16 rows (the
+  small-batch masking pass): six whole decode steps, every row over every token.
 * The C-like 262,144-token workload on the benchmark's exact path: the batch restored from a
   saved copy (psc_state_copy), then 32 steps of psc_decode_step_mask +
   psc_decode_step_advance on fresh logits; the oracle is advanced by the same
@@ -212,6 +214,42 @@ def test_c_like_262144_prefix_states_all_rows_all_tokens(psc):
     np.testing.assert_array_equal(bm.cpu().numpy().view(np.uint32), ref)
     np.testing.assert_array_equal(raw_bits(x), reference_masked(logits, allowed))
     np.testing.assert_array_equal(tok.cpu().numpy(), cpu_greedy(logits, allowed))
+
+
+@pytest.mark.parametrize("B", [1, 3, 16])
+def test_c_like_262144_small_batches_whole_decode(psc, B):
+    """Batches of 1, 3 and 16 rows of the 262,144-token workload (the small-batch
+    masking pass, a warp per 1024-column chunk, when the mask ids are current):
+    six whole decode steps; after every step the bitmask (left out on odd steps),
+    the masked logits and the greedy tokens of every row over every token, and
+    the statuses, equal the oracle's."""
+    b = big(psc, 5)
+    w = b.w
+    V = w.V
+    st = psc.psc_state_init(b.h, B, CAP)
+    tm = torch.from_numpy(w.token_matrix()[:B]).cuda()
+    for j in range(tm.shape[1]):
+        psc.psc_advance(b.h, st, tm[:, j].contiguous())
+    ocs = [oc.copy() for oc in b.ocs0[:B]]
+    tok = torch.empty(B, dtype=torch.int32, device="cuda")
+    stat = torch.empty(B, dtype=torch.int32, device="cuda")
+    for step in range(6):
+        x, logits = device_logits(B, V, 8000 + 10 * B + step, w.spec.sigma)
+        bm = torch.zeros(B, b.h.W, dtype=torch.int32, device="cuda") if step % 2 == 0 else None
+        psc.psc_decode_step(b.h, st, x, tok, bm, stat)
+        torch.cuda.synchronize()
+        ref = b.o.masks(ocs, b.voc, threads=THREADS)
+        if bm is not None:
+            np.testing.assert_array_equal(bm.cpu().numpy().view(np.uint32), ref, err_msg=f"step {step}")
+        allowed = bits_of(ref, V)
+        np.testing.assert_array_equal(raw_bits(x), reference_masked(logits, allowed), err_msg=f"step {step}")
+        t = tok.cpu().numpy()
+        np.testing.assert_array_equal(t, cpu_greedy(logits, allowed), err_msg=f"step {step}")
+        s = stat.cpu().numpy()
+        for r in range(B):
+            if t[r] >= 0:
+                ost = b.o.advance(ocs[r], None if t[r] == w.eos_id else w.vocab[t[r]])
+                assert s[r] == STATUS[ost], (step, r, s[r], ost)
 
 
 def greedy_rivals(xf, t):
