@@ -673,6 +673,51 @@ def run_profile(args):
     print(json.dumps({"mode": "profile", "steps": 3, "rows_with_a_token": int((tok >= 0).sum())}))
 
 
+def run_paths(args):
+    """A small case for profiler captures of the plain mask paths on config 5's
+    tables and prefix states (one 512 MiB logits buffer), each in an NVTX range:
+    "fill_apply" (psc_fill_apply: masks applied from the current mask ids,
+    k_apply_rows), "fill_mask" (psc_fill_mask, k_fill), "apply_mask"
+    (psc_apply_mask from that bitmask, k_apply_rows), "classify_walk"
+    (psc_fill_apply_noalloc on the same rows as plain arrays: every stack walked
+    from the top by k_classify, then k_apply_rows), "classify_bottom_up" (a
+    psc_advance with no tokens: every row classified again through its kept
+    bottom-up states)."""
+    import numpy as np
+    import torch
+    from paper_2608_03065_gb300 import build, psc
+    from workloads import configs
+    build.build()
+    w = configs.load(WORKLOAD)
+    B, V = w.B, w.V
+    h = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id)
+    st = psc.psc_state_init(h, B, 256)
+    tm = torch.from_numpy(w.token_matrix()).cuda()
+    for j in range(tm.shape[1]):
+        psc.psc_advance(h, st, tm[:, j].contiguous())
+    rows = psc.psc_states_download(st)
+    q = torch.from_numpy(rows["q"]).cuda()
+    depth = torch.from_numpy(rows["depth"]).cuda()
+    status = torch.from_numpy(rows["status"]).cuda()
+    stack = torch.from_numpy(rows["stack"].view(np.int16)).cuda()
+    g = torch.Generator(device="cuda").manual_seed(9)
+    x = (torch.randn(B, V, generator=g, device="cuda") * w.spec.sigma).to(torch.bfloat16)
+    bm = torch.empty(B, h.W, dtype=torch.int32, device="cuda")
+    none = torch.full((B,), -1, dtype=torch.int32, device="cuda")
+    torch.cuda.synchronize()
+    steps = [("fill_apply", lambda: psc.psc_fill_apply(h, st, x, bm)),
+             ("fill_mask", lambda: psc.psc_fill_mask(h, st, bm)),
+             ("apply_mask", lambda: psc.psc_apply_mask(x, bm, B, V)),
+             ("classify_walk", lambda: psc.psc_fill_apply_noalloc(h, q, depth, status, stack, x)),
+             ("classify_bottom_up", lambda: psc.psc_advance(h, st, none))]
+    for name, fn in steps:
+        torch.cuda.nvtx.range_push(name)
+        fn()
+        torch.cuda.synchronize()
+        torch.cuda.nvtx.range_pop()
+    print(json.dumps({"mode": "paths", "ranges": [n for n, _ in steps]}))
+
+
 # ------------------------------------------------------------------ main arm
 def main():
     ap = argparse.ArgumentParser()
@@ -683,12 +728,14 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cfg", type=int, default=WORKLOAD)
     ap.add_argument("--vocab", type=int, default=0)
-    ap.add_argument("--mode", default="decode", choices=["decode", "teacher", "sweep", "profile", "compile",
+    ap.add_argument("--mode", default="decode", choices=["decode", "teacher", "sweep", "profile", "paths", "compile",
                                                          "compile-one"],
                     help="decode: the benchmark line; teacher: teacher-forcing pass rates and "
                          "batch-1 step latency (the paper's RQ1/RQ2 measurements on these workloads); "
                          "sweep: decode-step time over batch sizes and logit types on config 5's tables; "
                          "profile: three decode steps in NVTX ranges, a small case for profiler captures; "
+                         "paths: the plain mask paths (fill_apply, fill_mask, apply_mask, classification) in "
+                         "NVTX ranges, for profiler captures; "
                          "compile: construction time, peak RSS and table sizes at real-grammar scale")
     args = ap.parse_args()
     if args.impl == "reference":
@@ -699,6 +746,8 @@ def main():
         return run_sweep(args)
     if args.mode == "profile":
         return run_profile(args)
+    if args.mode == "paths":
+        return run_paths(args)
     if args.mode == "compile":
         return run_compile(args)
     if args.mode == "compile-one":
