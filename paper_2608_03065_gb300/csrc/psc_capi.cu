@@ -1727,7 +1727,7 @@ __global__ void __launch_bounds__(256) k_step_warp(uint16_t* logits, int64_t str
     uint32_t mhi = __reduce_max_sync(FULL, khi);
     uint32_t mlo = __reduce_max_sync(FULL, khi == mhi ? klo : 0u);
     key = ((unsigned long long)mhi << 32) | mlo;
-    if (lane == 0 && key && best_key) atomicMax(best_key + b, key);
+    if (lane == 0 && key) atomicMax(best_key + b, key);
 }
 
 // One decode masking pass (classification, mask, apply, greedy key) with the
@@ -1957,7 +1957,7 @@ __global__ void __launch_bounds__(TMA_WARPS * 32, 3) k_step_tma(T* logits, int64
             uint32_t mlo = __reduce_max_sync(FULL, khi == mhi ? klo : 0u);
             key = ((unsigned long long)mhi << 32) | mlo;
             if (lane == 0) {
-                if (key && best_key) atomicMax(best_key + b, key);
+                if (key) atomicMax(best_key + b, key);
                 mbar_arrive(mempty0 + 8 * slot);
             }
         }
@@ -2114,12 +2114,9 @@ psc_status launch_advance(const psc_handle* h, psc_states* st, const int32_t* d_
     return s;
 }
 
-// keys = false: the masking pass without the greedy choice (psc_fill_apply); only
-// for 16-byte aligned rows.
 psc_status launch_fused(const psc_handle* h, const psc_states* st, void* d_logits, psc_dtype dtype, int64_t row_stride,
-                        int V, uint32_t* d_bitmask_out, cudaStream_t cs, bool keys = true) {
+                        int V, uint32_t* d_bitmask_out, cudaStream_t cs) {
     int B = st->d.B;
-    unsigned long long* best = keys ? st->d.best : nullptr;
     MaskSrc M{nullptr, h->d.mchunks, h->d.mrows, st->d.mid, h->d.W, h->d.nch, d_bitmask_out};
     size_t esz = dtype == PSC_BF16 ? 2 : 4;
     int vec = aligned16(d_logits) && ((row_stride * (int64_t)esz) % 16 == 0);
@@ -2139,9 +2136,9 @@ psc_status launch_fused(const psc_handle* h, const psc_states* st, void* d_logit
         // against 157.6)
         if (dtype == PSC_BF16 && have_mid && (long)B * cpr <= WARP_STEP_CHUNKS) {
             s = launch_pdl(k_step_warp, dim3(B * ((cpr + 7) / 8)), dim3(256), 0, cs, "k_step_warp",
-                           (uint16_t*)d_logits, row_stride, B, V, d_bitmask_out, best, h->d, st->d);
+                           (uint16_t*)d_logits, row_stride, B, V, d_bitmask_out, st->d.best, h->d, st->d);
             if (s == PSC_OK) const_cast<psc_states*>(st)->mid_gen = st->gen;
-            const_cast<psc_states*>(st)->after_mask = s == PSC_OK && keys;
+            const_cast<psc_states*>(st)->after_mask = s == PSC_OK;
             return s;
         }
         long want = ((long)B * cpr + resident - 1) / resident;
@@ -2150,11 +2147,11 @@ psc_status launch_fused(const psc_handle* h, const psc_states* st, void* d_logit
         int tgrid = (int)std::max(1L, std::min<long>(titems, resident));
         if (dtype == PSC_BF16)
             s = launch_pdl(k_step_tma<uint16_t>, dim3(tgrid), dim3(TMA_WARPS * 32), TmaShape<uint16_t>::SMEM, cs,
-                           "k_step_tma", (uint16_t*)d_logits, row_stride, B, V, d_bitmask_out, best, h->d,
+                           "k_step_tma", (uint16_t*)d_logits, row_stride, B, V, d_bitmask_out, st->d.best, h->d,
                            st->d, have_mid, seg);
         else
             s = launch_pdl(k_step_tma<uint32_t>, dim3(tgrid), dim3(TMA_WARPS * 32), TmaShape<uint32_t>::SMEM, cs,
-                           "k_step_tma", (uint32_t*)d_logits, row_stride, B, V, d_bitmask_out, best, h->d,
+                           "k_step_tma", (uint32_t*)d_logits, row_stride, B, V, d_bitmask_out, st->d.best, h->d,
                            st->d, have_mid, seg);
     } else {
         // rows not 16-byte aligned: warp-per-chunk pass, 4 resident CTAs of 256 threads per SM
@@ -2172,7 +2169,7 @@ psc_status launch_fused(const psc_handle* h, const psc_states* st, void* d_logit
         s = launch_check("k_apply_argmax");
     }
     if (s == PSC_OK) const_cast<psc_states*>(st)->mid_gen = st->gen;
-    const_cast<psc_states*>(st)->after_mask = s == PSC_OK && vec && have_mid && keys;
+    const_cast<psc_states*>(st)->after_mask = s == PSC_OK && vec && have_mid;
     return s;
 }
 
@@ -2871,9 +2868,6 @@ psc_status psc_fill_apply(const psc_handle* h, const psc_states* st, int32_t B, 
         return fail_with(PSC_ERR_ARG, "psc_fill_apply: bad arguments");
     cudaStream_t cs = (cudaStream_t)stream;
     if ((s = ensure_mid(h, st, cs)) != PSC_OK) return s;
-    size_t esz = dtype == PSC_BF16 ? 2 : 4;
-    if (aligned16(d_logits) && ((row_stride * (int64_t)esz) % 16 == 0))   // the decode masking pass, no greedy choice
-        return launch_fused(h, st, d_logits, dtype, row_stride, V, d_bitmask_out, cs, false);
     MaskSrc M{nullptr, h->d.mchunks, h->d.mrows, st->d.mid, h->d.W, h->d.nch, d_bitmask_out};
     return launch_apply(d_logits, dtype, row_stride, M, B, V, cs, h->device);
 }
