@@ -588,7 +588,8 @@ def run_compile(args):
     262,144-token C-like
     tables with the advance's tables staged in shared memory or read from
     global memory."""
-    jobs = [(2, None), (3, None), (4, None), (5, None), (6, 1024), (6, 2048), (6, 4096), (7, 131072), (7, None)]
+    jobs = [(2, None), (3, None), (4, None), (5, None), (6, 1024), (6, 2048), (6, 4096), (7, 131072), (7, None),
+            (8, 32768), (8, None)]
     if args.steps > 1000:   # --steps above 1000: also the 8,192-token Java-sized vocabulary
         jobs.append((6, 8192))
     rows = []
@@ -609,7 +610,8 @@ def run_compile(args):
             build.build()
             import tempfile
             for cfg, key, opts in ((6, "java_like_decode_step_us", {"bottom_up": False}),
-                                   (7, "java_like_pretok_262144_decode_step_us", {})):
+                                   (7, "java_like_pretok_262144_decode_step_us", {}),
+                                   (8, "sql_like_pretok_128256_decode_step_us", {"bottom_up": False})):
                 w = configs.load(cfg)
                 h = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id, **opts, **configs.COMPILE_LIMITS[cfg])
                 i = h.info()
@@ -621,7 +623,7 @@ def run_compile(args):
                     path = os.path.join(d, "t.psc")
                     psc.psc_save(h, path)
                     del h
-                    hg = psc.psc_load(path, global_tables=True, bottom_up="bottom_up" not in opts)
+                    hg = psc.psc_load(path, global_tables=True, bottom_up=opts.get("bottom_up", True))
                     rec["graph_us_global_tables"] = graph_step_us(psc, hg, w, w.B)
                     del hg
                     if cfg == 7:
@@ -652,8 +654,8 @@ def run_profile(args):
     build.build()
     w = configs.load(args.cfg)
     opts = dict(configs.COMPILE_LIMITS.get(args.cfg, {}))
-    if args.cfg == 6:
-        opts["bottom_up"] = False   # over its construction budget on this grammar and vocabulary
+    if args.cfg in (6, 8):
+        opts["bottom_up"] = False   # over its construction budget on these grammars and vocabularies
     h = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id, **opts)
     st = psc.psc_state_init(h, w.B, 256)
     tm = torch.from_numpy(w.token_matrix()).cuda()

@@ -17,6 +17,9 @@ the CPU oracle.
   default options (bottom-up classifier too): all rows over all tokens at the
   prefix states (fused masking pass with the greedy choice) and through four
   whole decode steps.
+* The SQL-like grammar (576 LALR(1) states) with a pre-tokenized vocabulary of
+  128,256 tokens, 256 rows: all rows over all tokens at the prefix states and
+  through three whole decode steps.
 * The C-like 262,144-token workload at batches of 1, 3 and 16 rows (the
   small-batch masking pass): six whole decode steps, every row over every token.
 * The C-like 262,144-token workload on the benchmark's exact path: the batch restored from a
@@ -214,6 +217,31 @@ def test_c_like_262144_prefix_states_all_rows_all_tokens(psc):
     np.testing.assert_array_equal(bm.cpu().numpy().view(np.uint32), ref)
     np.testing.assert_array_equal(raw_bits(x), reference_masked(logits, allowed))
     np.testing.assert_array_equal(tok.cpu().numpy(), cpu_greedy(logits, allowed))
+
+
+def test_sql_like_128256_pretokenized_all_rows_all_tokens(psc):
+    """The SQL-like grammar (576 LALR(1) states, case-insensitive keywords ranked
+    above names, contextual lexer) with a pre-tokenized vocabulary of 128,256
+    tokens, 256 rows (parser tables packed to fit shared memory, stacks walked from
+    the top): the fused masking pass at the prefix states, then three whole decode
+    steps, every row over every token."""
+    b = big(psc, 8, bottom_up=False, **configs.COMPILE_LIMITS[8])
+    w = b.w
+    info = b.h.info()
+    assert info.n_parser_states >= 500 and info.advance_tables_packed == 1
+    assert w.V == 128256 and w.B == 256
+    ref = b.o.masks(b.ocs0, b.voc, threads=THREADS)
+    st, _ = b.restored(psc)
+    x, logits = device_logits(w.B, w.V, 8500, w.spec.sigma)
+    bm = torch.zeros(w.B, b.h.W, dtype=torch.int32, device="cuda")
+    tok = torch.empty(w.B, dtype=torch.int32, device="cuda")
+    psc.psc_fill_apply_argmax(b.h, st, x, tok, bm)
+    torch.cuda.synchronize()
+    allowed = bits_of(ref, w.V)
+    np.testing.assert_array_equal(bm.cpu().numpy().view(np.uint32), ref)
+    np.testing.assert_array_equal(raw_bits(x), reference_masked(logits, allowed))
+    np.testing.assert_array_equal(tok.cpu().numpy(), cpu_greedy(logits, allowed))
+    whole_decode_all_rows_all_tokens(psc, b, 3, 8600)
 
 
 @pytest.mark.parametrize("B", [1, 3, 16])

@@ -13,7 +13,8 @@ torch = pytest.importorskip("torch")
 SINGLES = {bytes([b]) for b in list(range(0x20, 0x7F)) + [9, 10, 13]}
 
 
-@pytest.mark.parametrize("cfg_id,batch", [(1, None), (2, None), (3, 16), (4, 16), (5, 16), (6, 16), (7, 16)])
+@pytest.mark.parametrize("cfg_id,batch", [(1, None), (2, None), (3, 16), (4, 16), (5, 16), (6, 16), (7, 16),
+                                          (8, 16)])
 def test_vocabulary_and_prefixes(cfg_id, batch):
     w = configs.load(cfg_id, batch=batch)
     s = configs.SPECS[cfg_id]

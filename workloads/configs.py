@@ -9,6 +9,8 @@
 6. (extra) Java-sized language (1,001 LALR(1) states), V=4,096, B=64, prefixes of 64-2048 bytes
 7. (extra) the same language with a pre-tokenized vocabulary of V=262,144 (the size of the
    paper's largest tokenizer), B=256, prefixes of 64-2048 bytes
+8. (extra) SQL-like language (576 LALR(1) states, case-insensitive keywords), pre-tokenized
+   vocabulary of V=128,256, B=256, prefixes of 64-2048 bytes
 
 N(0,2) is read as variance 2 (sigma = sqrt 2).  The paper's datasets, JSON
 schemas and tokenizers are not available; these stand in for them.
@@ -61,9 +63,12 @@ SPECS = {
     # the byte-level BPE tokenizers the paper uses); 3 % of the tokens are punctuation runs
     7: WorkloadSpec(7, "java_like_pretok_v262144_b256", 256, 262144, "bf16", math.sqrt(2), 64, 2048, 24,
                     0.0, max_depth=60, vocab_style="pretokenized"),
+    # not a benchmark configuration: the SQL-like grammar at the Llama 3 vocabulary size
+    8: WorkloadSpec(8, "sql_like_pretok_v128256_b256", 256, 128256, "bf16", math.sqrt(2), 64, 2048, 24,
+                    0.0, max_depth=40, vocab_style="pretokenized"),
 }
 # the Java-sized constructions build ~20 M states (6) and ~16 M states (7)
-COMPILE_LIMITS = {6: {"max_states": 64_000_000}, 7: {"max_states": 64_000_000}}
+COMPILE_LIMITS = {6: {"max_states": 64_000_000}, 7: {"max_states": 64_000_000}, 8: {"max_states": 64_000_000}}
 
 
 def grammar_spec(cfg: int) -> grammars.GrammarSpec:
@@ -75,6 +80,8 @@ def grammar_spec(cfg: int) -> grammars.GrammarSpec:
         return grammars.schema_json(seed=int(np.random.default_rng([3, 1]).integers(0, 2**31)))
     if cfg in (6, 7):
         return grammars.java_like()
+    if cfg == 8:
+        return grammars.sql_like()
     return grammars.c_like()
 
 

@@ -798,3 +798,265 @@ def java_like() -> GrammarSpec:
     nesting = {("stmt", 2), ("if_else_stmt", 0), ("stmt_wts", 0), ("while_stmt", 0), ("for_stmt", 0),
                ("primary_nna", 3), ("class_body_decl", 1)}
     return GrammarSpec("java_like", rules, terms, "contextual", _c_sep, weights=weights, nesting=nesting)
+
+
+# ------------------------------------------------------------------- SQL-like
+SQL_KEYWORDS = [
+    "select", "distinct", "all", "from", "where", "group", "by", "having", "order", "asc", "desc", "nulls",
+    "first", "last", "limit", "offset", "union", "except", "intersect", "with", "recursive", "as", "join",
+    "inner", "left", "right", "full", "outer", "cross", "natural", "on", "using", "and", "or", "not", "is",
+    "null", "true", "false", "between", "in", "like", "exists", "case", "when", "then", "else", "end", "cast",
+    "over", "partition", "insert", "into", "values", "update", "set", "delete", "create", "table", "if",
+    "index", "unique", "view", "drop", "alter", "add", "column", "rename", "to", "primary", "key", "foreign",
+    "references", "check", "constraint", "default", "begin", "commit", "rollback", "integer", "int",
+    "bigint", "smallint", "real", "double", "precision", "float", "boolean", "text", "date", "timestamp",
+    "varchar", "char", "decimal", "numeric", "any", "some", "escape", "returning", "conflict", "do",
+    "nothing", "rows", "range", "unbounded", "preceding", "following", "current", "row", "filter", "extract",
+    "coalesce", "nullif", "interval", "temporary", "cascade", "restrict",
+]
+
+
+def _sql_keyword(word: str):
+    def sample(rng) -> bytes:
+        r = rng.random()
+        if r < 0.5:
+            return word.upper().encode()
+        if r < 0.9:
+            return word.encode()
+        return "".join(c.upper() if rng.random() < 0.5 else c for c in word).encode()
+    return sample
+
+
+def _sql_name(rng) -> bytes:
+    while True:
+        r = rng.random()
+        if r < 0.6:
+            w = _word(rng, 1, 10)
+        elif r < 0.9:
+            w = _word(rng, 1, 6) + "_" + _word(rng, 1, 6)
+        else:
+            w = _word(rng, 1, 1) + _digits(rng, 1, 2)
+        if w not in SQL_KEYWORDS:
+            return w.encode()
+
+
+def _sql_string(rng) -> bytes:
+    s = "".join("''" if rng.random() < 0.05 else _word(rng, 1, 1, _LOWER + " %_-.")
+                for _ in range(int(rng.integers(0, 10))))
+    return ("'" + s + "'").encode()
+
+
+def _sql_number(rng) -> bytes:
+    r = rng.random()
+    if r < 0.6:
+        return (_digits(rng, 1, 3) + "." + _digits(rng, 1, 3)).encode()
+    if r < 0.8:
+        return ("." + _digits(rng, 1, 3)).encode()
+    return (_digits(rng, 1, 2) + "e" + _digits(rng, 1, 2)).encode()
+
+
+def _sql_param(rng) -> bytes:
+    r = rng.random()
+    if r < 0.4:
+        return b"?"
+    if r < 0.7:
+        return (":" + _word(rng, 1, 6)).encode()
+    return ("$" + _digits(rng, 1, 2)).encode()
+
+
+def _sql_sep(rng, a, b):
+    r = rng.random()
+    if r < 0.85:
+        return b" "
+    if r < 0.97:
+        return b"\n" + b"  " * int(rng.integers(0, 4))
+    return b" -- " + _word(rng, 1, 8).encode() + b"\n"
+
+
+def sql_like() -> GrammarSpec:
+    """Synthetic SQL-like language (stands in for the paper's SQL grammar): statement
+    lists of queries (WITH [RECURSIVE] common table expressions, set operations,
+    SELECT with DISTINCT, joins of every kind with ON / USING, WHERE, GROUP BY,
+    HAVING, ORDER BY with NULLS FIRST/LAST, LIMIT / OFFSET), expressions over
+    OR / AND / NOT, comparisons with quantified subqueries, IS [NOT] NULL,
+    [NOT] BETWEEN / IN / LIKE [ESCAPE], EXISTS, CASE, CAST, EXTRACT, COALESCE,
+    function calls with DISTINCT, FILTER and window clauses (PARTITION BY, ORDER BY,
+    ROWS / RANGE frames), INSERT (VALUES or a query, ON CONFLICT, RETURNING),
+    UPDATE, DELETE, CREATE TABLE / INDEX / VIEW, DROP, ALTER TABLE and transaction
+    statements.  Keywords are case-insensitive regex terminals ranked above NAME
+    (contextual lexer: a keyword spelling is a name wherever the keyword cannot
+    follow).  Written LALR(1): a parenthesized query appears only where an
+    expression or a table reference is expected, and INSERT takes a bare SELECT."""
+    K = {w: w.upper() for w in SQL_KEYWORDS}   # keyword terminal names
+    L = lambda s: _lit(s)  # noqa: E731
+    k = lambda w: K[w]  # noqa: E731
+    rules = {
+        "start": [["stmts"]],
+        "stmts": [["stmt", L(";")], ["stmts", "stmt", L(";")]],
+        "stmt": [["query"], ["insert"], ["update"], ["delete"], ["create_table"], ["create_index"],
+                 ["create_view"], ["drop"], ["alter"], [k("begin")], [k("commit")], [k("rollback")]],
+        # queries
+        "query": [["query_body"], ["with_clause", "query_body"]],
+        "with_clause": [[k("with"), "ctes"], [k("with"), k("recursive"), "ctes"]],
+        "ctes": [["cte"], ["ctes", L(","), "cte"]],
+        "cte": [["NAME", k("as"), L("("), "query", L(")")],
+                ["NAME", L("("), "name_list", L(")"), k("as"), L("("), "query", L(")")]],
+        "query_body": [["set_expr"], ["set_expr", "order_by"], ["set_expr", "limit_clause"],
+                       ["set_expr", "order_by", "limit_clause"]],
+        "set_expr": [["set_term"], ["set_expr", k("union"), "set_term"], ["set_expr", k("union"), k("all"), "set_term"],
+                     ["set_expr", k("except"), "set_term"]],
+        "set_term": [["select_core"], ["set_term", k("intersect"), "select_core"]],
+        "select_core": [[k("select"), "set_quant", "select_list", "opt_from", "opt_where", "opt_group",
+                         "opt_having"]],
+        "set_quant": [[], [k("distinct")], [k("all")]],
+        "select_list": [["select_item"], ["select_list", L(","), "select_item"]],
+        "select_item": [["expr"], ["expr", "NAME"], ["expr", k("as"), "NAME"], [L("*")], ["qname", L("."), L("*")]],
+        "opt_from": [[], [k("from"), "table_refs"]],
+        "table_refs": [["table_ref"], ["table_refs", L(","), "table_ref"]],
+        "table_ref": [["table_primary"], ["joined"]],
+        "joined": [["table_ref", "join_type", k("join"), "table_primary", "join_cond"],
+                   ["table_ref", k("cross"), k("join"), "table_primary"],
+                   ["table_ref", k("natural"), "join_type", k("join"), "table_primary"]],
+        "join_type": [[], [k("inner")], [k("left")], [k("left"), k("outer")], [k("right")],
+                      [k("right"), k("outer")], [k("full")], [k("full"), k("outer")]],
+        "join_cond": [[k("on"), "expr"], [k("using"), L("("), "name_list", L(")")]],
+        "table_primary": [["qname"], ["qname", "alias"], [L("("), "query", L(")"), "alias"],
+                          [L("("), "joined", L(")")]],
+        "alias": [["NAME"], [k("as"), "NAME"], [k("as"), "NAME", L("("), "name_list", L(")")]],
+        "opt_where": [[], [k("where"), "expr"]],
+        "opt_group": [[], [k("group"), k("by"), "expr_list"]],
+        "opt_having": [[], [k("having"), "expr"]],
+        "order_by": [[k("order"), k("by"), "order_items"]],
+        "order_items": [["order_item"], ["order_items", L(","), "order_item"]],
+        "order_item": [["expr", "opt_dir", "opt_nulls"]],
+        "opt_dir": [[], [k("asc")], [k("desc")]],
+        "opt_nulls": [[], [k("nulls"), k("first")], [k("nulls"), k("last")]],
+        "limit_clause": [[k("limit"), "expr"], [k("limit"), "expr", k("offset"), "expr"], [k("offset"), "expr"]],
+        # expressions
+        "expr": [["or_expr"]],
+        "or_expr": [["and_expr"], ["or_expr", k("or"), "and_expr"]],
+        "and_expr": [["not_expr"], ["and_expr", k("and"), "not_expr"]],
+        "not_expr": [["pred"], [k("not"), "not_expr"]],
+        "pred": [["add_expr"], ["add_expr", "comp_op", "add_expr"],
+                 ["add_expr", "comp_op", "quantifier", L("("), "query", L(")")],
+                 ["add_expr", k("is"), k("null")], ["add_expr", k("is"), k("not"), k("null")],
+                 ["add_expr", k("is"), k("true")], ["add_expr", k("is"), k("false")],
+                 ["add_expr", k("between"), "add_expr", k("and"), "add_expr"],
+                 ["add_expr", k("not"), k("between"), "add_expr", k("and"), "add_expr"],
+                 ["add_expr", k("in"), L("("), "expr_list", L(")")],
+                 ["add_expr", k("not"), k("in"), L("("), "expr_list", L(")")],
+                 ["add_expr", k("in"), L("("), "query", L(")")],
+                 ["add_expr", k("not"), k("in"), L("("), "query", L(")")],
+                 ["add_expr", k("like"), "add_expr"], ["add_expr", k("not"), k("like"), "add_expr"],
+                 ["add_expr", k("like"), "add_expr", k("escape"), "STRING"],
+                 [k("exists"), L("("), "query", L(")")]],
+        "quantifier": [[k("any")], [k("some")], [k("all")]],
+        "comp_op": [[L(o)] for o in ["=", "<>", "!=", "<", "<=", ">", ">="]],
+        "add_expr": [["mul_expr"], ["add_expr", L("+"), "mul_expr"], ["add_expr", L("-"), "mul_expr"],
+                     ["add_expr", L("||"), "mul_expr"]],
+        "mul_expr": [["unary"], ["mul_expr", L("*"), "unary"], ["mul_expr", L("/"), "unary"],
+                     ["mul_expr", L("%"), "unary"]],
+        "unary": [["primary"], [L("-"), "unary"], [L("+"), "unary"]],
+        "primary": [["literal"], ["qname"], ["PARAM"], [L("("), "expr", L(")")], [L("("), "query", L(")")],
+                    ["func_call"], ["case_expr"], [k("cast"), L("("), "expr", k("as"), "type_name", L(")")],
+                    [k("extract"), L("("), "NAME", k("from"), "expr", L(")")],
+                    [k("coalesce"), L("("), "expr_list", L(")")],
+                    [k("nullif"), L("("), "expr", L(","), "expr", L(")")],
+                    [k("interval"), "STRING"]],
+        "literal": [["INT"], ["NUMBER"], ["STRING"], [k("null")], [k("true")], [k("false")],
+                    [k("date"), "STRING"], [k("timestamp"), "STRING"]],
+        "func_call": [["qname", L("("), "func_args", L(")"), "opt_filter", "opt_over"]],
+        "func_args": [[], ["expr_list"], [k("distinct"), "expr_list"], [L("*")]],
+        "opt_filter": [[], [k("filter"), L("("), k("where"), "expr", L(")")]],
+        "opt_over": [[], [k("over"), L("("), "window_spec", L(")")], [k("over"), "NAME"]],
+        "window_spec": [["opt_partition", "opt_window_order", "opt_frame"]],
+        "opt_partition": [[], [k("partition"), k("by"), "expr_list"]],
+        "opt_window_order": [[], ["order_by"]],
+        "opt_frame": [[], ["frame_unit", "frame_bound"],
+                      ["frame_unit", k("between"), "frame_bound", k("and"), "frame_bound"]],
+        "frame_unit": [[k("rows")], [k("range")]],
+        "frame_bound": [[k("unbounded"), k("preceding")], [k("unbounded"), k("following")],
+                        [k("current"), k("row")], ["INT", k("preceding")], ["INT", k("following")]],
+        "case_expr": [[k("case"), "when_list", "opt_else", k("end")],
+                      [k("case"), "expr", "when_list", "opt_else", k("end")]],
+        "when_list": [[k("when"), "expr", k("then"), "expr"], ["when_list", k("when"), "expr", k("then"), "expr"]],
+        "opt_else": [[], [k("else"), "expr"]],
+        "expr_list": [["expr"], ["expr_list", L(","), "expr"]],
+        "name_list": [["NAME"], ["name_list", L(","), "NAME"]],
+        "qname": [["NAME"], ["qname", L("."), "NAME"]],
+        "type_name": [[k("integer")], [k("int")], [k("bigint")], [k("smallint")], [k("real")],
+                      [k("double"), k("precision")], [k("float")], [k("boolean")], [k("text")], [k("date")],
+                      [k("timestamp")], [k("varchar"), L("("), "INT", L(")")], [k("char"), L("("), "INT", L(")")],
+                      [k("decimal"), L("("), "INT", L(","), "INT", L(")")],
+                      [k("numeric"), L("("), "INT", L(","), "INT", L(")")]],
+        # data manipulation
+        "insert": [[k("insert"), k("into"), "qname", "insert_src", "opt_conflict", "opt_returning"],
+                   [k("insert"), k("into"), "qname", L("("), "name_list", L(")"), "insert_src", "opt_conflict",
+                    "opt_returning"]],
+        "insert_src": [[k("values"), "value_rows"], ["select_core"], ["select_core", "order_by"],
+                       [k("default"), k("values")]],
+        "value_rows": [[L("("), "expr_list", L(")")], ["value_rows", L(","), L("("), "expr_list", L(")")]],
+        "opt_conflict": [[], [k("on"), k("conflict"), k("do"), k("nothing")],
+                         [k("on"), k("conflict"), L("("), "name_list", L(")"), k("do"), k("nothing")],
+                         [k("on"), k("conflict"), L("("), "name_list", L(")"), k("do"), k("update"), k("set"),
+                          "assignments"]],
+        "opt_returning": [[], [k("returning"), "select_list"]],
+        "update": [[k("update"), "qname", k("set"), "assignments", "opt_from", "opt_where", "opt_returning"]],
+        "assignments": [["assignment"], ["assignments", L(","), "assignment"]],
+        "assignment": [["NAME", L("="), "expr"], ["NAME", L("="), k("default")]],
+        "delete": [[k("delete"), k("from"), "qname", "opt_where", "opt_returning"]],
+        # definitions
+        "create_table": [[k("create"), "opt_temp", k("table"), "opt_if_not_exists", "qname", L("("), "table_elems",
+                          L(")")],
+                         [k("create"), "opt_temp", k("table"), "opt_if_not_exists", "qname", k("as"), "query"]],
+        "opt_temp": [[], [k("temporary")]],
+        "opt_if_not_exists": [[], [k("if"), k("not"), k("exists")]],
+        "table_elems": [["table_elem"], ["table_elems", L(","), "table_elem"]],
+        "table_elem": [["NAME", "type_name", "col_constraints"], ["table_constraint"],
+                       [k("constraint"), "NAME", "table_constraint"]],
+        "col_constraints": [[], ["col_constraints", "col_constraint"]],
+        "col_constraint": [[k("not"), k("null")], [k("null")], [k("primary"), k("key")], [k("unique")],
+                           [k("default"), "default_value"], [k("references"), "qname"],
+                           [k("references"), "qname", L("("), "name_list", L(")")],
+                           [k("check"), L("("), "expr", L(")")]],
+        "default_value": [["literal"], [L("-"), "INT"], [L("("), "expr", L(")")]],
+        "table_constraint": [[k("primary"), k("key"), L("("), "name_list", L(")")],
+                             [k("unique"), L("("), "name_list", L(")")],
+                             [k("foreign"), k("key"), L("("), "name_list", L(")"), k("references"), "qname",
+                              L("("), "name_list", L(")")],
+                             [k("check"), L("("), "expr", L(")")]],
+        "create_index": [[k("create"), k("index"), "NAME", k("on"), "qname", L("("), "index_items", L(")")],
+                         [k("create"), k("unique"), k("index"), "NAME", k("on"), "qname", L("("), "index_items",
+                          L(")")]],
+        "index_items": [["index_item"], ["index_items", L(","), "index_item"]],
+        "index_item": [["NAME", "opt_dir"]],
+        "create_view": [[k("create"), k("view"), "qname", k("as"), "query"],
+                        [k("create"), k("view"), "qname", L("("), "name_list", L(")"), k("as"), "query"]],
+        "drop": [[k("drop"), "drop_kind", "qname", "opt_drop_mode"],
+                 [k("drop"), "drop_kind", k("if"), k("exists"), "qname", "opt_drop_mode"]],
+        "drop_kind": [[k("table")], [k("view")], [k("index")]],
+        "opt_drop_mode": [[], [k("cascade")], [k("restrict")]],
+        "alter": [[k("alter"), k("table"), "qname", "alter_action"]],
+        "alter_action": [[k("add"), k("column"), "NAME", "type_name", "col_constraints"],
+                         [k("add"), "table_constraint"],
+                         [k("drop"), k("column"), "NAME"], [k("rename"), k("to"), "NAME"],
+                         [k("rename"), k("column"), "NAME", k("to"), "NAME"],
+                         [k("alter"), k("column"), "NAME", k("set"), k("default"), "default_value"],
+                         [k("alter"), k("column"), "NAME", k("drop"), k("default")]],
+    }
+    terms = {K[w]: TermSpec("/" + "".join(f"[{c.lower()}{c.upper()}]" if c.isalpha() else c for c in w) + "/",
+                            _sql_keyword(w), priority=2) for w in SQL_KEYWORDS}
+    terms.update({
+        "NAME": TermSpec("/[A-Za-z_][A-Za-z0-9_]*|\"([^\"]|\"\")+\"/", _sql_name),
+        "INT": TermSpec("/[0-9]+/", lambda r: _digits(r, 1, 4).encode()),
+        "NUMBER": TermSpec("/[0-9]+\\.[0-9]*([eE][+-]?[0-9]+)?|\\.[0-9]+([eE][+-]?[0-9]+)?|[0-9]+[eE][+-]?[0-9]+/",
+                           _sql_number),
+        "STRING": TermSpec("/'([^']|'')*'/", _sql_string),
+        "PARAM": TermSpec("/\\?|:[A-Za-z_][A-Za-z0-9_]*|\\$[0-9]+/", _sql_param),
+        "LINE_COMMENT": TermSpec("/--[^\\n]*/", lambda r: b"-- x", ignored=True),
+        "BLOCK_COMMENT": TermSpec("/\\/\\*([^*]|\\*+[^*\\/])*\\*+\\//", lambda r: b"/* x */", ignored=True),
+        "WS": TermSpec("/[ \\t\\r\\n]+/", lambda r: b" ", ignored=True),
+    })
+    weights = {("stmts", 1): 2.0, ("stmt", 0): 4.0, ("select_list", 1): 1.5, ("and_expr", 1): 1.2}
+    nesting = {("primary", 3), ("primary", 4), ("table_primary", 2), ("pred", 11)}
+    return GrammarSpec("sql_like", rules, terms, "contextual", _sql_sep, weights=weights, nesting=nesting)
