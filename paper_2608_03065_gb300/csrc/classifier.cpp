@@ -26,6 +26,9 @@
 #include <chrono>
 #include <cstring>
 #include <mutex>
+#include <climits>
+#include <memory>
+#include <map>
 #include <thread>
 #include <cstdio>
 #include <cstdlib>
@@ -813,8 +816,15 @@ Tables compile_tables(const std::string& text, const uint8_t* vb, const int64_t*
     }
     double t3 = now();
 
-    // ---- Moore minimisation, initial partition by mask
-    int N = (int)B.st_mask.size();
+    // ---- Moore minimisation, initial partition by mask.  Each round gives every
+    // state the signature (its class, the class of its default target, then the
+    // (symbol, class) of each exception whose target class differs from the
+    // default's) and numbers the distinct signatures in the order of their first
+    // state, which is what a serial scan gives.  The signatures are hashed in
+    // parallel; a shared open-addressing table keeps the first state of every hash,
+    // every state is compared with that state's full signature, and a state whose
+    // hash is shared by a different signature is grouped through a serial map.
+    const int N = (int)B.st_mask.size();
     std::vector<int32_t> cls(N);
     {
         std::unordered_map<int32_t, int32_t> m2c;
@@ -824,48 +834,123 @@ Tables compile_tables(const std::string& text, const uint8_t* vb, const int64_t*
             cls[s] = it->second;
         }
     }
-    int ncl = -1;
-    std::vector<int64_t> sig;
-    for (int iter = 0; iter < 100000; iter++) {
-        std::unordered_multimap<uint64_t, int32_t> idx;
-        std::vector<int64_t> sig_off{0};
-        std::vector<int64_t> sig_data;
-        std::vector<int32_t> nc(N);
-        std::vector<int32_t> rep_of_new;
-        int count = 0;
-        for (int s = 0; s < N; s++) {
-            sig.clear();
-            int32_t dc = cls[B.st_def[s]];
-            sig.push_back(cls[s]);
-            sig.push_back(dc);
-            for (int64_t e = B.exc_off[s]; e < B.exc_off[s + 1]; e++) {
-                int32_t tc = cls[B.exc_t[e]];
-                if (tc != dc) sig.push_back(((int64_t)B.exc_y[e] << 32) | (uint32_t)tc);
+    auto sig_of = [&](int s, std::vector<int64_t>& sig) {
+        sig.clear();
+        int32_t dc = cls[B.st_def[s]];
+        sig.push_back(cls[s]);
+        sig.push_back(dc);
+        for (int64_t e = B.exc_off[s]; e < B.exc_off[s + 1]; e++) {
+            int32_t tc = cls[B.exc_t[e]];
+            if (tc != dc) sig.push_back(((int64_t)B.exc_y[e] << 32) | (uint32_t)tc);
+        }
+    };
+    auto hash_of = [](const std::vector<int64_t>& sig) {
+        uint64_t h = 1469598103934665603ull;
+        for (int64_t x : sig) h = mix64(h ^ (uint64_t)x);
+        return h ? h : 1ull;   // 0 marks an empty slot
+    };
+    // contiguous chunks of [0, n), one worker per thread
+    auto chunks_of = [&](int64_t n, auto&& body) {
+        const int64_t step = 1 << 16;
+        std::atomic<int64_t> next{0};
+        auto run = [&]() {
+            std::vector<int64_t> a, b;
+            for (;;) {
+                int64_t lo = next.fetch_add(step);
+                if (lo >= n) break;
+                body(lo, std::min<int64_t>(n, lo + step), a, b);
             }
-            uint64_t h = 1469598103934665603ull;
-            for (int64_t x : sig) h = mix64(h ^ (uint64_t)x);
-            int32_t found = -1;
-            auto range = idx.equal_range(h);
-            for (auto it = range.first; it != range.second; ++it) {
-                int32_t c = it->second;
-                int64_t a = sig_off[c], b = sig_off[c + 1];
-                if ((size_t)(b - a) == sig.size() && std::equal(sig.begin(), sig.end(), sig_data.begin() + a)) {
-                    found = c;
-                    break;
+        };
+        int nt = (int)std::max<int64_t>(1, std::min<int64_t>(threads, (n + step - 1) / step));
+        if (nt <= 1) {
+            run();
+            return;
+        }
+        std::vector<std::thread> pool;
+        for (int k = 0; k < nt; k++) pool.emplace_back(run);
+        for (auto& th : pool) th.join();
+    };
+    auto chunks = [&](auto&& body) { chunks_of(N, body); };
+    size_t cap = 1024;
+    while (cap < 2 * (size_t)N) cap <<= 1;
+    std::unique_ptr<std::atomic<uint64_t>[]> tkey(new std::atomic<uint64_t>[cap]);
+    std::unique_ptr<std::atomic<int32_t>[]> tval(new std::atomic<int32_t>[cap]);
+    auto clear_table = [&]() {
+        chunks_of((int64_t)cap, [&](int64_t lo, int64_t hi, std::vector<int64_t>&, std::vector<int64_t>&) {
+            for (int64_t i = lo; i < hi; i++) {
+                tkey[i].store(0, std::memory_order_relaxed);
+                tval[i].store(INT32_MAX, std::memory_order_relaxed);
+            }
+        });
+    };
+    clear_table();
+    auto slot_of = [&](uint64_t h, bool insert) -> size_t {
+        size_t i = (size_t)h & (cap - 1);
+        for (;;) {
+            uint64_t k = tkey[i].load(std::memory_order_relaxed);
+            if (k == h) return i;
+            if (k == 0 && insert) {
+                uint64_t z = 0;
+                if (tkey[i].compare_exchange_strong(z, h) || z == h) return i;
+            }
+            i = (i + 1) & (cap - 1);
+        }
+    };
+    std::vector<uint64_t> hs(N);
+    std::vector<int32_t> first(N), nc(N);
+    std::vector<char> odd(N);
+    int ncl = -1;
+    for (int iter = 0; iter < 100000; iter++) {
+        // hashes, and the first state of every hash
+        chunks([&](int64_t lo, int64_t hi, std::vector<int64_t>& sig, std::vector<int64_t>&) {
+            for (int s = (int)lo; s < (int)hi; s++) {
+                sig_of(s, sig);
+                uint64_t h = hash_of(sig);
+                hs[s] = h;
+                std::atomic<int32_t>& v = tval[slot_of(h, true)];
+                int32_t cur = v.load(std::memory_order_relaxed);
+                while (s < cur && !v.compare_exchange_weak(cur, s)) {
                 }
             }
-            if (found < 0) {
-                found = count++;
-                sig_data.insert(sig_data.end(), sig.begin(), sig.end());
-                sig_off.push_back((int64_t)sig_data.size());
-                idx.emplace(h, found);
+        });
+        // every state against the first state of its hash
+        chunks([&](int64_t lo, int64_t hi, std::vector<int64_t>& a, std::vector<int64_t>& b) {
+            for (int s = (int)lo; s < (int)hi; s++) {
+                int32_t r = tval[slot_of(hs[s], false)].load(std::memory_order_relaxed);
+                first[s] = r;
+                odd[s] = 0;
+                if (r != s) {
+                    sig_of(s, a);
+                    sig_of(r, b);
+                    odd[s] = a != b;
+                }
             }
-            nc[s] = found;
+        });
+        // states whose hash is shared by another signature: grouped by full signature
+        {
+            std::map<std::vector<int64_t>, int32_t> groups;
+            std::vector<int64_t> sig;
+            for (int s = 0; s < N; s++)
+                if (odd[s]) {
+                    sig_of(s, sig);
+                    auto it = groups.emplace(sig, s).first;
+                    first[s] = it->second;
+                }
         }
+        // the distinct signatures numbered in the order of their first state
+        int count = 0;
+        for (int s = 0; s < N; s++)
+            if (first[s] == s) nc[s] = count++;
+        chunks([&](int64_t lo, int64_t hi, std::vector<int64_t>&, std::vector<int64_t>&) {
+            for (int s = (int)lo; s < (int)hi; s++)
+                if (first[s] != s) nc[s] = nc[first[s]];   // a first state is numbered above and not written here
+        });
         cls.swap(nc);
+        clear_table();
         if (count == ncl) break;
         ncl = count;
     }
+    if (getenv("PSC_LOG")) fprintf(stderr, "psc: minimisation: %d states -> %d classes\n", N, ncl);
     double t4 = now();
 
     // ---- flatten
