@@ -91,14 +91,18 @@ def _payload_start(data: bytes) -> int:
     return 32 + 16 * nb
 
 
-def test_compiled_tables_do_not_depend_on_the_thread_count(psc, tmp_path, uncompressed):
+@pytest.mark.parametrize("cfg_id,V", [(2, None), (8, 2048)])
+def test_compiled_tables_do_not_depend_on_the_thread_count(psc, tmp_path, uncompressed, cfg_id, V):
     """Files compiled with 1 and with 8 host threads are byte-identical except
     for the recorded compile time (and so the checksum): table ids are numbered
-    in an order that does not depend on which thread finishes first."""
-    w = configs.load(2, batch=2)
+    in an order that does not depend on which thread finishes first.  The
+    SQL-like grammar at 2,048 tokens builds a million classifier states, so the
+    minimisation's rounds run on many chunks in parallel."""
+    text = configs.grammar_spec(cfg_id).text()
+    toks = configs.vocab_for(cfg_id, V)
     data = []
     for th in (1, 8):
-        h = psc.psc_compile(w.grammar_text, w.vocab, w.eos_id, host_only=True, threads=th)
+        h = psc.psc_compile(text, toks, len(toks) - 1, host_only=True, threads=th, bottom_up=V is None)
         path = str(tmp_path / f"t{th}.psc")
         psc.psc_save(h, path)
         data.append(open(path, "rb").read())
