@@ -52,7 +52,8 @@ uint64_t mix(uint64_t h) {
     return h;
 }
 
-uint64_t hash_state(int t, const int32_t* g, size_t n) {
+template <typename G>
+uint64_t hash_state(int t, const G* g, size_t n) {
     uint64_t h = mix(0x9e3779b97f4a7c15ull ^ (uint64_t)t);
     for (size_t i = 0; i < n; i++) h = mix(h ^ ((uint64_t)(uint32_t)g[i] << 1) ^ i);
     return h;
@@ -82,9 +83,10 @@ double seconds() {
     return std::chrono::duration<double>(std::chrono::steady_clock::now().time_since_epoch()).count();
 }
 
-}  // namespace
-
-bool build_bottom_up(Tables& T, const Options& opt) {
+// G: the element type of the g vectors (mask ids): uint16_t when every mask id
+// fits, which halves the construction's memory, else int32_t.
+template <typename G>
+bool build_bottom_up_g(Tables& T, const Options& opt) {
     T.bu.clear();
     T.bu_slot.clear();
     T.bu_F.clear();
@@ -198,15 +200,15 @@ bool build_bottom_up(Tables& T, const Options& opt) {
     // in one growing block (realloc moves large blocks by remapping, not copying);
     // new states of a batch are numbered serially and copied in parallel.
     struct Arena {
-        int32_t* p = nullptr;
+        G* p = nullptr;
         size_t n = 0, cap = 0;
         ~Arena() { free(p); }
         bool grow(size_t need) {
             if (need <= cap) return true;
             size_t c = std::max(need, std::max<size_t>(cap * 2, (size_t)1 << 24));
-            void* q = realloc(p, c * sizeof(int32_t));
+            void* q = realloc(p, c * sizeof(G));
             if (!q) return false;
-            p = static_cast<int32_t*>(q);
+            p = static_cast<G*>(q);
             cap = c;
             return true;
         }
@@ -227,14 +229,14 @@ bool build_bottom_up(Tables& T, const Options& opt) {
         return r;
     };
     {
-        std::vector<int32_t> g0(D[0].size());
+        std::vector<G> g0(D[0].size());
         for (size_t i = 0; i < D[0].size(); i++) {
             int32_t nx = dfa_next(T, D[0][i], 0);
-            g0[i] = nx < 0 ? -nx - 1 : T.dfa_mask[nx];
+            g0[i] = (G)(nx < 0 ? -nx - 1 : T.dfa_mask[nx]);
         }
         new_state(0, hash_state(0, g0.data(), g0.size()));
         if (!arena.grow(arena.n)) return false;
-        std::memcpy(arena.p, g0.data(), g0.size() * 4);
+        std::memcpy(arena.p, g0.data(), g0.size() * sizeof(G));
     }
     double t_par = 0, t_ser = 0;
     int n_batches = 0;
@@ -246,7 +248,7 @@ bool build_bottom_up(Tables& T, const Options& opt) {
         int32_t found;
     };
     std::vector<Cand> cands;
-    std::vector<int32_t> buf;
+    std::vector<G> buf;
     std::vector<std::pair<int32_t, int64_t>> fresh;   // (new state, its vector's offset in buf)
     const int64_t batch_bytes = std::min<int64_t>(budget / 8, int64_t(256) << 20);
     while (!frontier.empty()) {
@@ -271,20 +273,20 @@ bool build_bottom_up(Tables& T, const Options& opt) {
             parallel_for(threads, cands.size(), [&](size_t ci) {
                 Cand& c = cands[ci];
                 int t = st_t[c.from];
-                const int32_t* g = arena.p + g_off[c.from];
+                const G* g = arena.p + g_off[c.from];
                 int pi = pred_index(c.u, t);
                 const int32_t* sp = step[c.u].data() + step_off[c.u][pi];
-                int32_t* out = buf.data() + c.off;
+                G* out = buf.data() + c.off;
                 size_t m = D[c.u].size();
                 for (size_t j = 0; j < m; j++) {
                     int32_t x = sp[j];
-                    out[j] = x < 0 ? -x - 1 : g[x];
+                    out[j] = x < 0 ? (G)(-x - 1) : g[x];
                 }
                 c.h = hash_state(c.u, out, m);
                 auto range = index.equal_range(c.h);   // read-only while the batch runs
                 for (auto it = range.first; it != range.second; ++it) {
                     int32_t r = it->second;
-                    if (st_t[r] == c.u && !memcmp(arena.p + g_off[r], out, m * 4)) {
+                    if (st_t[r] == c.u && !memcmp(arena.p + g_off[r], out, m * sizeof(G))) {
                         c.found = r;
                         break;
                     }
@@ -303,7 +305,8 @@ bool build_bottom_up(Tables& T, const Options& opt) {
                     for (auto it = range.first; it != range.second && r < 0; ++it) {
                         int32_t x = it->second;
                         if (x < first_new || st_t[x] != c.u) continue;   // older states were checked above
-                        if (!memcmp(buf.data() + fresh[x - first_new].second, buf.data() + c.off, m * 4)) r = x;
+                        if (!memcmp(buf.data() + fresh[x - first_new].second, buf.data() + c.off, m * sizeof(G)))
+                            r = x;
                     }
                     if (r < 0) {
                         r = new_state(c.u, c.h);
@@ -313,12 +316,18 @@ bool build_bottom_up(Tables& T, const Options& opt) {
                 }
                 tr[tr_off[c.from] + c.k] = r;
             }
-            if ((int64_t)arena.n * 4 + (int64_t)tr.size() * 4 + step_bytes > budget ||
-                (int64_t)st_t.size() > opt.max_states || !arena.grow(arena.n))
+            if ((int64_t)(arena.n * sizeof(G)) + (int64_t)tr.size() * 4 + step_bytes > budget ||
+                (int64_t)st_t.size() > opt.max_states || !arena.grow(arena.n)) {
+                if (log)
+                    fprintf(stderr, "psc: bottom-up classifier given up at %zu states, %.2f GiB of %.2f GiB\n",
+                            st_t.size(),
+                            ((double)arena.n * sizeof(G) + (double)tr.size() * 4 + (double)step_bytes) / (1 << 30),
+                            (double)budget / (1 << 30));
                 return false;
+            }
             parallel_for(threads, fresh.size(), [&](size_t i) {
                 int32_t r = fresh[i].first;
-                std::memcpy(arena.p + g_off[r], buf.data() + fresh[i].second, D[st_t[r]].size() * 4);
+                std::memcpy(arena.p + g_off[r], buf.data() + fresh[i].second, D[st_t[r]].size() * sizeof(G));
             });
             t_ser += seconds() - tp;
             n_batches++;
@@ -337,7 +346,7 @@ bool build_bottom_up(Tables& T, const Options& opt) {
         std::vector<int32_t> row(nq);
         for (int32_t r = 0; r < R; r++) {
             int t = st_t[r];
-            const int32_t* g = arena.p + g_off[r];
+            const G* g = arena.p + g_off[r];
             for (int q = 0; q < nq; q++) {
                 int32_t s = T.dfa_start[q];
                 row[q] = s < 0 ? -s - 1 : g[rank(t, s)];
@@ -382,10 +391,12 @@ bool build_bottom_up(Tables& T, const Options& opt) {
         fprintf(stderr, "psc: bottom-up classifier: %d states, %d final rows, %.2f GiB of construction vectors; "
                         "domains %.2f s, steps %.2f s, states %.2f s (%d batches: parallel %.2f s, serial %.2f s), "
                         "final %.2f s\n",
-                R, T.n_frow, ((double)arena.n * 4 + (double)tr.size() * 4 + (double)step_bytes) / (1 << 30),
+                R, T.n_frow, ((double)arena.n * sizeof(G) + (double)tr.size() * 4 + (double)step_bytes) / (1 << 30),
                 t1 - t0, t2 - t1, t3 - t2, n_batches, t_par, t_ser, seconds() - t3);
     return true;
 }
+
+}  // namespace
 
 int classify_host_bottom_up(const Tables& t, int q, const uint16_t* stack, int depth, int status) {
     if (status == 1) return 1;
@@ -400,6 +411,10 @@ int classify_host_bottom_up(const Tables& t, int q, const uint16_t* stack, int d
         e = t.bu[(size_t)e + 1 + k];
     }
     return t.bu_F[(size_t)t.bu[(size_t)e] * t.nq + q];
+}
+
+bool build_bottom_up(Tables& T, const Options& opt) {
+    return T.n_masks < 65536 ? build_bottom_up_g<uint16_t>(T, opt) : build_bottom_up_g<int32_t>(T, opt);
 }
 
 }  // namespace psc
