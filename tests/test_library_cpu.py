@@ -316,7 +316,7 @@ def test_host_tables_exhaustive_small_configurations(psc, which):
             assert h.host_advance(c, v, cap=64)["status"] == want_status[st], (c, v)
 
 
-@pytest.mark.parametrize("cfg_id", [1, 2, 3, 4])
+@pytest.mark.parametrize("cfg_id", [1, 2, 3, 4, 6, 8])
 def test_host_tables_on_sentences_and_mutations(psc, cfg_id):
     """Whole sentences of each workload grammar and copies with one byte
     inserted, deleted or replaced, fed byte by byte (a vocabulary of the 256
@@ -327,7 +327,7 @@ def test_host_tables_on_sentences_and_mutations(psc, cfg_id):
     spec = configs.grammar_spec(cfg_id)
     text = spec.text()
     vocab = [bytes([b]) for b in range(256)] + [b""]
-    h = psc.psc_compile(text, vocab, 256, host_only=True)
+    h = psc.psc_compile(text, vocab, 256, host_only=True, bottom_up=False, **configs.COMPILE_LIMITS.get(cfg_id, {}))
     o = Oracle(text)
     want_status = {ST_OK: psc.ROW_OK, ST_DONE: psc.ROW_DONE, ST_ERROR: psc.ROW_REJECTED}
     rng = np.random.default_rng([cfg_id, 11])
@@ -363,6 +363,42 @@ def test_host_tables_on_sentences_and_mutations(psc, cfg_id):
         stopped += st != ST_DONE
         n += 1
     assert n == 60 and stopped > 10
+
+
+@pytest.mark.parametrize("cfg_id", [6, 8])
+def test_host_masks_of_the_java_and_sql_grammars(psc, cfg_id):
+    """The Java-sized and SQL-like grammars with a 512-token vocabulary of their
+    workload's recipe: at every 7th token of sampled sentences, the mask the
+    compiled tables give (host classification, host mask rows) equals the
+    oracle's over every token, and so does the bottom-up classification."""
+    from workloads.sample import SentenceSampler, TrieTokenizer
+    spec = configs.grammar_spec(cfg_id)
+    text = spec.text()
+    toks = configs.vocab_for(cfg_id, 512)
+    eos = len(toks) - 1
+    h = psc.psc_compile(text, toks, eos, host_only=True, **configs.COMPILE_LIMITS.get(cfg_id, {}))
+    o = Oracle(text)
+    voc = Vocab.from_list(toks, eos)
+    tok = TrieTokenizer(toks)
+    rng = np.random.default_rng([cfg_id, 12])
+    sampler = SentenceSampler(spec, max_depth=12)
+    cfgs, ocs = [], []
+    while len(cfgs) < 120:
+        txt, _ = sampler.text(rng, 1500)
+        c, oc = h.host_initial(), o.initial()
+        for i, v in enumerate(tok.encode(txt)):
+            c = h.host_advance(c, v, cap=1024)
+            assert o.advance(oc, toks[v]) == ST_OK and c["status"] == psc.ROW_OK
+            if i % 7 == 6:
+                cfgs.append(dict(c))
+                ocs.append(oc.copy())
+    want = o.masks(ocs, voc, threads=os.cpu_count() or 1)
+    for c, m in zip(cfgs, want):
+        mid = h.host_classify(c["q"], c["stack"])
+        np.testing.assert_array_equal(h.host_mask_row(mid), m)
+        if h.info().bottom_up_states:
+            assert h.host_classify_bottom_up(c["q"], c["stack"]) == mid
+    assert len({bytes(m) for m in want}) > 10   # the configurations are not all alike
 
 
 def test_host_tables_terminal_rank(psc):
