@@ -420,7 +420,7 @@ def test_grammar_errors():
 
 
 # ---------------------------------------------------------------- invariants
-@pytest.mark.parametrize("cfg_id", [1, 2, 3])
+@pytest.mark.parametrize("cfg_id", [1, 2, 3, 6, 8])
 def test_invariants_on_workloads(cfg_id):
     w = configs.load(cfg_id, batch=8)
     o = Oracle(w.grammar_text)
@@ -449,7 +449,7 @@ def test_invariants_on_workloads(cfg_id):
     assert np.array_equal(m2, m[perm])                 # rows are independent
 
 
-@pytest.mark.parametrize("cfg_id", [1, 2, 3])
+@pytest.mark.parametrize("cfg_id", [1, 2, 3, 6, 8])
 def test_tokenwise_equals_bytewise(cfg_id):
     """The configuration (q, alpha) is a function of the bytes consumed (Section
     3.2): a prefix advanced token by token and byte by byte reaches the same
