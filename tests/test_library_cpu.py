@@ -634,6 +634,13 @@ def test_packed_advance_tables(psc):
                            global_tables=True).info().advance_table_bytes == 0
     with pytest.raises(ValueError):
         psc.psc_compile(w.grammar_text, w.vocab, w.eos_id, host_only=True, global_tables=True, packed_tables=True)
+    import tempfile
+    with tempfile.TemporaryDirectory() as d:   # the placement is chosen again when tables are loaded
+        path = os.path.join(d, "t.psc")
+        psc.psc_save(psc.psc_compile(w.grammar_text, w.vocab, w.eos_id, host_only=True), path)
+        assert psc.psc_load(path, host_only=True).info().advance_tables_packed == 0
+        assert psc.psc_load(path, host_only=True, packed_tables=True).info().advance_tables_packed == 1
+        assert psc.psc_load(path, host_only=True, global_tables=True).info().advance_table_bytes == 0
     rng = np.random.default_rng(5150)
     modes, multi = set(), 0
     done = 0
